@@ -1,0 +1,83 @@
+"""The pins must catch plausible mistakes in the oracle.
+
+Each mutant below is a one-line textual change to a temporary copy of
+oracle/bkv_oracle.c (a dropped term, a flipped sign, a wrong index or
+aggregation, a transposed pairing).  The copy is compiled on the CPU and the
+pin tests of tests/test_oracle_*.py are run against it: at least one must fail
+for every mutant.  The committed oracle itself is never modified.
+"""
+import os
+import shutil
+import subprocess
+import tempfile
+
+import pytest
+
+from oracle import oracle as O
+from tests import test_oracle_beacons as TB
+from tests import test_oracle_numerics as TN
+from tests import test_oracle_score_select as TS
+
+SRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "oracle", "bkv_oracle.c")
+
+_SCORE = [(TS.test_score_matches_scipy_softmax_max, dict(M=3, L=50, d=8)),
+          (TS.test_score_two_key_logistic_closed_form, {}), (TS.test_golden_worked_case, {}),
+          (TS.test_score_single_query_sums_to_one_and_ranks_by_dot, {})]
+_ROPE = [(TN.test_rope_is_complex_rotation_of_rotate_half_pairs, {}),
+         (TN.test_rope_preserves_norm_and_relative_position, {})]
+_FPS = [(TB.test_fps_matches_maxmin_brute_force, dict(seed=s)) for s in range(6)] + [
+    (TB.test_fps_orthonormal_basis_ties_go_to_lowest_index, {}), (TB.test_fps_outlier_first, {})]
+_UPD = [(TB.test_update_planted_assignment_uses_cosine_not_dot, {}),
+        (TB.test_update_single_beacon_is_global_mean, {}), (TB.test_update_centroid_is_mean_of_assigned, {})]
+_SEL = [(TS.test_select_matches_lexsort_and_invariants, dict(L=130, budget=100, W=8, npre=3)),
+        (TS.test_select_all_ties_take_lowest_indices, {})]
+
+MUTANTS = [
+    ("drop_inv_sqrt_d", "* inv_sqrt_d;", "* 1.0;", _SCORE),
+    ("no_max_shift_in_lse", "double lse = m + log(s);", "double lse = log(s);", _SCORE),
+    ("mean_instead_of_max", "if (w > score[j]) score[j] = w;", "score[j] = score[j] + w / M;", _SCORE),
+    ("rope_sign", "y[i] = x1 * cs - x2 * sn;", "y[i] = x1 * cs + x2 * sn;", _ROPE),
+    ("rope_interleaved_pairs", "double x1 = x[i], x2 = x[i + h];", "double x1 = x[2 * i], x2 = x[2 * i + 1];",
+     _ROPE),
+    ("rope_frequency_exponent", "-(double)(2 * i) / (double)d", "-(double)(i) / (double)d", _ROPE),
+    ("fps_min_update", "if (c > S[j]) S[j] = c;", "if (c < S[j]) S[j] = c;", _FPS),
+    ("fps_first_pick_argmax", "if (avg < best) {", "if (-avg < best) {", _FPS),
+    ("assign_by_dot_product", "double cs = cosine(qn, c + (size_t)b * d, d, NULL);",
+     "double cs = dot_seq(qn, c + (size_t)b * d, d);", _UPD),
+    ("centroid_forgets_history", "sums[(size_t)b * d + i] = sums[(size_t)b * d + i] + x[(size_t)n * d + i];",
+     "sums[(size_t)b * d + i] = x[(size_t)n * d + i];", _UPD),
+    ("tie_break_high_index", "return (x->j < y->j) ? -1 : (x->j > y->j);",
+     "return (x->j > y->j) ? -1 : (x->j < y->j);", _SEL),
+    ("window_off_by_one", "for (int j = L - W; j < L; ++j) kept[n_keep++] = j;",
+     "for (int j = L - W - 1; j < L - 1; ++j) kept[n_keep++] = j;", _SEL),
+    ("bf16_round_half_up", "u += 0x7fffu + lsb;", "u += 0x8000u;",
+     [(TN.test_bf16_known_patterns, {}), (TN.test_bf16_matches_torch_on_random_floats, {})]),
+    ("gather_wrong_row", "memcpy(tk + (size_t)i * d, K + (size_t)kept[i] * d, row);",
+     "memcpy(tk + (size_t)i * d, K + (size_t)i * d, row);", [(TS.test_gather_is_row_indexing, {})]),
+]
+
+
+@pytest.fixture(scope="module")
+def workdir():
+    d = tempfile.mkdtemp(prefix="bkv_mutants_")
+    yield d
+    shutil.rmtree(d, ignore_errors=True)
+
+
+@pytest.mark.parametrize("name,old,new,checks", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_pins_catch_mutant(workdir, name, old, new, checks):
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"mutation anchor for {name} not unique"
+    path_c = os.path.join(workdir, f"{name}.c")
+    path_so = os.path.join(workdir, f"lib{name}.so")
+    with open(path_c, "w") as f:
+        f.write(src.replace(old, new))
+    subprocess.check_call(["gcc", *O.CFLAGS, "-o", path_so, path_c, "-lm"])
+    lib = O.load(path_so)
+    failed = []
+    for fn, kw in checks:
+        try:
+            fn(lib, **kw)
+        except Exception as exc:  # noqa: BLE001 - any failure counts as a catch
+            failed.append((fn.__name__, type(exc).__name__))
+    assert failed, f"no pin caught mutant {name}"
