@@ -1,0 +1,203 @@
+/*
+ * bkv.h - C ABI of the BeaconKV KV-cache compression step on GB300 (sm_103a).
+ *
+ * BeaconKV (arXiv 2609.04971) keeps a KV cache within budget by scoring every
+ * cached key with the attention weights of a set of observation queries -
+ * "beacon" queries that represent recurring global query clusters plus the
+ * most recent queries - and keeping the best keys together with the recent
+ * window (Sections 4.1-4.3, Appendix D.2).  This library implements the two
+ * data-parallel parts of that step for a whole model (all layers, batch rows
+ * and KV heads at once):
+ *
+ *   beacon maintenance  - FPS seeding from prompt queries (Appendix D.1,
+ *                         Algorithm 1) and, per decode query, nearest-beacon
+ *                         assignment by cosine similarity followed by a
+ *                         running-mean centroid update;
+ *   compression         - observation queries (beacons rotated to the current
+ *                         step, recent queries at their own positions;
+ *                         Section 4.3), scoring (Eq. 4 softmax over the whole
+ *                         cache, Eq. 6 max form, maximum over the GQA group),
+ *                         selection (keep set + TopK, Eq. 7, Algorithm 2) and
+ *                         in-place compaction of K and V (Eq. 8).
+ *
+ * Terms.  An *instance* is one (layer, batch row, KV head).  G = n_q_heads /
+ * n_kv_heads query heads share a KV head; their queries all feed that KV
+ * head's beacons.  n_inst = n_layers * batch * n_kv_heads.  Instances are
+ * numbered (layer * batch + b) * n_kv_heads + g, which is also the row order
+ * of every per-instance array below.
+ *
+ * Memory.  Every tensor argument is a DEVICE pointer owned by the caller,
+ * row-major and contiguous, aligned to 16 bytes, unless the description says
+ * "host".  bf16 tensors hold IEEE binary32 values truncated to their top 16
+ * bits (bfloat16).  The library owns only what bkv_create allocates (beacon
+ * state and scratch) and frees it in bkv_destroy.
+ *
+ * Streams.  All work is enqueued on the CUDA stream given to bkv_create (or
+ * bkv_set_stream); calls return before it completes.  Outputs are valid once
+ * that stream has been synchronised (bkv_sync does so and reports device-side
+ * errors).  One context must not be used from two host threads at once.
+ *
+ * Errors.  Every call returns BKV_OK (0) or a negative code; nothing throws.
+ * Argument errors are detected on the host before any work is enqueued and
+ * leave all buffers untouched.  Kernels whose internal waits expire record
+ * BKV_ETIMEOUT in a device error word that the next bkv_sync returns.
+ * bkv_last_error(ctx) gives a one-line description of the last failure.
+ */
+#ifndef BKV_H
+#define BKV_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define BKV_OK 0
+#define BKV_EINVAL (-1)   /* bad shape, size, alignment, null pointer or range   */
+#define BKV_ENOMEM (-2)   /* device allocation failed                            */
+#define BKV_ECUDA (-3)    /* a CUDA runtime / driver call failed                 */
+#define BKV_ETIMEOUT (-4) /* a bounded device-side wait expired (kernel aborted) */
+#define BKV_ESTATE (-5)   /* call order violated (e.g. update before init)       */
+
+/* bkv_config.flags: no option is defined yet; pass 0. */
+#define BKV_F_NONE 0u
+
+typedef struct bkv_ctx bkv_ctx;
+
+/*
+ * Model / cache shape, fixed for the life of a context.
+ *   head_dim    64 or 128.
+ *   n_beacons   beacons per KV head, 0..32 (0 = recent queries only).
+ *   window      recent queries per query head kept for scoring AND number of
+ *               most recent cache rows that are always kept, 0..64.
+ *   n_prefix    number of leading cache rows that are always kept (>= 0).
+ *   capacity    rows allocated per instance in K and V (1..32768).
+ *   rope_theta  rotary base; 0 disables rotation.
+ * Limits: G * window + n_beacons must be in 1..128.
+ */
+typedef struct {
+  int32_t n_layers, batch, n_q_heads, n_kv_heads, head_dim;
+  int32_t n_beacons, window, n_prefix;
+  int32_t capacity;
+  double rope_theta;
+  uint32_t flags; /* reserved, must be 0 */
+} bkv_config;
+
+/*
+ * Creates a context on the current CUDA device and allocates its beacon state
+ * (fp32 centroids, fp64 sums, int64 counts; all zero, i.e. no beacon yet) and
+ * scratch.  `stream` is a cudaStream_t (NULL = legacy default stream).
+ * Returns BKV_EINVAL for a bad config, BKV_ENOMEM / BKV_ECUDA on failure.
+ */
+int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out);
+
+/* Frees everything the context owns (after synchronising its stream). NULL is ignored. */
+void bkv_destroy(bkv_ctx* ctx);
+
+/* Changes the stream used by later calls. */
+int bkv_set_stream(bkv_ctx* ctx, void* stream);
+
+/*
+ * Prefill seeding (Appendix D.2: FPS over the prompt's pre-RoPE queries;
+ * Algorithm 1).  For every instance, FPS runs over the G * n_init queries of
+ * its group (head-major order h * n_init + i, cosine similarity, ties to the
+ * lowest index) and beacon k becomes the k-th selected query with count 1.
+ *   q_init  bf16 [n_layers][batch][n_q_heads][n_init][head_dim], pre-RoPE.
+ * Requires G * n_init >= n_beacons and G * n_init <= 4096.
+ * Replaces any previous beacon state.
+ */
+int bkv_init_beacons(bkv_ctx* ctx, const void* q_init, int32_t n_init);
+
+/*
+ * Beacon maintenance for n_new decode queries per query head.  Each query q
+ * is assigned to argmax_b cos(q, c_b) over the beacons with count > 0 and a
+ * non-zero centroid, using the centroids as they were when the call started
+ * (ties go to the lowest b; a zero query is skipped).  Then for each beacon
+ * sums_b += sum of its assigned queries (exact), counts_b += their number and
+ * c_b = fp32(sums_b / counts_b).
+ *   q_new       bf16 [n_layers][batch][n_q_heads][n_new][head_dim], pre-RoPE.
+ *   assign_out  int32 [n_layers][batch][n_q_heads][n_new] or NULL: the beacon
+ *               chosen for each query, -1 when it was skipped.
+ * n_new == 0 is a no-op.  BKV_ESTATE if bkv_init_beacons / bkv_set_state was
+ * never called.
+ */
+int bkv_update_beacons(bkv_ctx* ctx, const void* q_new, int32_t n_new, int32_t* assign_out);
+
+/*
+ * One compression of every instance's cache from L rows to `budget` rows.
+ * Observation queries (Section 4.3): for each instance, the recent queries of
+ * its G query heads, query (h, w) rotated to position recent_pos[w], and its
+ * beacons with count > 0 rotated to t_pos; each is rounded to bf16 after the
+ * rotation.  Score[j] = max over those queries of the softmax weight of key
+ * j over all L cached keys (Eq. 4, Eq. 6 max form; logits q.k / sqrt(d)).
+ * Kept rows = [0, n_prefix) U [L - window, L) U the (budget - n_prefix -
+ * window) other rows with the largest Score (ties to the lower index), in
+ * ascending order (Eq. 7, Algorithm 2).  Row i of K and V then holds what row
+ * kept[i] held (Eq. 8); rows >= budget are left unspecified.
+ *   K, V          bf16 [n_layers][batch][n_kv_heads][capacity][head_dim]; rows
+ *                 [0, L) are read, rows [0, budget) rewritten in place.  Keys
+ *                 are taken as already rotated (post-RoPE).
+ *   L             current rows per instance, 1..capacity.
+ *   budget        rows to keep, >= n_prefix + window.  L <= budget: nothing
+ *                 is evicted, K/V are not touched and kept_idx_out[i] = i for
+ *                 i < L, -1 for L <= i < budget.
+ *   t_pos         absolute position of the current decode step (beacons).
+ *   q_recent      bf16 [n_layers][batch][n_q_heads][window][head_dim], pre-RoPE.
+ *   recent_pos    HOST int64 [window]: absolute position of recent slot w.
+ *   kept_idx_out  int32 [n_layers][batch][n_kv_heads][budget].
+ *   scores_out    fp32 [n_layers][batch][n_kv_heads][capacity] or NULL:
+ *                 Score[j] for j < L (only written when L > budget).
+ * BKV_ESTATE if n_beacons > 0 and no beacon state was set.
+ */
+int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int64_t t_pos,
+                 const void* q_recent, const int64_t* recent_pos, int32_t* kept_idx_out, float* scores_out);
+
+/*
+ * Copies the beacon state to / from caller DEVICE buffers:
+ *   centroids fp32 [n_inst][n_beacons][head_dim]
+ *   sums      fp64 [n_inst][n_beacons][head_dim]
+ *   counts    int64 [n_inst][n_beacons]
+ * Any pointer may be NULL to skip that array (get only).  bkv_set_state
+ * needs all three and marks the state as initialised (checkpoint / resume).
+ */
+int bkv_get_state(bkv_ctx* ctx, float* centroids, double* sums, int64_t* counts);
+int bkv_set_state(bkv_ctx* ctx, const float* centroids, const double* sums, const int64_t* counts);
+
+/*
+ * Waits for the context's stream, then reads and clears the device error
+ * word.  Returns BKV_OK, BKV_ETIMEOUT (a kernel gave up a bounded wait and
+ * its outputs are invalid) or BKV_ECUDA.
+ */
+int bkv_sync(bkv_ctx* ctx);
+
+/*
+ * Per-kernel timing (tracing).  While enabled, every kernel launch made by
+ * this context is bracketed by CUDA events on the context's stream.
+ * bkv_profile_read synchronises the stream, then writes for each kernel k
+ * (BKV_K_* below, n_kernels entries at most) the summed device time in
+ * milliseconds (ms[k]) and the number of launches (launches[k]) since the
+ * previous read, and resets the totals.  Either output may be NULL.
+ */
+#define BKV_K_FPS 0
+#define BKV_K_UPDATE 1
+#define BKV_K_QOBS 2
+#define BKV_K_SCORE 3
+#define BKV_K_SELECT_GATHER 4
+#define BKV_K_KEEP_ALL 5
+#define BKV_NUM_KERNELS 6
+int bkv_profile_enable(bkv_ctx* ctx, int on);
+int bkv_profile_read(bkv_ctx* ctx, double* ms, int64_t* launches, int32_t n_kernels);
+
+/* Static description of an error code. */
+const char* bkv_strerror(int code);
+
+/* One-line description of the last error on this context ("" if none). */
+const char* bkv_last_error(const bkv_ctx* ctx);
+
+/* Version string of the library build. */
+const char* bkv_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* BKV_H */

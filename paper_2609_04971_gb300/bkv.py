@@ -1,0 +1,252 @@
+"""Python binding of the C ABI in include/bkv.h (argument marshalling only).
+
+Each ``bkv_*`` function has the C function's name and meaning; tensors are
+torch tensors whose device pointers are handed to the library, and the CUDA
+stream defaults to torch's current stream.  Nothing here computes: every step
+of the method runs in libbkv.so, and this module raises if the library cannot
+be loaded (there is no other implementation to fall back on).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import _build
+
+BKV_OK = 0
+BKV_EINVAL = -1
+BKV_ENOMEM = -2
+BKV_ECUDA = -3
+BKV_ETIMEOUT = -4
+BKV_ESTATE = -5
+
+KERNEL_NAMES = ("fps_init", "update", "qobs", "score", "select_gather", "keep_all")
+
+
+class BkvConfig(ctypes.Structure):
+    _fields_ = [
+        ("n_layers", ctypes.c_int32), ("batch", ctypes.c_int32), ("n_q_heads", ctypes.c_int32),
+        ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("n_beacons", ctypes.c_int32),
+        ("window", ctypes.c_int32), ("n_prefix", ctypes.c_int32), ("capacity", ctypes.c_int32),
+        ("rope_theta", ctypes.c_double), ("flags", ctypes.c_uint32),
+    ]
+
+
+class BkvError(RuntimeError):
+    def __init__(self, code: int, where: str, detail: str = ""):
+        self.code = code
+        super().__init__(f"{where}: {bkv_strerror(code)} ({code})" + (f": {detail}" if detail else ""))
+
+
+_lib = None
+_lock = threading.Lock()
+_P = ctypes.c_void_p
+
+
+def load_library(path: str | None = None, build: bool = True):
+    """Load libbkv.so (building it in-tree first if it is missing or stale)."""
+    global _lib
+    with _lock:
+        if _lib is not None and path is None:
+            return _lib
+        p = path or (_build.build() if build else _build.LIB_PATH)
+        if not os.path.exists(p):
+            raise RuntimeError(f"libbkv.so not found at {p}; run __graft_entry__.build()")
+        lib = ctypes.CDLL(p)
+        sig = {
+            "bkv_create": (ctypes.c_int, [ctypes.POINTER(BkvConfig), _P, ctypes.POINTER(_P)]),
+            "bkv_destroy": (None, [_P]),
+            "bkv_set_stream": (ctypes.c_int, [_P, _P]),
+            "bkv_init_beacons": (ctypes.c_int, [_P, _P, ctypes.c_int32]),
+            "bkv_update_beacons": (ctypes.c_int, [_P, _P, ctypes.c_int32, _P]),
+            "bkv_compress": (ctypes.c_int, [_P, _P, _P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, _P, _P,
+                                            _P, _P]),
+            "bkv_get_state": (ctypes.c_int, [_P, _P, _P, _P]),
+            "bkv_set_state": (ctypes.c_int, [_P, _P, _P, _P]),
+            "bkv_sync": (ctypes.c_int, [_P]),
+            "bkv_profile_enable": (ctypes.c_int, [_P, ctypes.c_int]),
+            "bkv_profile_read": (ctypes.c_int, [_P, _P, _P, ctypes.c_int32]),
+            "bkv_strerror": (ctypes.c_char_p, [ctypes.c_int]),
+            "bkv_last_error": (ctypes.c_char_p, [_P]),
+            "bkv_version": (ctypes.c_char_p, []),
+        }
+        for name, (res, args) in sig.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        if path is None:
+            _lib = lib
+        return lib
+
+
+def _l():
+    return _lib if _lib is not None else load_library()
+
+
+def _ptr(t: torch.Tensor | None, dtype: torch.dtype, name: str, device=None):
+    if t is None:
+        return None
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        if not torch.cuda.is_available():
+            return ctypes.c_void_p(0)
+        stream = torch.cuda.current_stream()
+    handle = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+    return ctypes.c_void_p(handle)
+
+
+def _check(rc: int, where: str, ctx=None) -> None:
+    if rc != BKV_OK:
+        detail = _l().bkv_last_error(ctx).decode() if ctx is not None else ""
+        raise BkvError(rc, where, detail)
+
+
+# ---------------------------------------------------------------- C-ABI mirror
+def bkv_version() -> str:
+    return _l().bkv_version().decode()
+
+
+def bkv_strerror(code: int) -> str:
+    return _l().bkv_strerror(int(code)).decode()
+
+
+def bkv_last_error(ctx) -> str:
+    return _l().bkv_last_error(ctx).decode()
+
+
+def bkv_create(cfg: BkvConfig, stream=None) -> ctypes.c_void_p:
+    out = ctypes.c_void_p()
+    _check(_l().bkv_create(ctypes.byref(cfg), _stream(stream), ctypes.byref(out)), "bkv_create")
+    return out
+
+
+def bkv_destroy(ctx) -> None:
+    if ctx:
+        _l().bkv_destroy(ctx)
+
+
+def bkv_set_stream(ctx, stream=None) -> None:
+    _check(_l().bkv_set_stream(ctx, _stream(stream)), "bkv_set_stream", ctx)
+
+
+def bkv_init_beacons(ctx, q_init: torch.Tensor, n_init: int) -> None:
+    _check(_l().bkv_init_beacons(ctx, _ptr(q_init, torch.bfloat16, "q_init"), int(n_init)), "bkv_init_beacons", ctx)
+
+
+def bkv_update_beacons(ctx, q_new: torch.Tensor, n_new: int, assign_out: torch.Tensor | None = None) -> None:
+    _check(_l().bkv_update_beacons(ctx, _ptr(q_new, torch.bfloat16, "q_new"), int(n_new),
+                                   _ptr(assign_out, torch.int32, "assign_out")), "bkv_update_beacons", ctx)
+
+
+def bkv_compress(ctx, K: torch.Tensor, V: torch.Tensor, L: int, budget: int, t_pos: int,
+                 q_recent: torch.Tensor | None, recent_pos, kept_idx_out: torch.Tensor,
+                 scores_out: torch.Tensor | None = None) -> None:
+    pos = (ctypes.c_int64 * max(1, len(recent_pos)))(*[int(p) for p in recent_pos])
+    _check(_l().bkv_compress(ctx, _ptr(K, torch.bfloat16, "K"), _ptr(V, torch.bfloat16, "V"), int(L), int(budget),
+                             int(t_pos), _ptr(q_recent, torch.bfloat16, "q_recent"), ctypes.cast(pos, _P),
+                             _ptr(kept_idx_out, torch.int32, "kept_idx_out"),
+                             _ptr(scores_out, torch.float32, "scores_out")), "bkv_compress", ctx)
+
+
+def bkv_get_state(ctx, centroids=None, sums=None, counts=None) -> None:
+    _check(_l().bkv_get_state(ctx, _ptr(centroids, torch.float32, "centroids"), _ptr(sums, torch.float64, "sums"),
+                              _ptr(counts, torch.int64, "counts")), "bkv_get_state", ctx)
+
+
+def bkv_set_state(ctx, centroids, sums, counts) -> None:
+    _check(_l().bkv_set_state(ctx, _ptr(centroids, torch.float32, "centroids"), _ptr(sums, torch.float64, "sums"),
+                              _ptr(counts, torch.int64, "counts")), "bkv_set_state", ctx)
+
+
+def bkv_sync(ctx) -> None:
+    _check(_l().bkv_sync(ctx), "bkv_sync", ctx)
+
+
+def bkv_profile_enable(ctx, on: bool = True) -> None:
+    _check(_l().bkv_profile_enable(ctx, int(bool(on))), "bkv_profile_enable", ctx)
+
+
+def bkv_profile_read(ctx) -> dict:
+    """{kernel name: (total ms, launches)} since the previous read (syncs the stream)."""
+    n = len(KERNEL_NAMES)
+    ms = (ctypes.c_double * n)()
+    cnt = (ctypes.c_int64 * n)()
+    _check(_l().bkv_profile_read(ctx, ctypes.cast(ms, _P), ctypes.cast(cnt, _P), n), "bkv_profile_read", ctx)
+    return {KERNEL_NAMES[k]: (ms[k], cnt[k]) for k in range(n)}
+
+
+# ---------------------------------------------------------------- convenience
+class BeaconKV:
+    """Owns one context for a model shape and allocates outputs with torch.
+
+    Example::
+        bk = BeaconKV(n_layers=36, batch=16, n_q_heads=32, n_kv_heads=8, head_dim=128,
+                      n_beacons=8, window=8, capacity=4224, rope_theta=1e6)
+        bk.init_beacons(q_init)                       # [L, B, Hq, n_init, d] bf16
+        bk.update(q_new)                              # [L, B, Hq, n_new, d] bf16
+        kept = bk.compress(K, V, L=4224, budget=4096, t_pos=4223, q_recent=q, recent_pos=[...])
+    """
+
+    def __init__(self, *, n_layers, batch, n_q_heads, n_kv_heads, head_dim, n_beacons, window, capacity,
+                 rope_theta=0.0, n_prefix=0, stream=None):
+        self.cfg = BkvConfig(n_layers, batch, n_q_heads, n_kv_heads, head_dim, n_beacons, window, n_prefix,
+                             capacity, float(rope_theta), 0)
+        self.ctx = bkv_create(self.cfg, stream)
+        self.n_inst = n_layers * batch * n_kv_heads
+
+    @classmethod
+    def for_workload(cls, wl, stream=None, capacity=None) -> "BeaconKV":
+        return cls(n_layers=wl.n_layers, batch=wl.batch, n_q_heads=wl.n_q_heads, n_kv_heads=wl.n_kv_heads,
+                   head_dim=wl.head_dim, n_beacons=wl.n_beacons, window=wl.window,
+                   capacity=capacity or wl.capacity, rope_theta=wl.rope_theta, n_prefix=wl.n_prefix, stream=stream)
+
+    def close(self):
+        if self.ctx:
+            bkv_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:  # noqa: BLE001 - interpreter shutdown
+            pass
+
+    def init_beacons(self, q_init: torch.Tensor):
+        bkv_init_beacons(self.ctx, q_init, q_init.shape[-2])
+
+    def update(self, q_new: torch.Tensor, assign_out: torch.Tensor | None = None):
+        bkv_update_beacons(self.ctx, q_new, q_new.shape[-2], assign_out)
+
+    def compress(self, K, V, *, L, budget, t_pos, q_recent, recent_pos, kept_out=None, scores_out=None):
+        c = self.cfg
+        if kept_out is None:
+            kept_out = torch.empty(c.n_layers, c.batch, c.n_kv_heads, budget, dtype=torch.int32, device=K.device)
+        bkv_compress(self.ctx, K, V, L, budget, t_pos, q_recent, recent_pos, kept_out, scores_out)
+        return kept_out
+
+    def state(self):
+        c = self.cfg
+        dev = torch.device("cuda", torch.cuda.current_device())
+        cent = torch.empty(self.n_inst, c.n_beacons, c.head_dim, dtype=torch.float32, device=dev)
+        sums = torch.empty(self.n_inst, c.n_beacons, c.head_dim, dtype=torch.float64, device=dev)
+        counts = torch.empty(self.n_inst, c.n_beacons, dtype=torch.int64, device=dev)
+        bkv_get_state(self.ctx, cent, sums, counts)
+        return cent, sums, counts
+
+    def set_state(self, cent, sums, counts):
+        bkv_set_state(self.ctx, cent, sums, counts)
+
+    def sync(self):
+        bkv_sync(self.ctx)

@@ -1,0 +1,464 @@
+// C ABI of the BeaconKV compression step (declared in include/bkv.h):
+// argument validation, context and scratch ownership, tensor-map encoding,
+// the rotary table, and kernel launches on the context's stream.
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "bkv.h"
+#include "bkv_internal.h"
+
+using bkv::Shape;
+
+struct bkv_ctx {
+  bkv_config cfg{};
+  Shape shape{};
+  cudaStream_t stream = nullptr;
+  int device = 0;
+  // beacon state
+  float* cent = nullptr;
+  double* sums = nullptr;
+  long long* counts = nullptr;
+  bool state_ready = false;
+  // scratch
+  __nv_bfloat16* qobs = nullptr;  // [n_inst][n_obs_pad][d]
+  uint32_t* valid = nullptr;      // [n_inst][4]
+  float* rscore = nullptr;        // [n_inst][cap]
+  double2* rope = nullptr;        // [W + 1][d / 2]
+  int* err = nullptr;             // device error word
+  std::vector<double2> rope_host;
+  std::string last_error;
+  // per-kernel timing
+  struct Rec {
+    cudaEvent_t start, stop;
+    int kernel;
+  };
+  bool prof = false;
+  std::vector<Rec> pending;
+  std::vector<cudaEvent_t> spare;
+  double prof_ms[BKV_NUM_KERNELS] = {};
+  long long prof_n[BKV_NUM_KERNELS] = {};
+};
+
+namespace {
+
+int fail(bkv_ctx* c, int code, const char* fmt, ...) {
+  if (c) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    c->last_error = buf;
+  }
+  return code;
+}
+
+int cuda_fail(bkv_ctx* c, cudaError_t e, const char* what) {
+  return fail(c, BKV_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+cudaEvent_t take_event(bkv_ctx* c) {
+  if (!c->spare.empty()) {
+    cudaEvent_t ev = c->spare.back();
+    c->spare.pop_back();
+    return ev;
+  }
+  cudaEvent_t ev = nullptr;
+  cudaEventCreate(&ev);
+  return ev;
+}
+
+// Brackets one kernel launch with events when timing is enabled.
+struct ProfScope {
+  bkv_ctx* c;
+  int kernel;
+  cudaEvent_t start = nullptr;
+  ProfScope(bkv_ctx* ctx, int k) : c(ctx), kernel(k) {
+    if (c->prof && (start = take_event(c))) cudaEventRecord(start, c->stream);
+  }
+  ~ProfScope() {
+    if (!start) return;
+    cudaEvent_t stop = take_event(c);
+    if (!stop) return;
+    cudaEventRecord(stop, c->stream);
+    c->pending.push_back({start, stop, kernel});
+  }
+};
+
+void fold_profile(bkv_ctx* c) {
+  for (auto& r : c->pending) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, r.start, r.stop) == cudaSuccess) {
+      c->prof_ms[r.kernel] += ms;
+      c->prof_n[r.kernel] += 1;
+    }
+    c->spare.push_back(r.start);
+    c->spare.push_back(r.stop);
+  }
+  c->pending.clear();
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor [rows][d] viewed in boxes of [box_rows][64] with 128-byte swizzle.
+int encode_rows(bkv_ctx* c, CUtensorMap* map, const void* base, uint64_t rows, int d, uint32_t box_rows) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return fail(c, BKV_ECUDA, "cuTensorMapEncodeTiled is unavailable");
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(d) * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(c, BKV_ECUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+  return BKV_OK;
+}
+
+int validate_config(const bkv_config* cfg, std::string& why) {
+  char buf[256];
+  auto bad = [&](const char* m) {
+    why = m;
+    return BKV_EINVAL;
+  };
+  if (!cfg) return bad("config is NULL");
+  if (cfg->n_layers < 1 || cfg->batch < 1 || cfg->n_q_heads < 1 || cfg->n_kv_heads < 1)
+    return bad("n_layers, batch, n_q_heads and n_kv_heads must be >= 1");
+  if (cfg->n_q_heads % cfg->n_kv_heads != 0) return bad("n_q_heads must be a multiple of n_kv_heads");
+  if (cfg->head_dim != 64 && cfg->head_dim != 128) return bad("head_dim must be 64 or 128");
+  if (cfg->n_beacons < 0 || cfg->n_beacons > bkv::kMaxBeacons) return bad("n_beacons must be in 0..32");
+  if (cfg->window < 0 || cfg->window > bkv::kMaxWindow) return bad("window must be in 0..64");
+  if (cfg->n_prefix < 0) return bad("n_prefix must be >= 0");
+  if (cfg->capacity < 1 || cfg->capacity > bkv::kMaxCapacity) return bad("capacity must be in 1..32768");
+  if (!(cfg->rope_theta >= 0.0) || !std::isfinite(cfg->rope_theta)) return bad("rope_theta must be finite and >= 0");
+  if (cfg->flags != 0) return bad("flags must be 0");
+  const long long G = cfg->n_q_heads / cfg->n_kv_heads;
+  const long long n_obs = G * cfg->window + cfg->n_beacons;
+  if (n_obs < 1 || n_obs > bkv::kMaxObs) {
+    snprintf(buf, sizeof buf, "G * window + n_beacons = %lld must be in 1..128", n_obs);
+    why = buf;
+    return BKV_EINVAL;
+  }
+  const long long n_inst = 1LL * cfg->n_layers * cfg->batch * cfg->n_kv_heads;
+  if (n_inst * cfg->capacity >= (1LL << 31) || n_inst * 128 >= (1LL << 31))
+    return bad("n_layers * batch * n_kv_heads * capacity must be below 2^31");
+  return BKV_OK;
+}
+
+template <typename T>
+cudaError_t dmalloc(T** p, size_t n) {
+  return cudaMalloc(reinterpret_cast<void**>(p), sizeof(T) * (n ? n : 1));
+}
+
+void free_all(bkv_ctx* c) {
+  for (auto& r : c->pending) {
+    cudaEventDestroy(r.start);
+    cudaEventDestroy(r.stop);
+  }
+  c->pending.clear();
+  for (auto ev : c->spare) cudaEventDestroy(ev);
+  c->spare.clear();
+  cudaFree(c->cent);
+  cudaFree(c->sums);
+  cudaFree(c->counts);
+  cudaFree(c->qobs);
+  cudaFree(c->valid);
+  cudaFree(c->rscore);
+  cudaFree(c->rope);
+  cudaFree(c->err);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* bkv_version(void) { return "bkv 0.1.0 (sm_103a, tcgen05)"; }
+
+const char* bkv_strerror(int code) {
+  switch (code) {
+    case BKV_OK: return "ok";
+    case BKV_EINVAL: return "invalid argument";
+    case BKV_ENOMEM: return "device allocation failed";
+    case BKV_ECUDA: return "CUDA error";
+    case BKV_ETIMEOUT: return "device wait timed out; outputs are invalid";
+    case BKV_ESTATE: return "beacon state not initialised";
+    default: return "unknown error";
+  }
+}
+
+const char* bkv_last_error(const bkv_ctx* ctx) { return ctx ? ctx->last_error.c_str() : ""; }
+
+int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
+  if (!out) return BKV_EINVAL;
+  *out = nullptr;
+  std::string why;
+  if (validate_config(cfg, why) != BKV_OK) return BKV_EINVAL;
+  auto* c = new (std::nothrow) bkv_ctx();
+  if (!c) return BKV_ENOMEM;
+  c->cfg = *cfg;
+  Shape& s = c->shape;
+  s.G = cfg->n_q_heads / cfg->n_kv_heads;
+  s.n_inst = cfg->n_layers * cfg->batch * cfg->n_kv_heads;
+  s.d = cfg->head_dim;
+  s.nb = cfg->n_beacons;
+  s.W = cfg->window;
+  s.n_prefix = cfg->n_prefix;
+  s.cap = cfg->capacity;
+  s.n_obs = s.G * s.W + s.nb;
+  s.n_obs_pad = (s.n_obs + 15) / 16 * 16;
+  c->stream = static_cast<cudaStream_t>(stream);
+  cudaGetDevice(&c->device);
+
+  const size_t ni = static_cast<size_t>(s.n_inst);
+  cudaError_t e = cudaSuccess;
+  if ((e = dmalloc(&c->cent, ni * s.nb * s.d)) != cudaSuccess ||
+      (e = dmalloc(&c->sums, ni * s.nb * s.d)) != cudaSuccess ||
+      (e = dmalloc(&c->counts, ni * s.nb)) != cudaSuccess ||
+      (e = dmalloc(&c->qobs, ni * s.n_obs_pad * s.d)) != cudaSuccess ||
+      (e = dmalloc(&c->valid, ni * 4)) != cudaSuccess ||
+      (e = dmalloc(&c->rscore, ni * s.cap)) != cudaSuccess ||
+      (e = dmalloc(&c->rope, static_cast<size_t>(s.W + 1) * (s.d / 2))) != cudaSuccess ||
+      (e = dmalloc(&c->err, 1)) != cudaSuccess) {
+    const int code = (e == cudaErrorMemoryAllocation) ? BKV_ENOMEM : BKV_ECUDA;
+    cudaGetLastError();
+    free_all(c);
+    delete c;
+    return code;
+  }
+  if ((e = cudaMemsetAsync(c->cent, 0, sizeof(float) * ni * s.nb * s.d + 0, c->stream)) != cudaSuccess ||
+      (e = cudaMemsetAsync(c->sums, 0, sizeof(double) * ni * s.nb * s.d, c->stream)) != cudaSuccess ||
+      (e = cudaMemsetAsync(c->counts, 0, sizeof(long long) * ni * s.nb, c->stream)) != cudaSuccess ||
+      (e = cudaMemsetAsync(c->err, 0, sizeof(int), c->stream)) != cudaSuccess) {
+    free_all(c);
+    delete c;
+    return BKV_ECUDA;
+  }
+  c->rope_host.resize(static_cast<size_t>(s.W + 1) * (s.d / 2));
+  *out = c;
+  return BKV_OK;
+}
+
+void bkv_destroy(bkv_ctx* ctx) {
+  if (!ctx) return;
+  cudaStreamSynchronize(ctx->stream);
+  free_all(ctx);
+  delete ctx;
+}
+
+int bkv_set_stream(bkv_ctx* ctx, void* stream) {
+  if (!ctx) return BKV_EINVAL;
+  ctx->stream = static_cast<cudaStream_t>(stream);
+  return BKV_OK;
+}
+
+int bkv_init_beacons(bkv_ctx* ctx, const void* q_init, int32_t n_init) {
+  if (!ctx) return BKV_EINVAL;
+  const Shape& s = ctx->shape;
+  if (s.nb == 0) {
+    ctx->state_ready = true;
+    return BKV_OK;
+  }
+  if (!q_init || !aligned16(q_init)) return fail(ctx, BKV_EINVAL, "q_init must be a non-NULL 16-byte aligned pointer");
+  const long long N = 1LL * s.G * n_init;
+  if (n_init < 1 || N < s.nb || N > bkv::kMaxFpsRows)
+    return fail(ctx, BKV_EINVAL, "G * n_init = %lld must be in n_beacons..4096", N);
+  ProfScope ps(ctx, BKV_K_FPS);
+  cudaError_t e = bkv::launch_fps_init(s, static_cast<const __nv_bfloat16*>(q_init), n_init, ctx->cent, ctx->sums,
+                                       ctx->counts, ctx->stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "fps_init launch");
+  ctx->state_ready = true;
+  return BKV_OK;
+}
+
+int bkv_update_beacons(bkv_ctx* ctx, const void* q_new, int32_t n_new, int32_t* assign_out) {
+  if (!ctx) return BKV_EINVAL;
+  const Shape& s = ctx->shape;
+  if (n_new < 0) return fail(ctx, BKV_EINVAL, "n_new must be >= 0");
+  if (n_new == 0) return BKV_OK;
+  if (!q_new || !aligned16(q_new)) return fail(ctx, BKV_EINVAL, "q_new must be a non-NULL 16-byte aligned pointer");
+  if (assign_out && (reinterpret_cast<uintptr_t>(assign_out) & 3u))
+    return fail(ctx, BKV_EINVAL, "assign_out must be 4-byte aligned");
+  if (1LL * s.n_inst * s.G * n_new >= (1LL << 31)) return fail(ctx, BKV_EINVAL, "n_new too large");
+  if (s.nb == 0) {
+    if (assign_out) {
+      cudaError_t e =
+          cudaMemsetAsync(assign_out, 0xff, sizeof(int32_t) * s.n_inst * s.G * static_cast<size_t>(n_new), ctx->stream);
+      if (e != cudaSuccess) return cuda_fail(ctx, e, "assign_out memset");
+    }
+    return BKV_OK;
+  }
+  if (!ctx->state_ready) return fail(ctx, BKV_ESTATE, "update before bkv_init_beacons / bkv_set_state");
+  ProfScope ps(ctx, BKV_K_UPDATE);
+  cudaError_t e = bkv::launch_update(s, static_cast<const __nv_bfloat16*>(q_new), n_new, ctx->cent, ctx->sums,
+                                     ctx->counts, assign_out, ctx->stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "update launch");
+  return BKV_OK;
+}
+
+int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int64_t t_pos, const void* q_recent,
+                 const int64_t* recent_pos, int32_t* kept_idx_out, float* scores_out) {
+  if (!ctx) return BKV_EINVAL;
+  const Shape& s = ctx->shape;
+  if (!K || !V || !kept_idx_out) return fail(ctx, BKV_EINVAL, "K, V and kept_idx_out must be non-NULL");
+  if (!aligned16(K) || !aligned16(V)) return fail(ctx, BKV_EINVAL, "K and V must be 16-byte aligned");
+  if (reinterpret_cast<uintptr_t>(kept_idx_out) & 3u) return fail(ctx, BKV_EINVAL, "kept_idx_out must be 4-byte aligned");
+  if (scores_out && (reinterpret_cast<uintptr_t>(scores_out) & 3u))
+    return fail(ctx, BKV_EINVAL, "scores_out must be 4-byte aligned");
+  if (L < 1 || L > s.cap) return fail(ctx, BKV_EINVAL, "L = %d must be in 1..capacity (%d)", L, s.cap);
+  if (budget < s.n_prefix + s.W)
+    return fail(ctx, BKV_EINVAL, "budget = %d is below n_prefix + window = %d", budget, s.n_prefix + s.W);
+  if (budget < 1) return fail(ctx, BKV_EINVAL, "budget must be >= 1");
+  if (1LL * s.n_inst * budget >= (1LL << 31)) return fail(ctx, BKV_EINVAL, "budget too large");
+  cudaError_t e;
+  if (L <= budget) {
+    ProfScope ps(ctx, BKV_K_KEEP_ALL);
+    e = bkv::launch_keep_all(s, L, budget, kept_idx_out, ctx->stream);
+    return e == cudaSuccess ? BKV_OK : cuda_fail(ctx, e, "keep_all launch");
+  }
+  if (s.W > 0 && (!q_recent || !aligned16(q_recent) || !recent_pos))
+    return fail(ctx, BKV_EINVAL, "q_recent (16-byte aligned) and recent_pos are required when window > 0");
+  if (s.nb > 0 && !ctx->state_ready) return fail(ctx, BKV_ESTATE, "compress before bkv_init_beacons / bkv_set_state");
+
+  // rotary table: slot w < W is recent_pos[w], slot W is t_pos
+  const int h = s.d / 2;
+  const double theta = ctx->cfg.rope_theta;
+  const int rotate = theta != 0.0;
+  if (rotate) {
+    for (int slot = 0; slot <= s.W; ++slot) {
+      const double pos = static_cast<double>(slot < s.W ? recent_pos[slot] : t_pos);
+      for (int i = 0; i < h; ++i) {
+        const double inv_freq = std::pow(theta, -static_cast<double>(2 * i) / static_cast<double>(s.d));
+        const double ang = pos * inv_freq;
+        ctx->rope_host[static_cast<size_t>(slot) * h + i] = make_double2(std::cos(ang), std::sin(ang));
+      }
+    }
+    e = cudaMemcpyAsync(ctx->rope, ctx->rope_host.data(), sizeof(double2) * ctx->rope_host.size(),
+                        cudaMemcpyHostToDevice, ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "rope table upload");
+  }
+  {
+    ProfScope ps(ctx, BKV_K_QOBS);
+    e = bkv::launch_qobs(s, static_cast<const __nv_bfloat16*>(q_recent), ctx->cent, ctx->counts, ctx->rope, rotate,
+                         ctx->qobs, ctx->valid, ctx->stream);
+  }
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "qobs launch");
+
+  CUtensorMap kmap, qmap;
+  int rc = encode_rows(ctx, &kmap, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 128);
+  if (rc != BKV_OK) return rc;
+  rc = encode_rows(ctx, &qmap, ctx->qobs, static_cast<uint64_t>(s.n_inst) * s.n_obs_pad, s.d,
+                   static_cast<uint32_t>(s.n_obs_pad));
+  if (rc != BKV_OK) return rc;
+  bkv::ScoreArgs sa;
+  sa.L = L;
+  sa.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(s.d)));
+  sa.valid = ctx->valid;
+  sa.r_out = ctx->rscore;
+  sa.scores_out = scores_out;
+  sa.err = ctx->err;
+  {
+    ProfScope ps(ctx, BKV_K_SCORE);
+    e = bkv::launch_score(s, kmap, qmap, sa, ctx->stream);
+  }
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "score launch");
+  {
+    ProfScope ps(ctx, BKV_K_SELECT_GATHER);
+    e = bkv::launch_select_gather(s, ctx->rscore, L, budget, static_cast<__nv_bfloat16*>(K),
+                                  static_cast<__nv_bfloat16*>(V), kept_idx_out, ctx->stream);
+  }
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "select_gather launch");
+  return BKV_OK;
+}
+
+int bkv_get_state(bkv_ctx* ctx, float* centroids, double* sums, int64_t* counts) {
+  if (!ctx) return BKV_EINVAL;
+  const Shape& s = ctx->shape;
+  const size_t n = static_cast<size_t>(s.n_inst) * s.nb;
+  cudaError_t e = cudaSuccess;
+  if (centroids && (e = cudaMemcpyAsync(centroids, ctx->cent, sizeof(float) * n * s.d, cudaMemcpyDeviceToDevice,
+                                        ctx->stream)) != cudaSuccess)
+    return cuda_fail(ctx, e, "get_state centroids");
+  if (sums && (e = cudaMemcpyAsync(sums, ctx->sums, sizeof(double) * n * s.d, cudaMemcpyDeviceToDevice,
+                                   ctx->stream)) != cudaSuccess)
+    return cuda_fail(ctx, e, "get_state sums");
+  if (counts && (e = cudaMemcpyAsync(counts, ctx->counts, sizeof(int64_t) * n, cudaMemcpyDeviceToDevice,
+                                     ctx->stream)) != cudaSuccess)
+    return cuda_fail(ctx, e, "get_state counts");
+  return BKV_OK;
+}
+
+int bkv_set_state(bkv_ctx* ctx, const float* centroids, const double* sums, const int64_t* counts) {
+  if (!ctx) return BKV_EINVAL;
+  const Shape& s = ctx->shape;
+  if (!centroids || !sums || !counts) return fail(ctx, BKV_EINVAL, "set_state needs all three arrays");
+  const size_t n = static_cast<size_t>(s.n_inst) * s.nb;
+  cudaError_t e;
+  if ((e = cudaMemcpyAsync(ctx->cent, centroids, sizeof(float) * n * s.d, cudaMemcpyDeviceToDevice, ctx->stream)) !=
+          cudaSuccess ||
+      (e = cudaMemcpyAsync(ctx->sums, sums, sizeof(double) * n * s.d, cudaMemcpyDeviceToDevice, ctx->stream)) !=
+          cudaSuccess ||
+      (e = cudaMemcpyAsync(ctx->counts, counts, sizeof(int64_t) * n, cudaMemcpyDeviceToDevice, ctx->stream)) !=
+          cudaSuccess)
+    return cuda_fail(ctx, e, "set_state copy");
+  ctx->state_ready = true;
+  return BKV_OK;
+}
+
+int bkv_profile_enable(bkv_ctx* ctx, int on) {
+  if (!ctx) return BKV_EINVAL;
+  ctx->prof = on != 0;
+  return BKV_OK;
+}
+
+int bkv_profile_read(bkv_ctx* ctx, double* ms, int64_t* launches, int32_t n_kernels) {
+  if (!ctx || n_kernels < 0) return BKV_EINVAL;
+  cudaError_t e = cudaStreamSynchronize(ctx->stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "stream synchronize");
+  fold_profile(ctx);
+  for (int k = 0; k < BKV_NUM_KERNELS && k < n_kernels; ++k) {
+    if (ms) ms[k] = ctx->prof_ms[k];
+    if (launches) launches[k] = ctx->prof_n[k];
+  }
+  for (int k = 0; k < BKV_NUM_KERNELS; ++k) {
+    ctx->prof_ms[k] = 0.0;
+    ctx->prof_n[k] = 0;
+  }
+  return BKV_OK;
+}
+
+int bkv_sync(bkv_ctx* ctx) {
+  if (!ctx) return BKV_EINVAL;
+  cudaError_t e = cudaStreamSynchronize(ctx->stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "stream synchronize");
+  int h = 0;
+  if ((e = cudaMemcpy(&h, ctx->err, sizeof(int), cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(ctx, e, "error word read");
+  if (h != 0) {
+    cudaMemset(ctx->err, 0, sizeof(int));
+    return fail(ctx, BKV_ETIMEOUT, "device wait expired (code %d)", h);
+  }
+  return BKV_OK;
+}
+
+}  // extern "C"

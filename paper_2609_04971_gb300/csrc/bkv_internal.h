@@ -1,0 +1,60 @@
+// Host-side declarations shared between the C-ABI layer (bkv_api.cu) and the
+// kernel translation units.  Not part of the public interface.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace bkv {
+
+// Per-context shape, derived once from bkv_config.
+struct Shape {
+  int n_inst;      // layers * batch * kv_heads
+  int G;           // query heads per KV head
+  int d;           // head_dim (64 or 128)
+  int nb;          // beacons per KV head
+  int W;           // recent window
+  int n_prefix;    // always-kept leading rows
+  int cap;         // rows per instance in K / V
+  int n_obs;       // G * W + nb scoring queries
+  int n_obs_pad;   // n_obs rounded up to 16
+};
+
+constexpr int kMaxBeacons = 32;
+constexpr int kMaxObs = 128;
+constexpr int kMaxWindow = 64;
+constexpr int kMaxCapacity = 32768;
+constexpr int kMaxFpsRows = 4096;
+
+// ---- beacon maintenance (k_fps.cu, k_update.cu)
+cudaError_t launch_fps_init(const Shape& s, const __nv_bfloat16* q_init, int n_init, float* cent, double* sums,
+                            long long* counts, cudaStream_t st);
+
+cudaError_t launch_update(const Shape& s, const __nv_bfloat16* q_new, int n_new, float* cent, double* sums,
+                          long long* counts, int* assign_out, cudaStream_t st);
+
+// ---- compression (k_qobs.cu, k_score.cu, k_select_gather.cu)
+// rope: [W + 1][d / 2] (cos, sin) pairs; entry w < W is recent slot w, entry W
+// is the beacon position.  rotate == 0 leaves vectors unrotated.
+cudaError_t launch_qobs(const Shape& s, const __nv_bfloat16* q_recent, const float* cent, const long long* counts,
+                        const double2* rope, int rotate, __nv_bfloat16* qobs, uint32_t* valid, cudaStream_t st);
+
+struct ScoreArgs {
+  int L;
+  float scale_log2;        // log2(e) / sqrt(d)
+  const uint32_t* valid;   // [n_inst][4] bitmask of valid scoring rows
+  float* r_out;            // [n_inst][cap] log2-domain scores (max_q logit - lse)
+  float* scores_out;       // [n_inst][cap] probabilities, or nullptr
+  int* err;                // device error word
+};
+cudaError_t launch_score(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreArgs& a,
+                         cudaStream_t st);
+
+cudaError_t launch_select_gather(const Shape& s, const float* r, int L, int budget, __nv_bfloat16* K,
+                                 __nv_bfloat16* V, int* kept, cudaStream_t st);
+
+cudaError_t launch_keep_all(const Shape& s, int L, int budget, int* kept, cudaStream_t st);
+
+}  // namespace bkv

@@ -1,0 +1,87 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds, loads and
+exports every function include/bkv.h declares; configuration validation and
+error strings behave as documented; the workload byte / FLOP accounting is
+consistent."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_04971_gb300 import _build, bkv
+from paper_2609_04971_gb300.workloads import LLAMA_8B, QWEN3_14B, QWEN3_4B, TINY, n_obs_padded
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "bkv.h")
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(bkv_[a-z_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return bkv.load_library()
+
+
+def test_header_declares_the_api():
+    names = _declared()
+    for n in ("bkv_create", "bkv_destroy", "bkv_init_beacons", "bkv_update_beacons", "bkv_compress",
+              "bkv_get_state", "bkv_set_state", "bkv_sync", "bkv_strerror"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    raw = ctypes.CDLL(_build.LIB_PATH)
+    missing = [n for n in _declared() if not hasattr(raw, n)]
+    assert not missing, f"declared but not exported: {missing}"
+
+
+def test_binding_mirrors_every_declared_symbol():
+    missing = [n for n in _declared() if not hasattr(bkv, n)]
+    assert not missing, f"no Python binding for: {missing}"
+
+
+def test_strerror_and_version(lib):
+    assert bkv.bkv_strerror(0) == "ok"
+    assert "invalid" in bkv.bkv_strerror(-1)
+    assert bkv.bkv_strerror(-99) == "unknown error"
+    assert "sm_103a" in bkv.bkv_version()
+
+
+@pytest.mark.parametrize("field,value", [
+    ("n_kv_heads", 3), ("head_dim", 96), ("n_beacons", 33), ("window", -1), ("window", 65),
+    ("capacity", 0), ("capacity", 40000), ("rope_theta", -1.0), ("flags", 1), ("n_layers", 0),
+    ("n_prefix", -2)])
+def test_create_rejects_bad_config_before_touching_the_gpu(lib, field, value):
+    cfg = bkv.BkvConfig(1, 1, 4, 2, 64, 4, 8, 0, 1088, 1e4, 0)
+    setattr(cfg, field, value)
+    out = ctypes.c_void_p()
+    assert lib.bkv_create(ctypes.byref(cfg), None, ctypes.byref(out)) == bkv.BKV_EINVAL
+    assert not out.value
+
+
+def test_create_rejects_too_many_scoring_queries(lib):
+    cfg = bkv.BkvConfig(1, 1, 64, 4, 128, 8, 8, 0, 1024, 1e4, 0)   # 16 * 8 + 8 = 136 > 128
+    out = ctypes.c_void_p()
+    assert lib.bkv_create(ctypes.byref(cfg), None, ctypes.byref(out)) == bkv.BKV_EINVAL
+
+
+def test_null_arguments(lib):
+    assert lib.bkv_create(None, None, None) == bkv.BKV_EINVAL
+    assert lib.bkv_sync(None) == bkv.BKV_EINVAL
+    assert lib.bkv_compress(None, None, None, 1, 1, 0, None, None, None, None) == bkv.BKV_EINVAL
+    lib.bkv_destroy(None)
+    assert lib.bkv_last_error(None) == b""
+
+
+def test_byte_accounting_matches_closed_form():
+    wl = QWEN3_4B
+    per_inst = 4224 * 128 * 2 + 4096 * 128 * 2 * 4 + 4 * 8 * 128 * 2 + 4096 * 4
+    assert wl.compress_bytes() == per_inst * 36 * 16 * 8
+    assert abs(wl.step_bytes() / 1e9 - 25.06) < 0.02
+    assert wl.n_obs == 40 and n_obs_padded(wl.n_obs) == 48
+    assert LLAMA_8B.n_obs == 48 and QWEN3_14B.n_obs == 56 and TINY.n_obs == 20
+    assert n_obs_padded(QWEN3_14B.n_obs) == 64 and n_obs_padded(TINY.n_obs) == 32

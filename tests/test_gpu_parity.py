@@ -1,0 +1,117 @@
+"""CUDA path (through the C ABI) against the fp64 oracle, element by element.
+
+Sizes span several 128-key tiles and ragged tails; the full-size workloads run
+in the launch configuration bench.py times and are checked on sampled
+instances.  Tolerances are stated in tests/parity.py.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_04971_gb300.workloads import LLAMA_8B, QWEN3_14B, QWEN3_4B, TINY
+
+pytestmark = pytest.mark.gpu
+
+if torch.cuda.is_available():
+    from tests import parity as P
+
+
+def _run(wl, seed=0, sample=None, **kw):
+    run = P.run_gpu(wl, seed=seed, sample=sample, **kw)
+    rep = P.check_run(run, L=kw.get("L"), budget=kw.get("budget"))
+    print(f"{wl.name}: {rep}")
+    return run, rep
+
+
+def test_tiny_workload_all_instances():
+    _run(TINY)
+
+
+@pytest.mark.parametrize("wl", [
+    QWEN3_4B.scaled(name="qwen3_4b_1L_b2", n_layers=1, batch=2),
+    LLAMA_8B.scaled(name="llama_8b_1L_b2", n_layers=1, batch=2),
+    QWEN3_14B.scaled(name="qwen3_14b_1L_b1", n_layers=1, batch=1),
+], ids=lambda w: w.name)
+def test_reduced_batch_full_length(wl):
+    _run(wl)
+
+
+@pytest.mark.parametrize("L,budget", [(1000, 700), (100, 50), (129, 128), (300, 17), (640, 639)])
+def test_ragged_lengths(L, budget):
+    wl = QWEN3_4B.scaled(name=f"ragged_L{L}_B{budget}", n_layers=1, batch=1, L=L, budget=budget)
+    _run(wl, seed=L)
+
+
+def test_head_dim_64_ragged():
+    wl = TINY.scaled(name="d64_L777", L=777, budget=400, n_layers=2, batch=3)
+    _run(wl, seed=3)
+
+
+def test_prefix_kept():
+    wl = QWEN3_4B.scaled(name="prefix4", n_layers=1, batch=1, L=600, budget=300, n_prefix=4)
+    _run(wl, seed=5)
+
+
+def test_recent_only_no_beacons():
+    wl = QWEN3_4B.scaled(name="nb0", n_layers=1, batch=2, L=500, budget=260, n_beacons=0)
+    _run(wl, seed=6)
+
+
+def test_beacons_only_no_window():
+    wl = LLAMA_8B.scaled(name="w0", n_layers=1, batch=1, L=400, budget=200, window=0)
+    _run(wl, seed=7)
+
+
+def test_budget_equals_keep_set():
+    wl = QWEN3_4B.scaled(name="ksel0", n_layers=1, batch=1, L=300, budget=8)
+    _run(wl, seed=8)
+
+
+def test_no_eviction_when_cache_fits():
+    wl = QWEN3_4B.scaled(name="fits", n_layers=1, batch=1, L=256, budget=300)
+    _run(wl, seed=9)
+
+
+def test_no_rotation_and_max_queries():
+    # G * W + nb = 8 * 12 + 32 = 128 scoring queries (the maximum), theta = 0
+    wl = QWEN3_4B.scaled(name="m128", n_layers=1, batch=1, n_q_heads=64, n_kv_heads=8, window=12, n_beacons=32,
+                         L=700, budget=500, rope_theta=0.0, n_init=64, n_clusters=32)
+    _run(wl, seed=10)
+
+
+def test_identical_keys_tie_everywhere():
+    """All keys equal: every score is 1/L, the kept set is the lowest-index
+    candidates plus the window (ties go to the lower index)."""
+    wl = QWEN3_4B.scaled(name="flat", n_layers=1, batch=1, L=400, budget=100)
+    dev = torch.device("cuda")
+    from paper_2609_04971_gb300 import synth
+    inp = synth.step_inputs(wl, 11, dev)
+    inp["K"][:] = inp["K"][:, :, :, :1, :]
+    run = P.run_gpu(wl, inputs=inp)
+    want = np.concatenate([np.arange(92), np.arange(392, 400)])
+    for e in range(wl.n_inst):
+        np.testing.assert_array_equal(run.kept[e], want)
+        np.testing.assert_allclose(run.scores[e][:400], 1.0 / 400, rtol=1e-5)
+
+
+@pytest.mark.parametrize("wl", [QWEN3_4B, LLAMA_8B, QWEN3_14B], ids=lambda w: w.name)
+def test_full_size_sampled(wl):
+    rng = np.random.default_rng(0)
+    sample = np.unique(np.concatenate([[0, wl.n_inst - 1], rng.choice(wl.n_inst, 6, replace=False)]))
+    run, rep = _run(wl, sample=sample)
+    # every instance, not only the sampled ones: budget, order, keep set
+    kept = run.kept
+    assert kept.shape == (wl.n_inst, wl.budget)
+    assert np.all(np.diff(kept, axis=1) > 0)
+    assert np.all(kept[:, -wl.window:] == np.arange(wl.L - wl.window, wl.L))
+    assert run.counts1.sum(axis=1).min() == wl.group * (wl.n_init * 0 + wl.n_new) + wl.n_beacons
+
+
+def test_deterministic_across_runs():
+    wl = QWEN3_4B.scaled(name="det", n_layers=1, batch=2, L=900, budget=500)
+    a = P.run_gpu(wl, seed=12)
+    b = P.run_gpu(wl, seed=12)
+    np.testing.assert_array_equal(a.kept, b.kept)
+    np.testing.assert_array_equal(a.scores, b.scores)
+    np.testing.assert_array_equal(a.cent1, b.cent1)
+    np.testing.assert_array_equal(a.K_after, b.K_after)
