@@ -1,0 +1,439 @@
+#!/usr/bin/env python
+"""Benchmark of the BeaconKV compress step on GB300.
+
+One step = one beacon update (128 decode queries per query head) followed by
+one compression of every (layer, batch row, KV head) cache from L = 4224 to a
+budget of 4096 rows, on the Qwen3-4B shape (36 layers, batch 16, 32 query / 8
+KV heads, head_dim 128, 8 beacons, 8-query recent window): 4608 instances.
+
+Between timed steps (outside the timed events) the 128 rows evicted by the
+previous compress are refilled with "new tokens", as a decode loop would, and
+L2 is flushed by writing 256 MB; the K/V working set (10 GB) exceeds L2 anyway.
+Every step is bracketed by CUDA events on the stream the library launches on.
+
+    python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+
+Prints one JSON line (rank 0).  --impl reference times the CPU oracle (the
+plain fp64 restatement of the method) on the host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "cached KV tokens scored+compacted/s per compress step"
+UNIT = "tokens/s"
+FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+
+
+def parse():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", type=int, default=2, help="workload number (2 = Qwen3-4B shape)")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--layers", type=int, default=0, help="override the layer count (small profiling captures)")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
+    except Exception:  # noqa: BLE001
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.path = tempfile.mktemp(prefix="bkv_clocks_", suffix=".csv")
+        self.proc = None
+        self.gpu_index = gpu_index
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu_index}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader",
+                 "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+            t0 = time.time()
+            while time.time() - t0 < 3.0 and os.path.getsize(self.path) == 0:
+                time.sleep(0.02)
+        except Exception:  # noqa: BLE001
+            self.proc = None
+
+    def stop(self) -> dict | None:
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:  # noqa: BLE001
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 10:
+                    continue
+                try:
+                    rows.append(dict(sm=float(parts[2].split()[0]), max=float(parts[3].split()[0]),
+                                     power=parts[4], reasons=parts[5:]))
+                except ValueError:
+                    continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["active_mask", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        seen = sorted({names[i] for r in rows for i, v in enumerate(r["reasons"]) if i > 0 and v == "Active"})
+        return {"sm_mhz": statistics.median(r["sm"] for r in rows), "sm_max_mhz": max(r["max"] for r in rows),
+                "samples": len(rows), "reasons": seen}
+
+
+# ------------------------------------------------------------------ CPU oracle
+def oracle_sample_step(wl, n_batch: int, seed: int):
+    """Prepare a CPU-side sample of the workload (n_batch batch rows of one layer)
+    for the oracle; returns a callable that runs one update + compress on it."""
+    import numpy as np
+    import torch
+    from oracle import oracle as O
+    from paper_2609_04971_gb300 import synth
+
+    sub = wl.scaled(n_layers=1, batch=n_batch)
+    inp = synth.step_inputs(sub, seed, "cpu")
+    n_inst, G, d, nb, W = sub.n_inst, sub.group, sub.head_dim, sub.n_beacons, sub.window
+
+    def bits(t):
+        return t.contiguous().view(torch.int16).numpy().view(np.uint16)
+
+    q_init = bits(inp["q_init"]).reshape(n_inst, G * sub.n_init, d)
+    base = dict(q_new=bits(inp["q_new"]).reshape(n_inst, G, sub.n_new, d).copy(),
+                q_recent=bits(inp["q_recent"]).reshape(n_inst, G, W, d).copy(),
+                K=bits(inp["K"]).reshape(n_inst, sub.capacity, d).copy(),
+                V=bits(inp["V"]).reshape(n_inst, sub.capacity, d).copy())
+    # Seeding is not part of the timed step: beacons start as the first nb prompt queries.
+    sums = O.bf16_to_f64(q_init[:, :nb]).copy()
+    cent = sums.astype(np.float32)
+    counts = np.ones((n_inst, nb), np.int64)
+
+    def run():
+        K, V = base["K"].copy(), base["V"].copy()
+        c, s, n = cent.copy(), sums.copy(), counts.copy()
+        kept = np.zeros((n_inst, sub.budget), np.int32)
+        t0 = time.perf_counter()
+        threads = O.step_many(np.arange(n_inst), G=G, d=d, nb=nb, W=W, n_prefix=sub.n_prefix, cap=sub.capacity,
+                              q_new=base["q_new"], n_new=sub.n_new, q_recent=base["q_recent"],
+                              recent_pos=np.asarray(inp["recent_pos"], np.int64), t_pos=inp["t_pos"],
+                              theta=sub.rope_theta, L=sub.L, budget=sub.budget, K=K, V=V, cent=c, sums=s,
+                              counts=n, kept=kept)
+        return time.perf_counter() - t0, threads
+
+    return run, n_inst
+
+
+def cpu_baseline(wl, target_s: float, seed: int) -> dict:
+    run, n_probe = oracle_sample_step(wl, 2, seed)
+    dt, threads = run()
+    per_inst = dt / n_probe * max(1, threads)          # single-thread seconds per instance
+    want = int(target_s * max(1, threads) / max(per_inst, 1e-6))
+    n_batch = max(2, min(wl.batch * wl.n_layers, want // wl.n_kv_heads))
+    run, n_inst = oracle_sample_step(wl, n_batch, seed)
+    dt, threads = run()
+    value = n_inst * wl.L / dt
+    return {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"{n_inst} of {wl.n_inst} instances ({n_batch} batch rows x {wl.n_kv_heads} KV heads), "
+                      f"one update + compress each, fp64 C oracle with OpenMP, {dt:.1f} s "
+                      f"(beacons seeded untimed with the first prompt queries)"}
+
+
+def reference_arm(args, wl, rank: int) -> None:
+    if rank != 0:
+        return
+    run, n_probe = oracle_sample_step(wl, 2, args.seed)
+    dt, threads = run()
+    per_inst = dt / n_probe * max(1, threads)
+    budget_s = 150.0 / max(1, args.steps + args.warmup)          # whole run within a few minutes
+    n_batch = max(1, min(wl.batch * wl.n_layers, int(budget_s * threads / per_inst) // wl.n_kv_heads))
+    run, n_inst = oracle_sample_step(wl, n_batch, args.seed)
+    for _ in range(args.warmup):
+        run()
+    times = []
+    for _ in range(args.steps):
+        dt, threads = run()
+        times.append(dt)
+    total = sum(times)
+    value = n_inst * wl.L * len(times) / total
+    sample = (f"{n_inst} of {wl.n_inst} instances per step ({n_batch} batch rows x {wl.n_kv_heads} KV heads), "
+              f"fp64 C oracle with OpenMP")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(times),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": config_block(wl, args.gpus),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def config_block(wl, n_gpus: int) -> dict:
+    return {"workload": wl.name, "layers": wl.n_layers, "batch": wl.batch, "q_heads": wl.n_q_heads,
+            "kv_heads": wl.n_kv_heads, "head_dim": wl.head_dim, "L": wl.L, "budget": wl.budget,
+            "window": wl.window, "beacons": wl.n_beacons, "new_queries_per_head": wl.n_new,
+            "instances_per_gpu": wl.n_inst, "rope_theta": wl.rope_theta,
+            "l2": "256 MB write before every timed step; K/V working set 10 GB > L2",
+            "parallelism": "replicas" if n_gpus == 1 else f"dp{n_gpus} (independent instances, no collective)"}
+
+
+# ------------------------------------------------------------------ traffic from ncu
+def traffic_from_profiles(kernel: str, n_inst: int):
+    """dram bytes per launch recorded by an ncu capture under profiles/, if the
+    kernel source has not changed since (matched by sha256 of the .cu file)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)[kernel]
+        src = os.path.join(ROOT, "paper_2609_04971_gb300", "csrc", rec["source"])
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        if h != rec["sha256"]:
+            return None
+        return rec["bytes_per_instance"] * n_inst
+    except Exception:  # noqa: BLE001
+        return None
+
+
+# ------------------------------------------------------------------ multi-rank
+def max_over_ranks(x: float, world: int, device) -> float:
+    """Largest value of x over all ranks (the job ends when the slowest rank does)."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate_throughput(tokens_per_step_per_rank: int, world: int, steps: int, total_ms: float) -> float:
+    """Whole-job tokens/s: every rank compresses its own instances (weak scaling)."""
+    return tokens_per_step_per_rank * world * steps / (total_ms / 1e3)
+
+
+def rank_seed(seed: int, rank: int) -> int:
+    """Each rank draws its own instances (independent problems, no exchange)."""
+    return seed + 7919 * rank
+
+
+# ------------------------------------------------------------------ main GPU bench
+def main():
+    args = parse()
+    from paper_2609_04971_gb300.workloads import WORKLOADS
+    wl = WORKLOADS[args.config]
+    if args.layers:
+        wl = wl.scaled(n_layers=args.layers, name=f"{wl.name}_{args.layers}layers")
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        reference_arm(args, wl, rank)
+        return
+
+    import torch
+    import torch.distributed as dist
+    from paper_2609_04971_gb300 import bkv, synth
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    hbm_gbs, bf16_tflops, peak_src = peaks()
+    inp = synth.step_inputs(wl, rank_seed(args.seed, rank), dev)
+    K, V = inp["K"], inp["V"]
+    L, budget = wl.L, wl.budget
+    new_k = K[:, :, :, budget:L].clone()      # "new tokens" written back after every compress
+    new_v = V[:, :, :, budget:L].clone()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    kept = torch.empty(wl.n_layers, wl.batch, wl.n_kv_heads, budget, dtype=torch.int32, device=dev)
+    bk = bkv.BeaconKV.for_workload(wl)
+    bk.init_beacons(inp["q_init"])
+    bk.sync()
+
+    def prepare(i):
+        if i > 0:
+            K[:, :, :, budget:L].copy_(new_k)
+            V[:, :, :, budget:L].copy_(new_v)
+        flush.fill_(i & 0xFF)
+
+    def step(i):
+        t_pos = inp["t_pos"] + (L - budget) * i
+        bk.update(inp["q_new"])
+        bk.compress(K, V, L=L, budget=budget, t_pos=t_pos, q_recent=inp["q_recent"],
+                    recent_pos=[p + (L - budget) * i for p in inp["recent_pos"]], kept_out=kept)
+
+    for i in range(args.warmup):
+        prepare(i)
+        step(i)
+    bk.sync()
+    bkv.bkv_profile_read(bk.ctx)
+    bkv.bkv_profile_enable(bk.ctx, True)
+
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    gpu_index = int(vis.split(",")[local_rank]) if vis and vis.split(",")[0].isdigit() else local_rank
+    sampler = ClockSampler(gpu_index)
+    sampler.start()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    barrier()
+    torch.cuda.synchronize()
+    for i in range(args.steps):
+        prepare(args.warmup + i)
+        ev[i][0].record()
+        step(args.warmup + i)
+        ev[i][1].record()
+    torch.cuda.synchronize()
+    barrier()
+    clocks = sampler.stop()
+    bk.sync()
+    prof = bkv.bkv_profile_read(bk.ctx)
+    bkv.bkv_profile_enable(bk.ctx, False)
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = max_over_ranks(sum(step_ms), world, dev)
+    ms_per_step = total_ms / args.steps
+    value = aggregate_throughput(wl.tokens_per_step(), world, args.steps, total_ms)
+
+    # per-kernel roofline (algorithmic bytes per launch / measured duration per launch)
+    d = wl.head_dim
+    alg_bytes = {
+        "update": wl.update_bytes(),
+        "qobs": wl.n_inst * wl.group * wl.window * d * 2,
+        "score": wl.n_inst * L * d * 2,
+        "select_gather": wl.n_inst * (budget * d * 2 * 4 + budget * 4),
+    }
+    kernels = {}
+    for name, b in alg_bytes.items():
+        ms, n = prof.get(name, (0.0, 0))
+        if n:
+            per = ms / n
+            kernels[name] = {"ms_per_launch": per, "launches": n, "alg_bytes_per_launch": b,
+                             "achieved_gbs": b / (per * 1e-3) / 1e9, "frac_of_hbm": b / (per * 1e-3) / 1e9 / hbm_gbs}
+    dom = max(kernels, key=lambda k: kernels[k]["ms_per_launch"] * kernels[k]["launches"])
+    kd = kernels[dom]
+    traffic = traffic_from_profiles(dom, wl.n_inst)
+    roofline = {"bound": "hbm", "kernel": dom, "achieved": kd["achieved_gbs"], "peak": hbm_gbs, "unit": "GB/s",
+                "frac": kd["achieved_gbs"] / hbm_gbs, "traffic": traffic,
+                "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else
+                f"fallback {FALLBACK_HBM_GBS} GB/s"}
+    step_roof_s = wl.roofline_seconds(hbm_gbs, bf16_tflops)
+    launches = sum(n for _, n in prof.values())
+
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config_block(wl, world),
+        "roofline": roofline,
+        "step_roofline": {"alg_bytes": wl.step_bytes(), "alg_flops": wl.step_flops(),
+                          "roofline_ms": step_roof_s * 1e3, "frac": step_roof_s * 1e3 / ms_per_step},
+        "kernels": kernels, "gpu_launches": launches, "clocks": clocks,
+        "step_ms_p10_p50_p90": [float(x) for x in
+                                (sorted(step_ms)[len(step_ms) // 10], statistics.median(step_ms),
+                                 sorted(step_ms)[(9 * len(step_ms)) // 10])],
+    }
+
+    # end to end through the public API with host buffers
+    if not args.no_e2e:
+        out["e2e"] = e2e(bk, wl, inp, args, dev, world, barrier)
+    del new_k, new_v, flush
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds, args.seed)
+    bk.close()
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def e2e(bk, wl, inp, args, dev, world, barrier) -> dict:
+    """Host-resident step: H2D of K, V (L rows), q_new, q_recent from pinned memory,
+    update + compress, D2H of the kept indices and the compacted K / V rows."""
+    import torch
+    L, budget = wl.L, wl.budget
+    def pinned_copy(t):
+        h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        h.copy_(t)
+        return h
+
+    K_h, V_h = pinned_copy(inp["K"]), pinned_copy(inp["V"])
+    qn_h, qr_h = pinned_copy(inp["q_new"]), pinned_copy(inp["q_recent"])
+    shape_out = (wl.n_layers, wl.batch, wl.n_kv_heads, budget, wl.head_dim)
+    Ko_h = torch.empty(shape_out, dtype=torch.bfloat16, pin_memory=True)
+    Vo_h = torch.empty(shape_out, dtype=torch.bfloat16, pin_memory=True)
+    kept_h = torch.empty(wl.n_layers, wl.batch, wl.n_kv_heads, budget, dtype=torch.int32, pin_memory=True)
+    K_d, V_d = inp["K"], inp["V"]
+    qn_d, qr_d = inp["q_new"], inp["q_recent"]
+    kept_d = torch.empty_like(kept_h, device=dev)
+    h2d = sum(t.numel() * t.element_size() for t in (K_h, V_h, qn_h, qr_h))
+    d2h = sum(t.numel() * t.element_size() for t in (Ko_h, Vo_h, kept_h))
+
+    def one(i):
+        K_d.copy_(K_h, non_blocking=True)
+        V_d.copy_(V_h, non_blocking=True)
+        qn_d.copy_(qn_h, non_blocking=True)
+        qr_d.copy_(qr_h, non_blocking=True)
+        bk.update(qn_d)
+        bk.compress(K_d, V_d, L=L, budget=budget, t_pos=inp["t_pos"], q_recent=qr_d, recent_pos=inp["recent_pos"],
+                    kept_out=kept_d)
+        Ko_h.copy_(K_d[:, :, :, :budget], non_blocking=True)
+        Vo_h.copy_(V_d[:, :, :, :budget], non_blocking=True)
+        kept_h.copy_(kept_d, non_blocking=True)
+
+    one(0)
+    torch.cuda.synchronize()
+    n = max(1, args.e2e_steps)
+    barrier()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for i in range(n):
+        one(i)
+    b.record()
+    torch.cuda.synchronize()
+    barrier()
+    ms = a.elapsed_time(b) / n
+    bk.sync()
+    return {"value": wl.tokens_per_step() * world / (ms / 1e3), "unit": UNIT, "ms_per_step": ms,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+
+if __name__ == "__main__":
+    main()
