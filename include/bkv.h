@@ -46,6 +46,7 @@
 #ifndef BKV_H
 #define BKV_H
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -187,6 +188,38 @@ int bkv_sync(bkv_ctx* ctx);
 #define BKV_NUM_KERNELS 6
 int bkv_profile_enable(bkv_ctx* ctx, int on);
 int bkv_profile_read(bkv_ctx* ctx, double* ms, int64_t* launches, int32_t n_kernels);
+
+/*
+ * bkv_compress_static - bkv_compress for callers that must not allocate
+ * device memory.  The paper has no counterpart: this entry point exists for
+ * integrations that cannot call cudaMalloc, such as a serving engine that has
+ * given all of HBM to its own KV-cache page allocator, or a plugin whose host
+ * framework owns every device allocation (cudaMalloc may also synchronise
+ * the device, which a decode loop on a latency budget cannot afford).
+ *
+ * Computes exactly what bkv_compress computes, with the same kernels, but
+ * takes everything from the caller: the shape (cfg, same limits as
+ * bkv_create), the beacon state (centroids fp32 [n_inst][n_beacons][d] and
+ * counts int64 [n_inst][n_beacons], device; may be NULL when n_beacons = 0)
+ * and the stream.  It needs no context and allocates or frees nothing.  Its
+ * scratch is one library-owned device array of 16 MiB (resident on every
+ * device that loads the library until the process exits); a call whose
+ * scratch exceeds it - n_inst * (4 * capacity + 2 * n_obs_pad * head_dim +
+ * 16) bytes plus the rotary table, each part rounded up to 256 bytes - is
+ * rejected with BKV_EINVAL and a message.
+ *   dev_status  device int32 or NULL: cleared by the call, set non-zero if a
+ *               kernel's bounded wait expires (outputs are then invalid).
+ *   err_msg     host buffer of err_len bytes or NULL: reason of a failure.
+ * All calls share the scratch array and it keeps the previous call's
+ * contents; calls that overlap on the GPU (other streams, other threads
+ * without ordering) race on it.  The array's device address is looked up
+ * with cudaGetSymbolAddress during the first call on each device (with that
+ * device current), so make that first call before any stream capture.
+ */
+int bkv_compress_static(const bkv_config* cfg, const float* centroids, const int64_t* counts, void* K, void* V,
+                        int32_t L, int32_t budget, int64_t t_pos, const void* q_recent, const int64_t* recent_pos,
+                        int32_t* kept_idx_out, float* scores_out, int32_t* dev_status, void* stream, char* err_msg,
+                        size_t err_len);
 
 /* Static description of an error code. */
 const char* bkv_strerror(int code);

@@ -67,6 +67,9 @@ def load_library(path: str | None = None, build: bool = True):
             "bkv_get_state": (ctypes.c_int, [_P, _P, _P, _P]),
             "bkv_set_state": (ctypes.c_int, [_P, _P, _P, _P]),
             "bkv_sync": (ctypes.c_int, [_P]),
+            "bkv_compress_static": (ctypes.c_int, [ctypes.POINTER(BkvConfig), _P, _P, _P, _P, ctypes.c_int32,
+                                                   ctypes.c_int32, ctypes.c_int64, _P, _P, _P, _P, _P, _P,
+                                                   ctypes.c_char_p, ctypes.c_size_t]),
             "bkv_profile_enable": (ctypes.c_int, [_P, ctypes.c_int]),
             "bkv_profile_read": (ctypes.c_int, [_P, _P, _P, ctypes.c_int32]),
             "bkv_strerror": (ctypes.c_char_p, [ctypes.c_int]),
@@ -185,6 +188,25 @@ def bkv_profile_read(ctx) -> dict:
     cnt = (ctypes.c_int64 * n)()
     _check(_l().bkv_profile_read(ctx, ctypes.cast(ms, _P), ctypes.cast(cnt, _P), n), "bkv_profile_read", ctx)
     return {KERNEL_NAMES[k]: (ms[k], cnt[k]) for k in range(n)}
+
+
+def bkv_compress_static(cfg: BkvConfig, centroids, counts, K, V, L: int, budget: int, t_pos: int, q_recent,
+                        recent_pos, kept_idx_out, scores_out=None, dev_status=None, stream=None) -> None:
+    """Context-free compress that allocates no device memory (see include/bkv.h).
+
+    For callers that cannot allocate on the device, e.g. an engine whose KV
+    page allocator owns all of HBM.  Scratch lives in a fixed 16 MiB array
+    inside the library; concurrent calls on different streams race on it."""
+    pos = (ctypes.c_int64 * max(1, len(recent_pos)))(*[int(p) for p in recent_pos])
+    msg = ctypes.create_string_buffer(256)
+    rc = _l().bkv_compress_static(
+        ctypes.byref(cfg), _ptr(centroids, torch.float32, "centroids"), _ptr(counts, torch.int64, "counts"),
+        _ptr(K, torch.bfloat16, "K"), _ptr(V, torch.bfloat16, "V"), int(L), int(budget), int(t_pos),
+        _ptr(q_recent, torch.bfloat16, "q_recent"), ctypes.cast(pos, _P), _ptr(kept_idx_out, torch.int32, "kept"),
+        _ptr(scores_out, torch.float32, "scores_out"), _ptr(dev_status, torch.int32, "dev_status"),
+        _stream(stream), msg, ctypes.sizeof(msg))
+    if rc != BKV_OK:
+        raise BkvError(rc, "bkv_compress_static", msg.value.decode())
 
 
 # ---------------------------------------------------------------- convenience

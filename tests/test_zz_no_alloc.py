@@ -1,0 +1,75 @@
+"""bkv_compress_static against bkv_compress, through the C ABI.
+
+bkv_compress_static is for callers that cannot allocate device memory (for
+example an engine whose KV page allocator owns all of HBM, or a plugin whose
+host framework owns every allocation): it runs the same compression with its
+scratch in a fixed array inside the library and takes the beacon state from
+the caller.  Several calls in a row must each match the context-based entry
+point (the scratch array keeps the previous call's contents), within the
+parity tolerances of tests/parity.py: identical kept indices and K / V bytes,
+scores within 1e-3 relative.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_04971_gb300.workloads import QWEN3_4B, TINY
+
+pytestmark = pytest.mark.gpu
+
+
+def _compare_once(wl, seed):
+    from paper_2609_04971_gb300 import bkv, synth
+    dev = torch.device("cuda")
+    inp = synth.step_inputs(wl, seed, dev)
+    bk = bkv.BeaconKV.for_workload(wl)
+    try:
+        bk.init_beacons(inp["q_init"])
+        bk.update(inp["q_new"])
+        cent, _, counts = bk.state()
+        K1, V1 = inp["K"].clone(), inp["V"].clone()
+        K2, V2 = inp["K"].clone(), inp["V"].clone()
+        shape_s = (wl.n_layers, wl.batch, wl.n_kv_heads, wl.capacity)
+        s1 = torch.zeros(shape_s, device=dev)
+        s2 = torch.full(shape_s, -1.0, device=dev)
+        kept1 = bk.compress(K1, V1, L=wl.L, budget=wl.budget, t_pos=inp["t_pos"], q_recent=inp["q_recent"],
+                            recent_pos=inp["recent_pos"], scores_out=s1)
+        kept2 = torch.full_like(kept1, -5)
+        status = torch.full((1,), 77, dtype=torch.int32, device=dev)
+        bkv.bkv_compress_static(bk.cfg, cent, counts, K2, V2, wl.L, wl.budget, inp["t_pos"], inp["q_recent"],
+                                inp["recent_pos"], kept2, s2, status)
+        torch.cuda.synchronize()
+        bk.sync()
+    finally:
+        bk.close()
+    assert int(status.item()) == 0
+    np.testing.assert_array_equal(kept2.cpu().numpy(), kept1.cpu().numpy())
+    a = s1[..., :wl.L].double().cpu().numpy()
+    b = s2[..., :wl.L].double().cpu().numpy()
+    assert np.max(np.abs(a - b) / np.maximum(np.abs(a), 1e-300)) <= 1e-3
+    assert torch.equal(K2[..., :wl.budget, :], K1[..., :wl.budget, :])
+    assert torch.equal(V2[..., :wl.budget, :], V1[..., :wl.budget, :])
+
+
+def test_static_compress_matches_context_compress_on_consecutive_calls():
+    ragged = QWEN3_4B.scaled(name="static_ragged", n_layers=1, batch=2, L=1000, budget=700)
+    _compare_once(ragged, seed=21)
+    _compare_once(ragged, seed=22)        # same shape, new data over the previous scratch contents
+    _compare_once(TINY, seed=23)          # another shape (head_dim 64) over the same scratch
+
+
+def test_static_compress_rejects_requests_beyond_its_scratch():
+    from paper_2609_04971_gb300 import bkv
+    wl = QWEN3_4B.scaled(name="static_big", n_layers=8)    # 1024 instances x 4224 rows: ~30 MB of scratch
+    dev = torch.device("cuda")
+    cfg = bkv.BkvConfig(wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.n_beacons, wl.window,
+                        0, wl.capacity, wl.rope_theta, 0)
+    K = torch.zeros(wl.n_layers, wl.batch, wl.n_kv_heads, wl.capacity, wl.head_dim, dtype=torch.bfloat16,
+                    device=dev)
+    kept = torch.empty(wl.n_layers, wl.batch, wl.n_kv_heads, wl.budget, dtype=torch.int32, device=dev)
+    cent = torch.zeros(wl.n_inst, wl.n_beacons, wl.head_dim, device=dev)
+    counts = torch.ones(wl.n_inst, wl.n_beacons, dtype=torch.int64, device=dev)
+    q = torch.zeros(wl.n_layers, wl.batch, wl.n_q_heads, wl.window, wl.head_dim, dtype=torch.bfloat16, device=dev)
+    with pytest.raises(bkv.BkvError) as ei:
+        bkv.bkv_compress_static(cfg, cent, counts, K, K, wl.L, wl.budget, wl.L - 1, q, list(range(wl.window)), kept)
+    assert ei.value.code == bkv.BKV_EINVAL and "scratch" in str(ei.value)
