@@ -30,9 +30,9 @@ struct bkv_ctx {
   __nv_bfloat16* qobs = nullptr;  // [n_inst][n_obs_pad][d]
   uint32_t* valid = nullptr;      // [n_inst][4]
   float* rscore = nullptr;        // [n_inst][cap]
-  double2* rope = nullptr;        // [W + 1][d / 2]
+  double2* rope = nullptr;        // [W + 1][d / 2] fp64 (cos, sin), then the same table in fp32
   int* err = nullptr;             // device error word
-  std::vector<double2> rope_host;
+  std::vector<double2> rope_host;  // fp64 entries followed by fp32 entries (packed two per double2)
   std::string last_error;
   // per-kernel timing
   struct Rec {
@@ -238,7 +238,7 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
       (e = dmalloc(&c->qobs, ni * s.n_obs_pad * s.d)) != cudaSuccess ||
       (e = dmalloc(&c->valid, ni * 4)) != cudaSuccess ||
       (e = dmalloc(&c->rscore, ni * s.cap)) != cudaSuccess ||
-      (e = dmalloc(&c->rope, static_cast<size_t>(s.W + 1) * (s.d / 2))) != cudaSuccess ||
+      (e = dmalloc(&c->rope, static_cast<size_t>(s.W + 1) * (s.d / 2) * 3 / 2 + 1)) != cudaSuccess ||
       (e = dmalloc(&c->err, 1)) != cudaSuccess) {
     const int code = (e == cudaErrorMemoryAllocation) ? BKV_ENOMEM : BKV_ECUDA;
     cudaGetLastError();
@@ -254,7 +254,7 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
     delete c;
     return BKV_ECUDA;
   }
-  c->rope_host.resize(static_cast<size_t>(s.W + 1) * (s.d / 2));
+  c->rope_host.resize(static_cast<size_t>(s.W + 1) * (s.d / 2) * 3 / 2 + 1);
   *out = c;
   return BKV_OK;
 }
@@ -345,15 +345,19 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
   const double theta = ctx->cfg.rope_theta;
   const int rotate = theta != 0.0;
   if (rotate) {
+    const size_t n = static_cast<size_t>(s.W + 1) * h;
+    float2* tab32 = reinterpret_cast<float2*>(ctx->rope_host.data() + n);
     for (int slot = 0; slot <= s.W; ++slot) {
       const double pos = static_cast<double>(slot < s.W ? recent_pos[slot] : t_pos);
       for (int i = 0; i < h; ++i) {
         const double inv_freq = std::pow(theta, -static_cast<double>(2 * i) / static_cast<double>(s.d));
         const double ang = pos * inv_freq;
-        ctx->rope_host[static_cast<size_t>(slot) * h + i] = make_double2(std::cos(ang), std::sin(ang));
+        const double c = std::cos(ang), sn = std::sin(ang);
+        ctx->rope_host[static_cast<size_t>(slot) * h + i] = make_double2(c, sn);
+        tab32[static_cast<size_t>(slot) * h + i] = make_float2(static_cast<float>(c), static_cast<float>(sn));
       }
     }
-    e = cudaMemcpyAsync(ctx->rope, ctx->rope_host.data(), sizeof(double2) * ctx->rope_host.size(),
+    e = cudaMemcpyAsync(ctx->rope, ctx->rope_host.data(), sizeof(double2) * n + sizeof(float2) * n,
                         cudaMemcpyHostToDevice, ctx->stream);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "rope table upload");
   }

@@ -36,7 +36,8 @@ cudaError_t launch_update(const Shape& s, const __nv_bfloat16* q_new, int n_new,
                           long long* counts, int* assign_out, cudaStream_t st);
 
 // ---- compression (k_qobs.cu, k_score.cu, k_select_gather.cu)
-// rope: [W + 1][d / 2] (cos, sin) pairs; entry w < W is recent slot w, entry W
+// rope: [W + 1][d / 2] fp64 (cos, sin) pairs, immediately followed by the same
+// [W + 1][d / 2] table as fp32 pairs; entry w < W is recent slot w, entry W
 // is the beacon position.  rotate == 0 leaves vectors unrotated.
 cudaError_t launch_qobs(const Shape& s, const __nv_bfloat16* q_recent, const float* cent, const long long* counts,
                         const double2* rope, int rotate, __nv_bfloat16* qobs, uint32_t* valid, cudaStream_t st);

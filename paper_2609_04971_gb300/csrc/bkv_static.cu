@@ -144,7 +144,7 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
   const size_t off_valid = off_qobs + align256(sizeof(__nv_bfloat16) * s.n_inst * s.n_obs_pad * s.d);
   const size_t off_score = off_valid + align256(sizeof(uint32_t) * 4 * s.n_inst);
   const size_t off_rope = off_score + align256(sizeof(float) * static_cast<size_t>(s.n_inst) * s.cap);
-  const size_t need = off_rope + align256(sizeof(double2) * static_cast<size_t>(s.W + 1) * (s.d / 2));
+  const size_t need = off_rope + align256((sizeof(double2) + sizeof(float2)) * static_cast<size_t>(s.W + 1) * (s.d / 2));
   if (need > kStaticScratchBytes) {
     char buf[160];
     std::snprintf(buf, sizeof buf, "needs %zu bytes of scratch; the static scratch holds %zu", need,
@@ -183,17 +183,22 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
   const double theta = cfg->rope_theta;
   const int rotate = theta != 0.0;
   if (rotate) {
-    double2 tab[(bkv::kMaxWindow + 1) * 64];
+    // fp64 (cos, sin) entries followed by the same entries in fp32
+    double2 tab[(bkv::kMaxWindow + 1) * 64 * 3 / 2];
+    const size_t n = static_cast<size_t>(s.W + 1) * h;
+    float2* tab32 = reinterpret_cast<float2*>(tab + n);
     for (int slot = 0; slot <= s.W; ++slot) {
       const double pos = static_cast<double>(slot < s.W ? recent_pos[slot] : t_pos);
       for (int i = 0; i < h; ++i) {
         const double inv_freq = std::pow(theta, -static_cast<double>(2 * i) / static_cast<double>(s.d));
         const double ang = pos * inv_freq;
-        tab[slot * h + i] = make_double2(std::cos(ang), std::sin(ang));
+        const double c = std::cos(ang), sn = std::sin(ang);
+        tab[slot * h + i] = make_double2(c, sn);
+        tab32[slot * h + i] = make_float2(static_cast<float>(c), static_cast<float>(sn));
       }
     }
     // pageable source: the copy has consumed `tab` when the call returns
-    if ((e = cudaMemcpyAsync(rope, tab, sizeof(double2) * (s.W + 1) * h, cudaMemcpyHostToDevice, st)) !=
+    if ((e = cudaMemcpyAsync(rope, tab, (sizeof(double2) + sizeof(float2)) * n, cudaMemcpyHostToDevice, st)) !=
         cudaSuccess) {
       message(err_msg, err_len, cudaGetErrorString(e));
       return BKV_ECUDA;

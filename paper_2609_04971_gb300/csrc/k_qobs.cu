@@ -7,10 +7,18 @@
 // valid [n_inst][4] is a 128-bit mask of rows that take part in the maximum
 // (all recent rows, beacons with count > 0).
 //
-// The rotation y_i = x_i c - x_{i+d/2} s, y_{i+d/2} = x_{i+d/2} c + x_i s is
-// evaluated in fp64 with separately rounded products (no fused
-// multiply-add) from host-computed fp64 cos / sin, then rounded fp64 -> fp32
-// -> bf16, so every scoring query is the correctly defined bf16 value.
+// Definition of each output element: y_i = x_i c - x_{i+d/2} s and
+// y_{i+d/2} = x_{i+d/2} c + x_i s evaluated in fp64 (separately rounded
+// products, host-computed fp64 cos / sin), then rounded fp64 -> fp32 -> bf16.
+// The kernel first evaluates y in fp32 (one FMA, fp32 copies of cos / sin).
+// The fp32 value v differs from the fp64 one by at most
+//   delta = 2^-22 (|x_a| + |x_b| + |v|)
+// (rounding of cos and sin to fp32, of the product and of the FMA, with a
+// factor 2 of margin).  The composite rounding can only change where the fp32
+// value crosses a bf16 rounding midpoint (low 16 bits 0x8000) or lands within
+// one fp32 ulp of it; if v is farther than delta + 1 ulp from the nearest
+// midpoint, bf16(v) is the defined value.  Otherwise (about 2e-4 of the
+// elements) the element is recomputed in fp64 exactly as defined.
 #include "bkv_device.cuh"
 #include "bkv_internal.h"
 
@@ -19,6 +27,28 @@ namespace {
 
 constexpr int kQobsThreads = 256;
 
+// Exact definition: fp64 products, fp64 sum, then fp32, then bf16.
+__device__ __forceinline__ __nv_bfloat16 rot_exact(double xa, double xb, double c, double s, bool plus) {
+  const double y = plus ? __dadd_rn(__dmul_rn(xa, c), __dmul_rn(xb, s)) : __dsub_rn(__dmul_rn(xa, c), __dmul_rn(xb, s));
+  return __float2bfloat16_rn(__double2float_rn(y));
+}
+
+// bf16 of (xa*c +- xb*s) through the fp32 fast path when provably equal to the definition.
+__device__ __forceinline__ __nv_bfloat16 rot_fast(float xa, float xb, float c32, float s32, double c, double s,
+                                                   bool plus) {
+  const float p = xb * s32;
+  const float v = fmaf(xa, c32, plus ? p : -p);
+  const uint32_t t = __float_as_uint(v);
+  const uint32_t ex = t & 0x7f800000u;
+  if (ex >= (25u << 23) && ex != 0x7f800000u) {
+    const float ulp = __uint_as_float(ex - (23u << 23));
+    const float delta = 0x1p-22f * (fabsf(xa) + fabsf(xb) + fabsf(v));
+    const int dist = abs(static_cast<int>(t & 0xffffu) - 0x8000);
+    if (static_cast<float>(dist - 1) * ulp > delta) return __float2bfloat16_rn(v);
+  }
+  return rot_exact(xa, xb, c, s, plus);
+}
+
 __global__ void __launch_bounds__(kQobsThreads) qobs_kernel(Shape s, const __nv_bfloat16* __restrict__ q_recent,
                                                              const float* __restrict__ cent,
                                                              const long long* __restrict__ counts,
@@ -26,37 +56,48 @@ __global__ void __launch_bounds__(kQobsThreads) qobs_kernel(Shape s, const __nv_
                                                              __nv_bfloat16* __restrict__ qobs,
                                                              uint32_t* __restrict__ valid) {
   const int e = blockIdx.x;
-  const int d = s.d, h = d / 2;
+  const int d = s.d, h = d / 2, h4 = h / 4;
   const int GW = s.G * s.W;
+  const float2* rope32 = reinterpret_cast<const float2*>(rope + static_cast<size_t>(s.W + 1) * h);
   __nv_bfloat16* out = qobs + static_cast<size_t>(e) * s.n_obs_pad * d;
-  for (int idx = threadIdx.x; idx < s.n_obs_pad * h; idx += blockDim.x) {
-    const int row = idx / h, i = idx % h;
-    float y1 = 0.f, y2 = 0.f;
-    if (row < s.n_obs) {
-      double x1, x2;
-      int slot;
-      if (row < GW) {
-        const __nv_bfloat16* src = q_recent + (static_cast<size_t>(e) * GW + row) * d;
-        x1 = __bfloat162float(src[i]);
-        x2 = __bfloat162float(src[i + h]);
-        slot = row % s.W;
+  for (int idx = threadIdx.x; idx < s.n_obs_pad * h4; idx += blockDim.x) {
+    const int row = idx / h4, i = (idx % h4) * 4;
+    float xa[4] = {0.f, 0.f, 0.f, 0.f}, xb[4] = {0.f, 0.f, 0.f, 0.f};
+    int slot = 0;
+    if (row < GW) {
+      const __nv_bfloat16* src = q_recent + (static_cast<size_t>(e) * GW + row) * d;
+      const uint2 a = *reinterpret_cast<const uint2*>(src + i);
+      const uint2 b = *reinterpret_cast<const uint2*>(src + i + h);
+      const float2 a0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&a.x));
+      const float2 a1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&a.y));
+      const float2 b0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&b.x));
+      const float2 b1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&b.y));
+      xa[0] = a0.x; xa[1] = a0.y; xa[2] = a1.x; xa[3] = a1.y;
+      xb[0] = b0.x; xb[1] = b0.y; xb[2] = b1.x; xb[3] = b1.y;
+      slot = row % s.W;
+    } else if (row < s.n_obs) {
+      const float* src = cent + (static_cast<size_t>(e) * s.nb + (row - GW)) * d;
+      const float4 a = *reinterpret_cast<const float4*>(src + i);
+      const float4 b = *reinterpret_cast<const float4*>(src + i + h);
+      xa[0] = a.x; xa[1] = a.y; xa[2] = a.z; xa[3] = a.w;
+      xb[0] = b.x; xb[1] = b.y; xb[2] = b.z; xb[3] = b.w;
+      slot = s.W;
+    }
+    __nv_bfloat16 y1[4], y2[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      if (row < s.n_obs && rotate) {
+        const double2 cs = rope[slot * h + i + k];
+        const float2 cs32 = rope32[slot * h + i + k];
+        y1[k] = rot_fast(xa[k], xb[k], cs32.x, cs32.y, cs.x, cs.y, false);
+        y2[k] = rot_fast(xb[k], xa[k], cs32.x, cs32.y, cs.x, cs.y, true);
       } else {
-        const float* src = cent + (static_cast<size_t>(e) * s.nb + (row - GW)) * d;
-        x1 = src[i];
-        x2 = src[i + h];
-        slot = s.W;
-      }
-      if (rotate) {
-        const double2 cs = rope[slot * h + i];
-        y1 = __double2float_rn(__dsub_rn(__dmul_rn(x1, cs.x), __dmul_rn(x2, cs.y)));
-        y2 = __double2float_rn(__dadd_rn(__dmul_rn(x2, cs.x), __dmul_rn(x1, cs.y)));
-      } else {
-        y1 = static_cast<float>(x1);
-        y2 = static_cast<float>(x2);
+        y1[k] = __float2bfloat16_rn(xa[k]);
+        y2[k] = __float2bfloat16_rn(xb[k]);
       }
     }
-    out[row * d + i] = __float2bfloat16_rn(y1);
-    out[row * d + i + h] = __float2bfloat16_rn(y2);
+    *reinterpret_cast<uint2*>(out + row * d + i) = *reinterpret_cast<const uint2*>(y1);
+    *reinterpret_cast<uint2*>(out + row * d + i + h) = *reinterpret_cast<const uint2*>(y2);
   }
   if (threadIdx.x < 4) {
     uint32_t m = 0;

@@ -1,5 +1,5 @@
 // Selection (Eq. 7 with the keep set of Algorithm 2) and in-place compaction
-// of K and V (Eq. 8), one CTA of 512 threads per instance.
+// of K and V (Eq. 8), one CTA of 256 threads per instance.
 //
 // Selection: the log2 scores of the candidates [n_prefix, L - W) are mapped to
 // order-preserving uint32 keys in shared memory; a 4-pass MSB-first radix
@@ -16,14 +16,15 @@
 // chunk's loads only touch rows at or beyond its own first destination,
 // which no earlier chunk writes.  Rows below the first evicted row already
 // hold their final contents and are skipped.  Transfers are 16-byte vectors,
-// coalesced along each 2*d-byte row.
+// coalesced along each 2*d-byte row; the kept indices are read from shared
+// memory (they overwrite the score keys once compaction has consumed them).
 #include "bkv_device.cuh"
 #include "bkv_internal.h"
 
 namespace bkv {
 namespace {
 
-constexpr int kSgThreads = 512;
+constexpr int kSgThreads = 256;
 constexpr int kSgWarps = kSgThreads / 32;
 
 // Exclusive block-wide prefix count of `flag`; also returns the block total.
@@ -125,6 +126,8 @@ __global__ void __launch_bounds__(kSgThreads) select_gather_kernel(Shape s, cons
   const int k_ties = k_sel > 0 ? static_cast<int>(sh_k) : 0;
 
   // ---------------------------------------------------------------- index-order compaction
+  // kept indices go to global memory and, in place of the consumed keys, to shared memory
+  int* kept_s = reinterpret_cast<int*>(keys);
   int run_tie = 0, run_keep = 0;
   for (int base = 0; base < L; base += kSgThreads) {
     const int j = base + tid;
@@ -133,14 +136,16 @@ __global__ void __launch_bounds__(kSgThreads) select_gather_kernel(Shape s, cons
     const uint32_t key = cand ? keys[j] : 0u;
     const bool tie = cand && key == T;
     int tie_excl, tie_total;
-    block_count_scan(tie, wsum, tie_excl, tie_total);
+    block_count_scan(tie, wsum, tie_excl, tie_total);  // also orders every read of keys[base..] before the writes
     const bool keep = in && (!cand || key > T || (tie && run_tie + tie_excl < k_ties));
     int keep_excl, keep_total;
     block_count_scan(keep, wsum, keep_excl, keep_total);
-    if (keep)
+    if (keep) {
       kept_e[run_keep + keep_excl] = j;
-    else if (in)
+      kept_s[run_keep + keep_excl] = j;  // position <= j: that key has been read already
+    } else if (in) {
       atomicMin(&sh_first_evicted, j);
+    }
     run_tie += tie_total;
     run_keep += keep_total;
   }
@@ -149,36 +154,28 @@ __global__ void __launch_bounds__(kSgThreads) select_gather_kernel(Shape s, cons
   // ---------------------------------------------------------------- in-place gather
   constexpr int kVpr = D * 2 / 16;                 // 16-byte vectors per row of one tensor
   constexpr int kRowVec = 2 * kVpr;                // K row then V row
-  constexpr int kPer = 4;                          // vectors per thread per chunk
-  constexpr int kChunkRows = kSgThreads * kPer / kRowVec;
-  uint4* Kb = reinterpret_cast<uint4*>(K + static_cast<size_t>(e) * s.cap * D);
-  uint4* Vb = reinterpret_cast<uint4*>(V + static_cast<size_t>(e) * s.cap * D);
+  constexpr int kPer = 8;                          // vectors per thread per chunk
+  constexpr int kRowsPerPass = kSgThreads / kRowVec;
+  constexpr int kChunkRows = kRowsPerPass * kPer;
+  const int col = tid % kRowVec;                   // fixed 16-byte column of this thread
+  const int row0 = tid / kRowVec;                  // first row of this thread inside a chunk
+  uint4* base_t = reinterpret_cast<uint4*>((col < kVpr ? K : V) + static_cast<size_t>(e) * s.cap * D) +
+                  (col < kVpr ? col : col - kVpr);
   const int first = sh_first_evicted;
 
   uint4 cur[kPer], nxt[kPer];
   auto load_chunk = [&](int i0, uint4 (&R)[kPer]) {
 #pragma unroll
     for (int u = 0; u < kPer; ++u) {
-      const int v = tid + kSgThreads * u;
-      const int row = i0 + v / kRowVec, col = v % kRowVec;
-      if (row < budget) {
-        const int src = __ldcg(kept_e + row);
-        const uint4* p = col < kVpr ? Kb + static_cast<size_t>(src) * kVpr + col
-                                    : Vb + static_cast<size_t>(src) * kVpr + (col - kVpr);
-        R[u] = __ldcg(p);
-      }
+      const int row = i0 + row0 + kRowsPerPass * u;
+      if (row < budget) R[u] = __ldcg(base_t + static_cast<size_t>(kept_s[row]) * kVpr);
     }
   };
   auto store_chunk = [&](int i0, const uint4 (&R)[kPer]) {
 #pragma unroll
     for (int u = 0; u < kPer; ++u) {
-      const int v = tid + kSgThreads * u;
-      const int row = i0 + v / kRowVec, col = v % kRowVec;
-      if (row < budget) {
-        uint4* p = col < kVpr ? Kb + static_cast<size_t>(row) * kVpr + col
-                              : Vb + static_cast<size_t>(row) * kVpr + (col - kVpr);
-        *p = R[u];
-      }
+      const int row = i0 + row0 + kRowsPerPass * u;
+      if (row < budget) base_t[static_cast<size_t>(row) * kVpr] = R[u];
     }
   };
   if (first < budget) load_chunk(first, cur);
