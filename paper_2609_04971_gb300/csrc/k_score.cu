@@ -2,51 +2,63 @@
 // form, maximum over the GQA group's observation queries; Section 4.3).
 //
 // Persistent kernel, one CTA per SM.  Instances are processed by
-// thread-block clusters of C CTAs (C = 1 or more, chosen from the cache
-// length); cluster k takes instances k, k + n_clusters, ...; CTA r of a
-// cluster owns the same contiguous range of 128-key tiles of every instance.
-// Each CTA is warp-specialised:
-//   warp 0      TMA producer: per instance the observation queries (into one
-//               of two buffers) and the CTA's K tiles (128 keys x d, 128-byte
-//               swizzle) twice, through a ring of shared-memory stages;
-//   warp 1      allocates TMEM and issues tcgen05.mma (bf16 x bf16 -> fp32):
-//               D = K_tile x Qobs^T, M = 128 keys (TMEM lanes), N = padded
-//               query count (TMEM columns), for both passes;
-//   warps 2..9  two epilogue groups of four warps (one TMEM lane quarter
-//               per warp).  With at most 64 query columns the groups take
-//               alternate tiles; with more, both read every tile of pass 1
-//               and each group owns 64 query columns.
-// Pass 1: each thread owns one key of the tile and keeps, for every query
-// column it owns, a running maximum m_q and sum s_q of 2^(y - m_q) over the
-// keys it has seen (y = logit * log2(e), one ex2 per element).  At the end of
-// the CTA's tiles the per-thread partials are merged (recursive halving
-// inside each warp, then shared memory across warps and groups) and the CTAs
-// of a cluster exchange theirs through distributed shared memory; every CTA
-// combines them in rank order, giving the same lse2_q = log2 sum_j 2^(y_qj)
-// over all L keys.  Pass 2 recomputes the tile (the K bytes are still in L2)
-// and takes r_j = max over valid q of (y_qj - lse2_q) = log2 Score_j.
+// thread-block clusters of C CTAs; cluster k takes instances k,
+// k + n_clusters, ...; CTA r of a cluster owns the same contiguous range of
+// 128-key tiles of every instance.
 //
-// Cross-CTA protocol (all waits bounded): barriers are initialised, then a
-// cluster barrier.  Per instance each CTA publishes its partials and arrives
-// on every peer's `part_ready`; after reading every peer it arrives on every
-// peer's `read_done`; it overwrites its partials for the next instance only
-// after its own `read_done` phase completed.  The exchange runs for every
-// instance even after a timeout, and the kernel ends with a cluster barrier,
-// so no CTA leaves while a peer may still touch its shared memory.
-// Outputs: r (log2 scores, for selection) and optionally Score = 2^r.
+// Each tile goes through the tensor cores once: D = K_tile x Qobs^T with
+// M = 128 keys (TMEM lanes) and N = padded query count (TMEM columns),
+// bf16 x bf16 -> fp32 (tcgen05.mma, operands staged by TMA with 128-byte
+// swizzle).  The fp32 logits of every tile a CTA owns stay resident in
+// tensor memory, in a ring of N-column slots that successive instances fill
+// in turn (slots left over by one instance let the next one's tiles land
+// while it finishes), so K is read from HBM exactly once.  y = logit * log2(e) is the base-2 logit.
+//   Pass 1 (statistics, as tiles land): each thread owns one key of the tile
+//     and keeps, for the query columns it owns, a running maximum m_q and sum
+//     s_q of 2^(y - m_q).  After the CTA's last tile the partials are merged
+//     (recursive halving inside each warp, shared memory across warps) and
+//     the CTAs of a cluster exchange theirs through distributed shared memory;
+//     every CTA combines them in rank order and gets the same
+//     lse2_q = log2 sum_j 2^(y_qj) over all L keys.
+//   Pass 2 (scores, from tensor memory): r_j = max over valid q of
+//     (y_qj - lse2_q) = log2 Score_j.
+// When a CTA owns more tiles than tensor memory holds (very long caches), the
+// tiles past the resident ones cycle through two streaming slots in pass 1
+// and are loaded and multiplied a second time for pass 2, into one slot per
+// pass-2 warp half.  Every slot barrier thus has a fixed set of warps that
+// waits on each of its uses in order, which keeps the parity waits exact.
+//
+// Warp roles (10 warps): warp 0 TMA producer (queries into one of two
+// buffers, K tiles through a ring of shared-memory stages); warp 1 TMEM
+// allocation and MMA issue; warps 2..9 epilogue, two warps per TMEM lane
+// quarter: in pass 1 each owns half of the query columns, in pass 2 each
+// takes every other tile with all columns.
+//
+// Cross-CTA exchange (all waits bounded): barriers are initialised, then a
+// cluster barrier.  Per instance every CTA pushes its (m, s) column partials
+// into each peer's receive buffer with st.async, whose bytes complete on the
+// peer's receive barrier; the receiver arms that barrier with the byte count
+// of all csize senders.  Receive buffers and barriers alternate between two
+// copies by instance parity: a sender can be at most one instance ahead of
+// any receiver, since it needs every peer's partials of the instance before.
+// No release fence at cluster scope sits on this path (one would wait for the
+// CTA's score stores, queued behind the K stream).  The exchange runs for
+// every instance even after a timeout, and the kernel ends with a cluster
+// barrier, so no CTA leaves while a peer may still write to its shared memory.
+// Outputs: r (log2 scores, for selection) and optionally 2^r.
 #include "bkv_device.cuh"
 #include "bkv_internal.h"
 
 namespace bkv {
 namespace {
 
-constexpr int kEpiGroups = 2;
-constexpr int kScThreads = 64 + 128 * kEpiGroups;
-constexpr int kTile = 128;                 // keys per tile (MMA M)
-constexpr uint32_t kBoxBytes = 128 * 128;  // [128 rows][64 bf16] swizzled box
-constexpr int kAcc = 4;                    // fp32 accumulators of 128 TMEM columns each
-constexpr uint32_t kTmemCols = 128 * kAcc;
+constexpr int kEpiWarps = 8;
+constexpr int kScThreads = 32 * (2 + kEpiWarps);
+constexpr int kTile = 128;                  // keys per tile (MMA M)
+constexpr uint32_t kBoxBytes = 128 * 128;   // [128 rows][64 bf16] swizzled box
+constexpr uint32_t kTmemCols = 512;
 constexpr int kMaxStages = 12;
+constexpr int kMaxSlots = 32;               // tensor-memory slots (resident + streaming)
 constexpr size_t kSmemBudget = 220 * 1024;  // dynamic shared memory of the one CTA per SM
 
 template <int D>
@@ -54,15 +66,27 @@ struct ScoreCfg {
   static constexpr int kBoxes = D / 64;                  // 64-column boxes per row
   static constexpr uint32_t kTileBytes = kTile * D * 2;  // one K tile
   static size_t q_bytes(int n_obs_pad) { return 2 * static_cast<size_t>(kBoxes) * n_obs_pad * 128; }
-  // as many K stages as fit next to the two query buffers
-  static int stages(int n_obs_pad) {
-    const size_t room = kSmemBudget - 1024 - q_bytes(n_obs_pad);
+  // two receive buffers of csize x n_obs_pad (m, s) pairs
+  static size_t recv_bytes(int n_obs_pad, int csize) {
+    return csize > 1 ? 2 * static_cast<size_t>(csize) * n_obs_pad * 8 : 0;
+  }
+  // as many K stages as fit next to the query and receive buffers
+  static int stages(int n_obs_pad, int csize) {
+    const size_t room = kSmemBudget - 1024 - q_bytes(n_obs_pad) - recv_bytes(n_obs_pad, csize);
     const int n = static_cast<int>(room / (static_cast<size_t>(kBoxes) * kBoxBytes));
     return n < kMaxStages ? n : kMaxStages;
   }
-  static size_t smem_bytes(int n_obs_pad) {
-    return 1024 + q_bytes(n_obs_pad) + static_cast<size_t>(stages(n_obs_pad)) * kBoxes * kBoxBytes;
+  static size_t smem_bytes(int n_obs_pad, int csize) {
+    return 1024 + q_bytes(n_obs_pad) + static_cast<size_t>(stages(n_obs_pad, csize)) * kBoxes * kBoxBytes +
+           recv_bytes(n_obs_pad, csize);
   }
+};
+
+// Placement of one instance's tiles: cluster size and resident ring slots;
+// `stream` adds four streaming slots after the ring (two rotating pass-1
+// slots, one pass-2 slot per epilogue half).
+struct Plan {
+  int csize, slots, stream;
 };
 
 // Wait used while draining after an abort: ignores the abort flag.
@@ -71,8 +95,24 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* 
   mbar_wait(bar, parity, &never, err, kDevTimeoutDrain);
 }
 
-__device__ __forceinline__ void mbar_arrive_n(uint64_t* bar, uint32_t n) {
-  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(n) : "memory");
+// Read-only global load emitted exactly here (the compiler may not sink it
+// towards its first use, where its latency behind the K stream would show).
+__device__ __forceinline__ uint32_t ld_nc_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.global.nc.u32 %0, [%1];" : "=r"(v) : "l"(p));
+  return v;
+}
+
+// Asynchronous store of (m, s) into a peer CTA's shared memory; its 8 bytes
+// complete on the peer's barrier `bar` (both shared::cluster addresses).
+__device__ __forceinline__ void st_async_pair(uint32_t dst, float m, float s, uint32_t bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(dst),
+               "f"(m), "f"(s), "r"(bar)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_cnt(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
 }
 
 // Merge of two base-2 log-sum-exp partials (m, s) -> (max, rescaled sum).
@@ -84,46 +124,98 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2
   s = a + b;
 }
 
-// Recursive-halving merge across the 32 lanes of a warp for NQ columns held
-// by every lane; afterwards lane l holds the warp's merge of columns
-// l * (NQ / 32) .. + NQ / 32 - 1 in m[0 .. NQ/32 - 1], s[...].
+// Merge of NQ per-lane column partials across the 32 lanes of a warp.  Steps
+// halve the columns a lane holds while their count is even and exchange all of
+// them otherwise.  Returns the first column of the lane's result block (the
+// block is m[0 .. count-1]); `writer` is true for one lane per block.
 template <int NQ>
-__device__ __forceinline__ void warp_reduce_scatter(float (&m)[NQ], float (&s)[NQ], int lane) {
+__device__ __forceinline__ int warp_merge_columns(float (&m)[NQ], float (&s)[NQ], int lane, bool& writer) {
+  int first = 0;
+  writer = true;
+  int cols = NQ;
 #pragma unroll
-  for (int half = NQ / 2, o = 16; half >= NQ / 32; half /= 2, o /= 2) {
-    const bool upper = (lane & o) != 0;  // keeps the upper half of its current columns
+  for (int o = 16; o >= 1; o >>= 1) {
+    if (cols % 2 == 0) {
+      const int half = cols / 2;
+      const bool upper = (lane & o) != 0;
 #pragma unroll
-    for (int i = 0; i < half; ++i) {
-      const float send_m = upper ? m[i] : m[i + half];
-      const float send_s = upper ? s[i] : s[i + half];
-      const float keep_m = upper ? m[i + half] : m[i];
-      const float keep_s = upper ? s[i + half] : s[i];
-      const float got_m = __shfl_xor_sync(0xffffffffu, send_m, o);
-      const float got_s = __shfl_xor_sync(0xffffffffu, send_s, o);
-      m[i] = keep_m;
-      s[i] = keep_s;
-      lse_merge(m[i], s[i], got_m, got_s);
+      for (int i = 0; i < NQ / 2; ++i) {
+        if (i < half) {
+          const float send_m = upper ? m[i] : m[i + half];
+          const float send_s = upper ? s[i] : s[i + half];
+          const float keep_m = upper ? m[i + half] : m[i];
+          const float keep_s = upper ? s[i + half] : s[i];
+          const float got_m = __shfl_xor_sync(0xffffffffu, send_m, o);
+          const float got_s = __shfl_xor_sync(0xffffffffu, send_s, o);
+          m[i] = keep_m;
+          s[i] = keep_s;
+          lse_merge(m[i], s[i], got_m, got_s);
+        }
+      }
+      if (upper) first += half;
+      cols = half;
+    } else {
+#pragma unroll
+      for (int i = 0; i < NQ; ++i) {
+        if (i < cols) {
+          const float got_m = __shfl_xor_sync(0xffffffffu, m[i], o);
+          const float got_s = __shfl_xor_sync(0xffffffffu, s[i], o);
+          lse_merge(m[i], s[i], got_m, got_s);
+        }
+      }
+      if (lane & o) writer = false;
     }
   }
+  return first;
+}
+
+// r = max over the N columns of (v * sc - lse2), columns read from tensor
+// memory in chunks of 32 (16 for a ragged last chunk).
+template <int N>
+__device__ __forceinline__ float tile_score(uint32_t taddr, const float* lse2, float sc) {
+  float r0 = -INFINITY, r1 = -INFINITY;
+#pragma unroll
+  for (int c0 = 0; c0 < N; c0 += 32) {
+    float v[32];
+    if (c0 + 32 <= N) {
+      tmem_ld32(taddr + c0, v);
+    } else {
+      tmem_ld16(taddr + c0, v);
+    }
+    tmem_wait_ld();
+#pragma unroll
+    for (int u = 0; u < 32; u += 4) {
+      if (c0 + u < N) {
+        const float4 l = *reinterpret_cast<const float4*>(lse2 + c0 + u);
+        r0 = fmaxf(r0, fmaf(v[u], sc, -l.x));
+        r1 = fmaxf(r1, fmaf(v[u + 1], sc, -l.y));
+        r0 = fmaxf(r0, fmaf(v[u + 2], sc, -l.z));
+        r1 = fmaxf(r1, fmaf(v[u + 3], sc, -l.w));
+      }
+    }
+  }
+  return fmaxf(r0, r1);
 }
 
 template <int D, int NQ>
 __global__ void __launch_bounds__(kScThreads, 1)
     score_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap, Shape s,
-                 ScoreArgs a, int csize, int n_stages) {
+                 ScoreArgs a, Plan plan, int n_stages) {
   using C = ScoreCfg<D>;
-  constexpr int kPer = NQ / 32;  // columns per lane after the warp merge
+  constexpr int N = 2 * NQ;  // padded query columns
+  static_assert(NQ % 8 == 0 && NQ <= 64, "query columns per pass-1 warp");
   extern __shared__ unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kMaxStages], empty_bar[kMaxStages];
-  __shared__ __align__(8) uint64_t accf_bar[kAcc], acce_bar[kAcc], qfull_bar[2], qempty_bar[2], drain_bar;
-  __shared__ __align__(8) uint64_t part_ready_bar, read_done_bar;
+  __shared__ __align__(8) uint64_t slot_full[kMaxSlots], slot_free[kMaxSlots];
+  __shared__ __align__(8) uint64_t qfull_bar[2], qempty_bar[2], drain_bar;
+  __shared__ __align__(8) uint64_t recv_bar[2];
   __shared__ uint32_t tmem_base_sh;
   __shared__ int abort_sh;
-  __shared__ float lse2_sh[128];
-  __shared__ float part_m[128], part_s[128];
-  __shared__ float wred_m[kEpiGroups * 4][64], wred_s[kEpiGroups * 4][64];
+  __shared__ __align__(16) float lse2_sh[128];
+  __shared__ float wred_m[kEpiWarps][64], wred_s[kEpiWarps][64];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int csize = plan.csize;
   const int crank = csize > 1 ? static_cast<int>(cluster_ctarank()) : 0;
   const int cluster_id = blockIdx.x / csize;
   const int n_clusters = gridDim.x / csize;
@@ -131,30 +223,34 @@ __global__ void __launch_bounds__(kScThreads, 1)
   const int T_all = (a.L + kTile - 1) / kTile;
   const int t0 = crank * T_all / csize;
   const int T = (crank + 1) * T_all / csize - t0;  // tiles this CTA owns in every instance
+  const int R = T < plan.slots ? T : plan.slots;     // resident tiles
+  const int n_str = T - R;                           // streaming tiles (plan.stream only)
+  const int ring = plan.slots;                       // resident slots, used in cyclic order
+  const int str_slot = ring;                         // pass-1 streaming slots; +2, +3: pass-2 slots
   const uint32_t qbox = static_cast<uint32_t>(s.n_obs_pad) * 128;
-  const bool split = s.n_obs_pad > 64;  // pass 1: both groups read every tile, 64 columns each
 
   unsigned char* base = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   unsigned char* q_smem = base;                         // [2 buffers][kBoxes][n_obs_pad rows x 128 B]
   unsigned char* k_smem = base + 2 * C::kBoxes * qbox;  // [n_stages][kBoxes][128 rows x 128 B]
+  float2* recv = reinterpret_cast<float2*>(k_smem + n_stages * C::kBoxes * kBoxBytes);  // [2][csize][N]
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < n_stages; ++i) {
       mbar_init(&full_bar[i], 1);
       mbar_init(&empty_bar[i], 1);
     }
-    for (int i = 0; i < kAcc; ++i) {
-      mbar_init(&accf_bar[i], 1);
-      mbar_init(&acce_bar[i], split ? 8 : 4);  // warp arrivals that free an accumulator
+    for (int i = 0; i < kMaxSlots; ++i) {
+      mbar_init(&slot_full[i], 1);
+      mbar_init(&slot_free[i], kEpiWarps);  // eight warp arrivals per use
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&qfull_bar[i], 1);
       mbar_init(&qempty_bar[i], 1);
     }
     mbar_init(&drain_bar, 1);
-    mbar_init(&part_ready_bar, csize);
-    mbar_init(&read_done_bar, csize);
+    mbar_init(&recv_bar[0], 1);
+    mbar_init(&recv_bar[1], 1);
     abort_sh = 0;
     fence_mbar_init();
   }
@@ -169,43 +265,46 @@ __global__ void __launch_bounds__(kScThreads, 1)
   const uint32_t tmem = tmem_base_sh;
   volatile int* abort_flag = &abort_sh;
 
+  // Job order of an instance (producer, MMA and epilogue agree on it):
+  // pass-1 jobs for tiles 0 .. T-1, then pass-2 jobs for the streaming tiles.
   if (warp == 0) {
     // ---------------------------------------------------------------- producer
     if (lane == 0) {
-      const uint64_t keep = l2_policy_evict_last(), stream = l2_policy_evict_first();
+      const uint64_t once = l2_policy_evict_first(), again = l2_policy_evict_last();
       prefetch_tmap(&kmap);
       prefetch_tmap(&qmap);
-      int g = 0;  // ring iteration over all instances
+      int g = 0;  // ring iteration
       bool ok = true;
       int q_issued = 0;
-      for (int li = 0; ok && li < n_my; ++li) {
-        const int e = cluster_id + li * n_clusters;
-        const int qb = li & 1;
-        if (li >= 2 && !mbar_wait(&qempty_bar[qb], ((li >> 1) - 1) & 1, abort_flag, a.err, kDevTimeoutProducer)) {
+      for (int i = 0; ok && i < n_my; ++i) {
+        const int e = cluster_id + i * n_clusters;
+        const int qb = i & 1;
+        if (i >= 2 && !mbar_wait(&qempty_bar[qb], ((i >> 1) - 1) & 1, abort_flag, a.err, kDevTimeoutProducer)) {
           ok = false;
           break;
         }
         mbar_arrive_expect_tx(&qfull_bar[qb], static_cast<uint32_t>(s.n_obs_pad) * D * 2);
         for (int b = 0; b < C::kBoxes; ++b)
-          tma_load_2d(q_smem + (qb * C::kBoxes + b) * qbox, &qmap, &qfull_bar[qb], b * 64, e * s.n_obs_pad, keep);
-        q_issued = li + 1;
-        for (int it = 0; it < 2 * T; ++it, ++g) {
+          tma_load_2d(q_smem + (qb * C::kBoxes + b) * qbox, &qmap, &qfull_bar[qb], b * 64, e * s.n_obs_pad, again);
+        q_issued = i + 1;
+        for (int j = 0; j < T + n_str; ++j) {
+          const int t = j < T ? j : R + (j - T);
           const int st = g % n_stages;
           if (g >= n_stages &&
               !mbar_wait(&empty_bar[st], ((g / n_stages) - 1) & 1, abort_flag, a.err, kDevTimeoutProducer)) {
             ok = false;
             break;
           }
-          const int t = t0 + (it < T ? it : it - T);
           mbar_arrive_expect_tx(&full_bar[st], C::kTileBytes);
           for (int b = 0; b < C::kBoxes; ++b)
             tma_load_2d(k_smem + (st * C::kBoxes + b) * kBoxBytes, &kmap, &full_bar[st], b * 64,
-                        e * s.cap + t * kTile, it < T ? keep : stream);
+                        e * s.cap + (t0 + t) * kTile, (j < T && t >= R) ? again : once);
+          ++g;
         }
       }
       if (!ok || *abort_flag) {  // let every copy already issued land before the CTA exits
-        for (int li = (q_issued > 2 ? q_issued - 2 : 0); li < q_issued; ++li)
-          drain_wait(&qfull_bar[li & 1], (li >> 1) & 1, a.err);
+        for (int p = (q_issued > 2 ? q_issued - 2 : 0); p < q_issued; ++p)
+          drain_wait(&qfull_bar[p & 1], (p >> 1) & 1, a.err);
         for (int j = (g > n_stages ? g - n_stages : 0); j < g; ++j)
           drain_wait(&full_bar[j % n_stages], (j / n_stages) & 1, a.err);
       }
@@ -214,23 +313,35 @@ __global__ void __launch_bounds__(kScThreads, 1)
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      const uint32_t idesc = idesc_bf16_f32(128, s.n_obs_pad);
-      int g = 0, ga = 0;
+      const uint32_t idesc = idesc_bf16_f32(128, N);
+      int g = 0, ks = 0, kp2_0 = 0, kp2_1 = 0;  // pass-1 streaming uses; pass-2 uses per half
+      int rs = 0, ru = 0;                        // next ring slot and its use count
       bool ok = true;
-      for (int li = 0; ok && li < n_my; ++li) {
-        const int qb = li & 1;
-        if (!mbar_wait(&qfull_bar[qb], (li >> 1) & 1, abort_flag, a.err, kDevTimeoutMma)) break;
-        const uint32_t q_addr = smem_u32(q_smem + qb * C::kBoxes * qbox);
-        for (int it = 0; it < 2 * T; ++it, ++g, ++ga) {
-          const int st = g % n_stages, acc = ga % kAcc;
+      for (int i = 0; ok && i < n_my; ++i) {
+        if (!mbar_wait(&qfull_bar[i & 1], (i >> 1) & 1, abort_flag, a.err, kDevTimeoutMma)) break;
+        for (int j = 0; j < T + n_str; ++j) {
+          const int st = g % n_stages;
+          int slot, u;
+          if (j < R) {
+            slot = rs;
+            u = ru;
+          } else if (j < T) {
+            slot = str_slot + (ks & 1);
+            u = ks >> 1;
+          } else {
+            const int h = (j - T) & 1;
+            slot = str_slot + 2 + h;
+            u = h ? kp2_1 : kp2_0;
+          }
           if (!mbar_wait(&full_bar[st], (g / n_stages) & 1, abort_flag, a.err, kDevTimeoutMma) ||
-              (ga >= kAcc && !mbar_wait(&acce_bar[acc], ((ga / kAcc) - 1) & 1, abort_flag, a.err, kDevTimeoutMma))) {
+              (u >= 1 && !mbar_wait(&slot_free[slot], (u - 1) & 1, abort_flag, a.err, kDevTimeoutMma))) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem + acc * 128;
+          const uint32_t d_tmem = tmem + slot * N;
           const uint32_t k_addr = smem_u32(k_smem + st * C::kBoxes * kBoxBytes);
+          const uint32_t q_addr = smem_u32(q_smem + (i & 1) * C::kBoxes * qbox);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const uint32_t qoff = (kk >> 2) * qbox + (kk & 3) * 32;
@@ -238,9 +349,19 @@ __global__ void __launch_bounds__(kScThreads, 1)
             mma_bf16_ss(d_tmem, sdesc_kmajor_sw128(k_addr + koff), sdesc_kmajor_sw128(q_addr + qoff), idesc, kk > 0);
           }
           mma_commit(&empty_bar[st]);
-          mma_commit(&accf_bar[acc]);
+          mma_commit(&slot_full[slot]);
+          ++g;
+          if (j < R && ++rs == ring) {
+            rs = 0;
+            ++ru;
+          }
+          if (j >= T) {
+            if ((j - T) & 1) ++kp2_1;
+            else ++kp2_0;
+          }
+          else if (j >= R) ++ks;
         }
-        if (ok) mma_commit(&qempty_bar[qb]);  // this query buffer is free once its MMAs finish
+        if (ok) mma_commit(&qempty_bar[i & 1]);  // this instance's queries are no longer read
       }
       mma_commit(&drain_bar);  // every MMA issued above has finished once this arrives
       drain_wait(&drain_bar, 0, a.err);
@@ -248,139 +369,160 @@ __global__ void __launch_bounds__(kScThreads, 1)
     __syncwarp();
   } else {
     // ---------------------------------------------------------------- epilogue
-    const int group = (warp - 2) >> 2;
-    const int wig = warp & 3;                 // TMEM lane quarter of this warp
-    const int key_row = wig * 32 + lane;      // key of the tile owned by this thread
-    const uint32_t lane_addr = static_cast<uint32_t>(wig * 32) << 16;
-    const int col0 = split ? 64 * group : 0;  // first query column of this group in pass 1
-    const bool leader = threadIdx.x == 64;
-    const int n_epi = 128 * kEpiGroups;
-    const int wslot = group * 4 + wig;        // slot of this warp in the cross-warp merge
+    const int we = warp - 2;                 // 0 .. 7
+    const int quarter = warp & 3;            // TMEM lane quarter
+    const int half = we >> 2;                // pass 1: column half; pass 2: tile parity
+    const int key_row = quarter * 32 + lane;
+    const uint32_t lane_addr = static_cast<uint32_t>(quarter * 32) << 16;
+    const int te = threadIdx.x - 64;         // 0 .. 255
+    const bool leader = te == 0;
     const float sc = a.scale_log2;
-    int ga = 0;
-    for (int li = 0; li < n_my; ++li) {
-      const int e = cluster_id + li * n_clusters;
-
-      // ---- pass 1: per-thread running (max, sum) of every owned query column
+    int ks = 0, kp2 = 0;  // uses of the pass-1 streaming slots / of this half's pass-2 slot
+    int rs = 0, ru = 0;   // ring slot and use count of this instance's first tile
+    // valid-row words are fetched one instance ahead: a global load queues
+    // behind the K stream for microseconds
+    uint32_t vnext = (te < 128 && n_my > 0) ? ld_nc_u32(&a.valid[cluster_id * 4 + (te >> 5)]) : 0u;
+    for (int i = 0; i < n_my; ++i) {
+      const int e = cluster_id + i * n_clusters;
+      const uint32_t vword = vnext;
+      if (te < 128 && i + 1 < n_my) vnext = ld_nc_u32(&a.valid[(e + n_clusters) * 4 + (te >> 5)]);
       float m[NQ], sm[NQ];
 #pragma unroll
-      for (int i = 0; i < NQ; ++i) {
-        m[i] = -INFINITY;
-        sm[i] = 0.f;
+      for (int c = 0; c < NQ; ++c) {
+        m[c] = -INFINITY;
+        sm[c] = 0.f;
       }
-      for (int t = 0; t < T; ++t, ++ga) {
-        if (!split && (ga & 1) != group) continue;
-        const int acc = ga % kAcc;
-        const bool have = !*abort_flag &&
-                          mbar_wait(&accf_bar[acc], (ga / kAcc) & 1, abort_flag, a.err, kDevTimeoutEpilogue);
-        const bool key_ok = (t0 + t) * kTile + key_row < a.L;
-        if (have) tc_fence_after();
-#pragma unroll
-        for (int c = 0; c < NQ / 32; ++c) {
-          float v[32];
-          if (have) {
-            tmem_ld32(tmem + acc * 128 + col0 + c * 32 + lane_addr, v);
-            tmem_wait_ld();
+      bool resident_ok = true;
+      // ---- pass 1
+      for (int j = 0; j < T; ++j) {
+        int slot, u;
+        if (j < R) {
+          slot = rs + j;
+          u = ru;
+          if (slot >= ring) {
+            slot -= ring;
+            ++u;
           }
-          if (c == NQ / 32 - 1) {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&acce_bar[acc]);  // all columns are in registers
-          }
-          if (have && key_ok) {
+        } else {
+          slot = str_slot + (ks & 1);
+          u = ks >> 1;
+        }
+        bool have = !*abort_flag && mbar_wait(&slot_full[slot], u & 1, abort_flag, a.err, kDevTimeoutEpilogue);
+        have = __all_sync(0xffffffffu, have);
+        if (j < R) resident_ok = resident_ok && have;
+        float v[NQ];
+        if (have) {
+          tc_fence_after();
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float y = v[i] * sc;
-              const float dlt = y - m[c * 32 + i];
-              const float u = ex2_approx(-fabsf(dlt));
-              const bool up = dlt > 0.f;
-              sm[c * 32 + i] = up ? fmaf(sm[c * 32 + i], u, 1.f) : sm[c * 32 + i] + u;
-              m[c * 32 + i] = up ? y : m[c * 32 + i];
-            }
+          for (int c = 0; c < NQ; c += 8) {
+            uint32_t r[8];
+            asm volatile(
+                "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                : "r"(tmem + slot * N + half * NQ + c + lane_addr));
+#pragma unroll
+            for (int q = 0; q < 8; ++q) v[c + q] = __uint_as_float(r[q]);
+          }
+          tmem_wait_ld();
+        }
+        if (j >= R) {  // a streaming slot is free once every warp has its columns
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&slot_free[slot]);
+          ++ks;
+        }
+        if (have && (t0 + j) * kTile + key_row < a.L) {
+#pragma unroll
+          for (int c = 0; c < NQ; ++c) {
+            const float y = v[c] * sc;
+            const float dlt = y - m[c];
+            const float w = ex2_approx(-fabsf(dlt));
+            const bool up = dlt > 0.f;
+            sm[c] = up ? fmaf(sm[c], w, 1.f) : sm[c] + w;
+            m[c] = up ? y : m[c];
           }
         }
       }
 
-      // ---- merge: warp lanes, then warps and groups, then the CTAs of the cluster
-      warp_reduce_scatter<NQ>(m, sm, lane);
+      // ---- merge: lanes, then the four warps of this column half, then the cluster
+      bool writer;
+      const int first = warp_merge_columns<NQ>(m, sm, lane, writer);
+      constexpr int kKeep = NQ % 32 == 0 ? NQ / 32 : (NQ % 16 == 0 ? NQ / 16 : NQ / 8);
+      if (writer)
 #pragma unroll
-      for (int k = 0; k < kPer; ++k) {
-        wred_m[wslot][lane * kPer + k] = m[k];
-        wred_s[wslot][lane * kPer + k] = sm[k];
-      }
-      named_barrier(1, n_epi);  // also: every thread finished the previous instance's pass 2
-      const int tq = threadIdx.x - 64;  // 0 .. 255: thread of the column merge
-      const bool col_thread = tq < s.n_obs_pad;
+        for (int c = 0; c < kKeep; ++c) {
+          wred_m[we][first + c] = m[c];
+          wred_s[we][first + c] = sm[c];
+        }
+      named_barrier(1, 32 * kEpiWarps);  // also: every pass-2 read of the previous lse2 is done
+      const bool col_thread = te < N;
       float cm = -INFINITY, cs = 0.f;
       if (col_thread) {
-        // column tq lives in group (tq / 64) when split, else in every group
-        const int g_lo = split ? tq / 64 : 0, g_hi = split ? g_lo + 1 : kEpiGroups;
-        const int cc = split ? tq % 64 : tq;
-        for (int g = g_lo; g < g_hi; ++g)
-          for (int w = 0; w < 4; ++w) lse_merge(cm, cs, wred_m[g * 4 + w][cc], wred_s[g * 4 + w][cc]);
+        const int h = te / NQ, cc = te % NQ;  // column te lives in the warps of half h
+        for (int w = 0; w < 4; ++w) lse_merge(cm, cs, wred_m[h * 4 + w][cc], wred_s[h * 4 + w][cc]);
       }
-      const bool my_valid = col_thread && ((a.valid[e * 4 + (tq >> 5)] >> (tq & 31)) & 1u);
+      const bool my_valid = col_thread && ((vword >> (te & 31)) & 1u);
+      float lse = INFINITY;
       if (csize == 1) {
-        if (tq < 128) lse2_sh[tq] = (my_valid && cm > -INFINITY) ? cm + lg2_approx(cs) : INFINITY;
-      } else {
-        // the peers have read this CTA's previous partials before they are overwritten
-        if (li > 0 && tq < 128) mbar_wait_cluster(&read_done_bar, (li - 1) & 1, a.err, kDevTimeoutCluster);
-        if (tq < 128) {
-          part_m[tq] = cm;
-          part_s[tq] = cs;
-        }
-        named_barrier(1, n_epi);
-        if (leader)
-          for (int c = 0; c < csize; ++c) mbar_arrive_remote(mapa_shared(smem_u32(&part_ready_bar), c));
-        if (tq < 128) {
-          const bool ok = mbar_wait_cluster(&part_ready_bar, li & 1, a.err, kDevTimeoutCluster);
-          float M = -INFINITY, S = 0.f;
-          if (ok && col_thread) {
-            const uint32_t am = smem_u32(&part_m[tq]), as = smem_u32(&part_s[tq]);
-            for (int c = 0; c < csize; ++c)
-              lse_merge(M, S, ld_shared_cluster_f32(mapa_shared(am, c)), ld_shared_cluster_f32(mapa_shared(as, c)));
+        if (my_valid && cm > -INFINITY) lse = cm + lg2_approx(cs);
+      } else if (col_thread) {
+        const int b = i & 1;
+        if (leader) mbar_arrive_expect_tx(&recv_bar[b], static_cast<uint32_t>(csize * N * 8));
+        const uint32_t dst = smem_u32(&recv[(b * csize + crank) * N + te]), bar = smem_u32(&recv_bar[b]);
+        for (int c = 0; c < csize; ++c) st_async_pair(mapa_shared(dst, c), cm, cs, mapa_shared(bar, c));
+        const bool ok = mbar_wait_cluster(&recv_bar[b], (i >> 1) & 1, a.err, kDevTimeoutCluster);
+        float M = -INFINITY, S = 0.f;
+        if (ok)
+          for (int c = 0; c < csize; ++c) {  // rank order: every CTA gets the same lse2
+            const float2 p = recv[(b * csize + c) * N + te];
+            lse_merge(M, S, p.x, p.y);
           }
-          if (!ok) *abort_flag = 1;
-          lse2_sh[tq] = (ok && my_valid && M > -INFINITY) ? M + lg2_approx(S) : INFINITY;
-        }
+        if (!ok) *abort_flag = 1;
+        if (ok && my_valid && M > -INFINITY) lse = M + lg2_approx(S);
       }
-      named_barrier(1, n_epi);  // lse2 complete; in a cluster, every peer read is done
-      if (csize > 1 && leader)
-        for (int c = 0; c < csize; ++c) mbar_arrive_remote(mapa_shared(smem_u32(&read_done_bar), c));
+      if (te < 128) lse2_sh[te] = lse;
+      named_barrier(1, 32 * kEpiWarps);  // lse2 written; every read of wred is done
 
-      // ---- pass 2: thread = key; r_j = max_q (y_qj - lse2_q); groups take alternate tiles
+      // ---- pass 2: warps of half h take the tiles with parity h, all columns
       float* r_e = a.r_out + static_cast<size_t>(e) * s.cap;
       float* s_e = a.scores_out ? a.scores_out + static_cast<size_t>(e) * s.cap : nullptr;
-      for (int t = 0; t < T; ++t, ++ga) {
-        if ((ga & 1) != group) continue;
-        const int acc = ga % kAcc;
-        const bool have = !*abort_flag &&
-                          mbar_wait(&accf_bar[acc], (ga / kAcc) & 1, abort_flag, a.err, kDevTimeoutEpilogue);
-        if (have) tc_fence_after();
-        float r0 = -INFINITY, r1 = -INFINITY;
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const bool used = c * 32 < s.n_obs_pad;
-          float v[32];
-          if (have && used) {
-            tmem_ld32(tmem + acc * 128 + c * 32 + lane_addr, v);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 32; i += 2) {
-              r0 = fmaxf(r0, fmaf(v[i], sc, -lse2_sh[c * 32 + i]));
-              r1 = fmaxf(r1, fmaf(v[i + 1], sc, -lse2_sh[c * 32 + i + 1]));
-            }
-          }
+      tc_fence_after();
+      for (int j = half; j < R; j += 2) {
+        const int slot = rs + j < ring ? rs + j : rs + j - ring;
+        float r = -INFINITY;
+        if (resident_ok) r = tile_score<N>(tmem + slot * N + lane_addr, lse2_sh, sc);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cnt(&slot_free[slot], 2);  // two arrivals: this warp stands for its pair
+        const int key = (t0 + j) * kTile + key_row;
+        if (resident_ok && key < a.L) {
+          r_e[key] = r;
+          if (s_e) s_e[key] = ex2_approx(r);
+        }
+      }
+      for (int j = R + half; j < T; j += 2) {  // streaming tiles come back from HBM / L2
+        const int slot = str_slot + 2 + half;
+        const int u = kp2++;
+        bool have = !*abort_flag && mbar_wait(&slot_full[slot], u & 1, abort_flag, a.err, kDevTimeoutEpilogue);
+        have = __all_sync(0xffffffffu, have);
+        float r = -INFINITY;
+        if (have) {
+          tc_fence_after();
+          r = tile_score<N>(tmem + slot * N + lane_addr, lse2_sh, sc);
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive_n(&acce_bar[acc], split ? 2 : 1);
-        const int j = (t0 + t) * kTile + key_row;
-        if (have && j < a.L) {
-          const float r = fmaxf(r0, r1);
-          r_e[j] = r;
-          if (s_e) s_e[j] = ex2_approx(r);
+        if (lane == 0) mbar_arrive_cnt(&slot_free[slot], 2);
+        const int key = (t0 + j) * kTile + key_row;
+        if (have && key < a.L) {
+          r_e[key] = r;
+          if (s_e) s_e[key] = ex2_approx(r);
         }
+      }
+      rs += R;  // the next instance starts where this one ended
+      if (rs >= ring) {
+        rs -= ring;
+        ++ru;
       }
     }
   }
@@ -394,57 +536,73 @@ __global__ void __launch_bounds__(kScThreads, 1)
   if (csize > 1) cluster_sync_all();  // no CTA leaves while a peer may still access its shared memory
 }
 
-// CTAs per instance: enough that the instances in flight (one per cluster,
-// one CTA per SM) hold about 90 MB of K between the two passes; at most 8.
-int cluster_size(int L, int d, int sms) {
-  const double bytes = static_cast<double>(sms) * L * d * 2;
-  int c = static_cast<int>(bytes / 90e6 + 0.999);
-  const int tiles = (L + kTile - 1) / kTile;
-  if (c > tiles) c = tiles;
-  return c < 1 ? 1 : (c > 8 ? 8 : c);
+// Cluster size and tensor-memory placement: the fewest CTAs per instance
+// whose tiles all fit the slot ring, with at least kSlack spare slots where
+// eight CTAs allow it; when not even eight CTAs hold an instance, eight CTAs
+// with streaming slots.  Slot barriers exist for kMaxSlots slots, and tensor
+// memory holds kTmemCols / n_obs_pad of them (at least 4, n_obs_pad <= 128).
+constexpr int kSlack = 1;
+
+Plan plan_score(int L, int n_obs_pad) {
+  const int T_all = (L + kTile - 1) / kTile;
+  int cap = static_cast<int>(kTmemCols) / n_obs_pad;
+  if (cap > kMaxSlots) cap = kMaxSlots;
+  const int cmax = T_all < 8 ? T_all : 8;
+  for (int slack = kSlack; slack >= 0; --slack)
+    for (int c = 1; c <= cmax; ++c)
+      if ((T_all + c - 1) / c + slack <= cap) return Plan{c, cap, 0};
+  return Plan{cmax, cap - 4, 1};
 }
 
 template <int D, int NQ>
 cudaError_t launch_score_dq(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreArgs& a,
                             cudaStream_t st) {
   using C = ScoreCfg<D>;
-  const size_t smem = C::smem_bytes(s.n_obs_pad);
-  const int n_stages = C::stages(s.n_obs_pad);
+  const Plan plan = plan_score(a.L, s.n_obs_pad);
+  const size_t smem = C::smem_bytes(s.n_obs_pad, plan.csize);
+  const int n_stages = C::stages(s.n_obs_pad, plan.csize);
   cudaError_t err = cudaFuncSetAttribute(score_kernel<D, NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
   if (err != cudaSuccess) return err;
   int dev = 0, sms = 0, max_clusters = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int csize = cluster_size(a.L, s.d, sms);
   cudaLaunchConfig_t cfg = {};
   cfg.blockDim = dim3(kScThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = static_cast<unsigned>(csize);
+  attr[0].val.clusterDim.x = static_cast<unsigned>(plan.csize);
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   // one resident wave of clusters, each looping over its share of the instances
-  cfg.gridDim = dim3(static_cast<unsigned>(csize * sms));
+  cfg.gridDim = dim3(static_cast<unsigned>(plan.csize * sms));
   if (cudaOccupancyMaxActiveClusters(&max_clusters, score_kernel<D, NQ>, &cfg) != cudaSuccess || max_clusters < 1) {
     cudaGetLastError();
-    max_clusters = sms / csize > 0 ? sms / csize : 1;
+    max_clusters = sms / plan.csize > 0 ? sms / plan.csize : 1;
   }
   const int n_clusters = max_clusters < s.n_inst ? max_clusters : s.n_inst;
-  cfg.gridDim = dim3(static_cast<unsigned>(n_clusters * csize));
-  return cudaLaunchKernelEx(&cfg, score_kernel<D, NQ>, kmap, qmap, s, a, csize, n_stages);
+  cfg.gridDim = dim3(static_cast<unsigned>(n_clusters * plan.csize));
+  return cudaLaunchKernelEx(&cfg, score_kernel<D, NQ>, kmap, qmap, s, a, plan, n_stages);
 }
 
 template <int D>
 cudaError_t launch_score_d(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreArgs& a,
                            cudaStream_t st) {
-  // query columns each epilogue thread tracks in pass 1
-  if (s.n_obs_pad <= 32) return launch_score_dq<D, 32>(s, kmap, qmap, a, st);
-  return launch_score_dq<D, 64>(s, kmap, qmap, a, st);
+  // query columns of each pass-1 warp: half of the padded query count
+  switch (s.n_obs_pad) {
+    case 16: return launch_score_dq<D, 8>(s, kmap, qmap, a, st);
+    case 32: return launch_score_dq<D, 16>(s, kmap, qmap, a, st);
+    case 48: return launch_score_dq<D, 24>(s, kmap, qmap, a, st);
+    case 64: return launch_score_dq<D, 32>(s, kmap, qmap, a, st);
+    case 80: return launch_score_dq<D, 40>(s, kmap, qmap, a, st);
+    case 96: return launch_score_dq<D, 48>(s, kmap, qmap, a, st);
+    case 112: return launch_score_dq<D, 56>(s, kmap, qmap, a, st);
+    default: return launch_score_dq<D, 64>(s, kmap, qmap, a, st);
+  }
 }
 
 }  // namespace

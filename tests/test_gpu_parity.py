@@ -79,6 +79,17 @@ def test_no_rotation_and_max_queries():
     _run(wl, seed=10)
 
 
+@pytest.mark.parametrize("wl", [
+    # 128 scoring queries, 40 tiles: tensor memory holds none of them resident past eight CTAs
+    QWEN3_4B.scaled(name="long_m128_L5000", n_layers=1, batch=1, n_q_heads=64, n_kv_heads=8, window=12,
+                    n_beacons=32, L=5000, budget=3000, n_init=64, n_clusters=32),
+    # 48 scoring queries, 157 tiles: resident tiles plus streaming tiles in every CTA
+    QWEN3_4B.scaled(name="long_L20000", n_layers=1, batch=1, L=20000, budget=12000),
+], ids=lambda w: w.name)
+def test_long_cache_streaming_tiles(wl):
+    _run(wl, seed=13)
+
+
 def test_identical_keys_tie_everywhere():
     """All keys equal: every score is 1/L, the kept set is the lowest-index
     candidates plus the window (ties go to the lower index)."""
