@@ -368,8 +368,10 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
   }
   if (e != cudaSuccess) return cuda_fail(ctx, e, "qobs launch");
 
-  CUtensorMap kmap, qmap;
+  CUtensorMap kmap, kmap32, qmap;
   int rc = encode_rows(ctx, &kmap, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 128);
+  if (rc != BKV_OK) return rc;
+  rc = encode_rows(ctx, &kmap32, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 32);
   if (rc != BKV_OK) return rc;
   rc = encode_rows(ctx, &qmap, ctx->qobs, static_cast<uint64_t>(s.n_inst) * s.n_obs_pad, s.d,
                    static_cast<uint32_t>(s.n_obs_pad));
@@ -383,7 +385,7 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
   sa.err = ctx->err;
   {
     ProfScope ps(ctx, BKV_K_SCORE);
-    e = bkv::launch_score(s, kmap, qmap, sa, ctx->stream);
+    e = bkv::launch_score(s, kmap, kmap32, qmap, sa, ctx->stream);
   }
   if (e != cudaSuccess) return cuda_fail(ctx, e, "score launch");
   {

@@ -50,8 +50,11 @@ struct ScoreArgs {
   float* scores_out;       // [n_inst][cap] probabilities, or nullptr
   int* err;                // device error word
 };
-cudaError_t launch_score(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreArgs& a,
-                         cudaStream_t st);
+// kmap / kmap32: K as [n_inst * cap][d] in 128-row and 32-row boxes of [64]
+// columns (128-byte swizzle); qmap: Qobs as [n_inst * n_obs_pad][d] in boxes
+// of n_obs_pad rows.
+cudaError_t launch_score(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32, const CUtensorMap& qmap,
+                         const ScoreArgs& a, cudaStream_t st);
 
 cudaError_t launch_select_gather(const Shape& s, const float* r, int L, int budget, __nv_bfloat16* K,
                                  __nv_bfloat16* V, int* kept, cudaStream_t st);

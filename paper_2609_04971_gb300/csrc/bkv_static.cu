@@ -206,8 +206,9 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
   }
   e = bkv::launch_qobs(s, static_cast<const __nv_bfloat16*>(q_recent), centroids,
                        reinterpret_cast<const long long*>(counts), rope, rotate, qobs, valid, st);
-  CUtensorMap kmap, qmap;
+  CUtensorMap kmap, kmap32, qmap;
   if (e == cudaSuccess && (!encode(&kmap, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 128) ||
+                           !encode(&kmap32, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 32) ||
                            !encode(&qmap, qobs, static_cast<uint64_t>(s.n_inst) * s.n_obs_pad, s.d,
                                    static_cast<uint32_t>(s.n_obs_pad)))) {
     message(err_msg, err_len, "cuTensorMapEncodeTiled failed");
@@ -221,7 +222,7 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
     sa.r_out = rscore;
     sa.scores_out = scores_out;
     sa.err = reinterpret_cast<int*>(dev_status);
-    e = bkv::launch_score(s, kmap, qmap, sa, st);
+    e = bkv::launch_score(s, kmap, kmap32, qmap, sa, st);
   }
   if (e == cudaSuccess)
     e = bkv::launch_select_gather(s, rscore, L, budget, static_cast<__nv_bfloat16*>(K),

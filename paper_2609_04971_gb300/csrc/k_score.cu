@@ -4,7 +4,9 @@
 // Persistent kernel, one CTA per SM.  Instances are processed by
 // thread-block clusters of C CTAs; cluster k takes instances k,
 // k + n_clusters, ...; CTA r of a cluster owns the same contiguous range of
-// 128-key tiles of every instance.
+// keys of every instance, the cache split in 32-key units as evenly as
+// possible, and walks it in 128-key tiles (a ragged last tile is loaded in
+// 32-row boxes; the MMA lanes past the range are ignored).
 //
 // Each tile goes through the tensor cores once: D = K_tile x Qobs^T with
 // M = 128 keys (TMEM lanes) and N = padded query count (TMEM columns),
@@ -14,8 +16,9 @@
 // in turn (slots left over by one instance let the next one's tiles land
 // while it finishes), so K is read from HBM exactly once.  y = logit * log2(e) is the base-2 logit.
 //   Pass 1 (statistics, as tiles land): each thread owns one key of the tile
-//     and keeps, for the query columns it owns, a running maximum m_q and sum
-//     s_q of 2^(y - m_q).  After the CTA's last tile the partials are merged
+//     and keeps, for the query columns it owns, a reference m_q and the sum
+//     s_q of 2^(y - m_q) over the keys it has seen (m_q follows the maximum
+//     lazily, so that the terms stay below 2^64).  After the CTA's last tile the partials are merged
 //     (recursive halving inside each warp, shared memory across warps) and
 //     the CTAs of a cluster exchange theirs through distributed shared memory;
 //     every CTA combines them in rank order and gets the same
@@ -199,8 +202,8 @@ __device__ __forceinline__ float tile_score(uint32_t taddr, const float* lse2, f
 
 template <int D, int NQ>
 __global__ void __launch_bounds__(kScThreads, 1)
-    score_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap, Shape s,
-                 ScoreArgs a, Plan plan, int n_stages) {
+    score_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap kmap32,
+                 const __grid_constant__ CUtensorMap qmap, Shape s, ScoreArgs a, Plan plan, int n_stages) {
   using C = ScoreCfg<D>;
   constexpr int N = 2 * NQ;  // padded query columns
   static_assert(NQ % 8 == 0 && NQ <= 64, "query columns per pass-1 warp");
@@ -220,9 +223,10 @@ __global__ void __launch_bounds__(kScThreads, 1)
   const int cluster_id = blockIdx.x / csize;
   const int n_clusters = gridDim.x / csize;
   const int n_my = cluster_id < s.n_inst ? (s.n_inst - cluster_id + n_clusters - 1) / n_clusters : 0;
-  const int T_all = (a.L + kTile - 1) / kTile;
-  const int t0 = crank * T_all / csize;
-  const int T = (crank + 1) * T_all / csize - t0;  // tiles this CTA owns in every instance
+  const int U = (a.L + 31) / 32;                     // 32-key units of the cache
+  const int k0 = (crank * U / csize) * 32;           // this CTA's keys: [k0, k1)
+  const int k1 = min(a.L, ((crank + 1) * U / csize) * 32);
+  const int T = (k1 - k0 + kTile - 1) / kTile;       // tiles this CTA owns in every instance
   const int R = T < plan.slots ? T : plan.slots;     // resident tiles
   const int n_str = T - R;                           // streaming tiles (plan.stream only)
   const int ring = plan.slots;                       // resident slots, used in cyclic order
@@ -272,6 +276,7 @@ __global__ void __launch_bounds__(kScThreads, 1)
     if (lane == 0) {
       const uint64_t once = l2_policy_evict_first(), again = l2_policy_evict_last();
       prefetch_tmap(&kmap);
+      prefetch_tmap(&kmap32);
       prefetch_tmap(&qmap);
       int g = 0;  // ring iteration
       bool ok = true;
@@ -295,10 +300,20 @@ __global__ void __launch_bounds__(kScThreads, 1)
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(&full_bar[st], C::kTileBytes);
-          for (int b = 0; b < C::kBoxes; ++b)
-            tma_load_2d(k_smem + (st * C::kBoxes + b) * kBoxBytes, &kmap, &full_bar[st], b * 64,
-                        e * s.cap + (t0 + t) * kTile, (j < T && t >= R) ? again : once);
+          const uint64_t pol = (j < T && t >= R) ? again : once;
+          const int row = e * s.cap + k0 + t * kTile;
+          const int rows = min(kTile, k1 - k0 - t * kTile);
+          unsigned char* dst = k_smem + st * C::kBoxes * kBoxBytes;
+          if (rows == kTile) {
+            mbar_arrive_expect_tx(&full_bar[st], C::kTileBytes);
+            for (int b = 0; b < C::kBoxes; ++b) tma_load_2d(dst + b * kBoxBytes, &kmap, &full_bar[st], b * 64, row, pol);
+          } else {  // ragged tile: 32-row boxes at 4 KB steps keep the 128-row swizzled layout
+            const int chunks = (rows + 31) / 32;
+            mbar_arrive_expect_tx(&full_bar[st], static_cast<uint32_t>(chunks * 32 * D * 2));
+            for (int q = 0; q < chunks; ++q)
+              for (int b = 0; b < C::kBoxes; ++b)
+                tma_load_2d(dst + b * kBoxBytes + q * 4096, &kmap32, &full_bar[st], b * 64, row + q * 32, pol);
+          }
           ++g;
         }
       }
@@ -431,15 +446,34 @@ __global__ void __launch_bounds__(kScThreads, 1)
           if (lane == 0) mbar_arrive(&slot_free[slot]);
           ++ks;
         }
-        if (have && (t0 + j) * kTile + key_row < a.L) {
+        // Running sums relative to a reference m that moves only when a base-2
+        // logit exceeds it by more than 64, so the terms stay below 2^64 and
+        // the common step is one FFMA, one ex2 and one add per column.
+        if (have) {
+          const bool key_ok = k0 + j * kTile + key_row < k1;
+          float t[NQ];
+          bool rebase = !__all_sync(0xffffffffu, key_ok);  // a ragged tile takes the careful path
 #pragma unroll
           for (int c = 0; c < NQ; ++c) {
-            const float y = v[c] * sc;
-            const float dlt = y - m[c];
-            const float w = ex2_approx(-fabsf(dlt));
-            const bool up = dlt > 0.f;
-            sm[c] = up ? fmaf(sm[c], w, 1.f) : sm[c] + w;
-            m[c] = up ? y : m[c];
+            t[c] = fmaf(v[c], sc, -m[c]);
+            rebase |= t[c] > 64.f;
+          }
+          if (__any_sync(0xffffffffu, rebase)) {
+            if (key_ok) {
+#pragma unroll
+              for (int c = 0; c < NQ; ++c) {
+                if (t[c] > 64.f) {  // also the first key: m = -inf gives t = +inf
+                  const float y = v[c] * sc;
+                  sm[c] = fmaf(sm[c], ex2_approx(m[c] - y), 1.f);
+                  m[c] = y;
+                } else {
+                  sm[c] += ex2_approx(t[c]);
+                }
+              }
+            }
+          } else {
+#pragma unroll
+            for (int c = 0; c < NQ; ++c) sm[c] += ex2_approx(t[c]);
           }
         }
       }
@@ -494,8 +528,8 @@ __global__ void __launch_bounds__(kScThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_cnt(&slot_free[slot], 2);  // two arrivals: this warp stands for its pair
-        const int key = (t0 + j) * kTile + key_row;
-        if (resident_ok && key < a.L) {
+        const int key = k0 + j * kTile + key_row;
+        if (resident_ok && key < k1) {
           r_e[key] = r;
           if (s_e) s_e[key] = ex2_approx(r);
         }
@@ -513,8 +547,8 @@ __global__ void __launch_bounds__(kScThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_cnt(&slot_free[slot], 2);
-        const int key = (t0 + j) * kTile + key_row;
-        if (have && key < a.L) {
+        const int key = k0 + j * kTile + key_row;
+        if (have && key < k1) {
           r_e[key] = r;
           if (s_e) s_e[key] = ex2_approx(r);
         }
@@ -544,19 +578,21 @@ __global__ void __launch_bounds__(kScThreads, 1)
 constexpr int kSlack = 1;
 
 Plan plan_score(int L, int n_obs_pad) {
-  const int T_all = (L + kTile - 1) / kTile;
+  const int U = (L + 31) / 32;
   int cap = static_cast<int>(kTmemCols) / n_obs_pad;
   if (cap > kMaxSlots) cap = kMaxSlots;
-  const int cmax = T_all < 8 ? T_all : 8;
+  const int cmax = U < 8 ? U : 8;  // every CTA owns at least one 32-key unit
   for (int slack = kSlack; slack >= 0; --slack)
-    for (int c = 1; c <= cmax; ++c)
-      if ((T_all + c - 1) / c + slack <= cap) return Plan{c, cap, 0};
+    for (int c = 1; c <= cmax; ++c) {
+      const int tiles = ((U + c - 1) / c + 3) / 4;  // tiles of the CTA with the most units
+      if (tiles + slack <= cap) return Plan{c, cap, 0};
+    }
   return Plan{cmax, cap - 4, 1};
 }
 
 template <int D, int NQ>
-cudaError_t launch_score_dq(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreArgs& a,
-                            cudaStream_t st) {
+cudaError_t launch_score_dq(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32,
+                            const CUtensorMap& qmap, const ScoreArgs& a, cudaStream_t st) {
   using C = ScoreCfg<D>;
   const Plan plan = plan_score(a.L, s.n_obs_pad);
   const size_t smem = C::smem_bytes(s.n_obs_pad, plan.csize);
@@ -586,30 +622,31 @@ cudaError_t launch_score_dq(const Shape& s, const CUtensorMap& kmap, const CUten
   }
   const int n_clusters = max_clusters < s.n_inst ? max_clusters : s.n_inst;
   cfg.gridDim = dim3(static_cast<unsigned>(n_clusters * plan.csize));
-  return cudaLaunchKernelEx(&cfg, score_kernel<D, NQ>, kmap, qmap, s, a, plan, n_stages);
+  return cudaLaunchKernelEx(&cfg, score_kernel<D, NQ>, kmap, kmap32, qmap, s, a, plan, n_stages);
 }
 
 template <int D>
-cudaError_t launch_score_d(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreArgs& a,
-                           cudaStream_t st) {
+cudaError_t launch_score_d(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32, const CUtensorMap& qmap,
+                           const ScoreArgs& a, cudaStream_t st) {
   // query columns of each pass-1 warp: half of the padded query count
   switch (s.n_obs_pad) {
-    case 16: return launch_score_dq<D, 8>(s, kmap, qmap, a, st);
-    case 32: return launch_score_dq<D, 16>(s, kmap, qmap, a, st);
-    case 48: return launch_score_dq<D, 24>(s, kmap, qmap, a, st);
-    case 64: return launch_score_dq<D, 32>(s, kmap, qmap, a, st);
-    case 80: return launch_score_dq<D, 40>(s, kmap, qmap, a, st);
-    case 96: return launch_score_dq<D, 48>(s, kmap, qmap, a, st);
-    case 112: return launch_score_dq<D, 56>(s, kmap, qmap, a, st);
-    default: return launch_score_dq<D, 64>(s, kmap, qmap, a, st);
+    case 16: return launch_score_dq<D, 8>(s, kmap, kmap32, qmap, a, st);
+    case 32: return launch_score_dq<D, 16>(s, kmap, kmap32, qmap, a, st);
+    case 48: return launch_score_dq<D, 24>(s, kmap, kmap32, qmap, a, st);
+    case 64: return launch_score_dq<D, 32>(s, kmap, kmap32, qmap, a, st);
+    case 80: return launch_score_dq<D, 40>(s, kmap, kmap32, qmap, a, st);
+    case 96: return launch_score_dq<D, 48>(s, kmap, kmap32, qmap, a, st);
+    case 112: return launch_score_dq<D, 56>(s, kmap, kmap32, qmap, a, st);
+    default: return launch_score_dq<D, 64>(s, kmap, kmap32, qmap, a, st);
   }
 }
 
 }  // namespace
 
-cudaError_t launch_score(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreArgs& a,
-                         cudaStream_t st) {
-  return s.d == 128 ? launch_score_d<128>(s, kmap, qmap, a, st) : launch_score_d<64>(s, kmap, qmap, a, st);
+cudaError_t launch_score(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32, const CUtensorMap& qmap,
+                         const ScoreArgs& a, cudaStream_t st) {
+  return s.d == 128 ? launch_score_d<128>(s, kmap, kmap32, qmap, a, st)
+                    : launch_score_d<64>(s, kmap, kmap32, qmap, a, st);
 }
 
 }  // namespace bkv
