@@ -309,9 +309,17 @@ int bkv_update_beacons(bkv_ctx* ctx, const void* q_new, int32_t n_new, int32_t* 
     return BKV_OK;
   }
   if (!ctx->state_ready) return fail(ctx, BKV_ESTATE, "update before bkv_init_beacons / bkv_set_state");
+  // a tile is at most 128 queries of one instance: boxes no taller than that
+  const uint64_t q_rows = static_cast<uint64_t>(s.n_inst) * s.G * n_new;
+  uint64_t box_rows = (static_cast<uint64_t>(s.G) * n_new + 7) / 8 * 8;
+  if (box_rows > 128) box_rows = 128;
+  if (box_rows > q_rows) box_rows = q_rows;
+  CUtensorMap qmap;
+  const int rc = encode_rows(ctx, &qmap, q_new, q_rows, s.d, static_cast<uint32_t>(box_rows));
+  if (rc != BKV_OK) return rc;
   ProfScope ps(ctx, BKV_K_UPDATE);
-  cudaError_t e = bkv::launch_update(s, static_cast<const __nv_bfloat16*>(q_new), n_new, ctx->cent, ctx->sums,
-                                     ctx->counts, assign_out, ctx->stream);
+  cudaError_t e = bkv::launch_update(s, qmap, static_cast<int>(box_rows), n_new, ctx->cent, ctx->sums, ctx->counts,
+                                     assign_out, ctx->err, ctx->stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e, "update launch");
   return BKV_OK;
 }

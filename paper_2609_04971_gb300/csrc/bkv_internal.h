@@ -32,8 +32,11 @@ constexpr int kMaxFpsRows = 4096;
 cudaError_t launch_fps_init(const Shape& s, const __nv_bfloat16* q_init, int n_init, float* cent, double* sums,
                             long long* counts, cudaStream_t st);
 
-cudaError_t launch_update(const Shape& s, const __nv_bfloat16* q_new, int n_new, float* cent, double* sums,
-                          long long* counts, int* assign_out, cudaStream_t st);
+// qmap: the new queries as [n_inst * G * n_new][d] bf16 in boxes of
+// [box_rows][64] (128-byte swizzle), box_rows = min(128, rows); err: device
+// error word.
+cudaError_t launch_update(const Shape& s, const CUtensorMap& qmap, int box_rows, int n_new, float* cent,
+                          double* sums, long long* counts, int* assign_out, int* err, cudaStream_t st);
 
 // ---- compression (k_qobs.cu, k_score.cu, k_select_gather.cu)
 // rope: [W + 1][d / 2] fp64 (cos, sin) pairs, immediately followed by the same

@@ -1,36 +1,100 @@
-// Beacon maintenance: nearest-beacon assignment by cosine similarity and the
-// running-mean centroid update, for every instance at once.
+// Beacon maintenance (Section 3.2, Appendix D): every new query is assigned to
+// the beacon of highest cosine similarity and that beacon's centroid becomes
+// the running mean of the queries assigned to it.
 //
-// One CTA of 256 threads per instance; its queries are processed in passes
-// of up to 2048:
-//   * Screening (4 threads per query, straight from global memory): fp32 dots
-//     of the query with unit-length centroids, four independent FMA chains
-//     per thread.  When the best and second-best dot differ by less than
-//     1e-4 |q| (far above the ~1e-5 |q| worst-case error of a 128-term fp32
-//     dot), the query is re-decided in fp64 by one warp: cos(q, c_b) =
-//     (q . c_b) / (|q| |c_b|) with fp64 products and sums, which can differ
-//     from a sequential fp64 evaluation only at ties below ~1e-15 (the lowest
-//     beacon wins ties).
-//   * Accumulation: each bf16 query element is converted to an int64 fixed
-//     point value with 40 fractional bits (exact for |x| >= 2^-33).  The
-//     queries are bucketed by beacon (counting sort); the thread that owns
-//     (beacon, column) sums its bucket in a register and adds it to its
-//     shared-memory cell, so the per-call sum is exact and independent of
-//     ordering.  It is then added once to the fp64 running sum.
-//   * Centroid: c = fp32(sum * (1 / count)) in fp64, within one fp32 ulp of
-//     fp32(sum / count).
+// Persistent kernel, one CTA per SM; CTA k takes instances k, k + grid, ...
+// An instance's queries stream through a ring of shared-memory stages in
+// tiles of up to 128 (TMA, 128-byte swizzle) and are read from HBM once.
+//
+// Screening on the tensor cores: per tile, D1 = Q x [c_hi ; c_lo]^T where
+// c_hi = bf16(c / |c|) and c_lo = bf16(c / |c| - c_hi), so dot_b = D1[:, b] +
+// D1[:, nbp + b] carries the unit-centroid dot to about 2^-16 |q| (bf16 x bf16
+// products are exact, the accumulation is fp32); D2 = Q x Q^T gives |q|^2 on
+// its diagonal.  When best and second-best dots differ by at most 4e-4 |q|
+// (several times their error bound), the query is re-decided exactly: the
+// beacon maximising (q . c_b) / |c_b| with fp64 products, warp-parallel fp64
+// sums and a correctly rounded fp64 1 / |c_b|; this agrees with the cosine
+// (q . c_b) / (|q| |c_b|) evaluated sequentially in fp64 except at ties below
+// ~1e-15 (the lowest beacon wins ties).  Zero queries and instances without a
+// valid beacon give -1.
+//
+// Sums: int64 fixed point with 40 fractional bits.  A tile's screened rows
+// are sorted by beacon (ballot counting sort); each accumulator warp takes an
+// equal slice of that order, its lanes owning D / 32 columns each, and keeps
+// three fp32 part sums per column that are exact by construction (see Parts;
+// exact for 2^-31 <= |x| < 2^14, the conversion to fixed point per beacon
+// change rather than per element); re-decided rows are converted directly.
+// The per-call sum is exact and independent of the order.  It is then
+// added once to the fp64 running sum, and c = fp32(sum * (1 / count)) in
+// fp64, within one fp32 ulp of fp32(sum / count).
+//
+// Warp roles (18 warps): warp 0 TMA producer; warp 1 TMEM allocation and MMA
+// issue; warps 2..5 screeners (one per TMEM lane quarter: decisions, the
+// sorted row list of the tile, exact re-decisions); warps 6..13 accumulators
+// (the sums of a tile, while the screeners work on the next one; the row
+// lists are double-buffered); warps 14..17 bookkeeping: they build the
+// unit-centroid operand of the next instance and fold the finished one into
+// the running state, from centroids and sums brought in by bulk copies
+// (accumulators double-buffered by instance).  All waits are bounded.
 #include "bkv_device.cuh"
 #include "bkv_internal.h"
 
 namespace bkv {
 namespace {
 
-constexpr int kUpdThreads = 256;
-constexpr int kUpdWarps = kUpdThreads / 32;
-constexpr int kPass = 2048;  // queries per pass (assignment buffer size)
+constexpr int kScreeners = 4;
+constexpr int kAccum = 8;
+constexpr int kKeepers = 4;
+constexpr int kUThreads = 32 * (2 + kScreeners + kAccum + kKeepers);
+constexpr int kQTile = 128;                 // queries per tile (MMA M)
+constexpr uint32_t kQBox = 128 * 128;       // [128 rows][64 bf16] swizzled box slot
+constexpr int kUMaxStages = 8;
+constexpr size_t kUSmemBudget = 216 * 1024;
+constexpr float kMarginRel = 4e-4f;
 
-__device__ __forceinline__ long long to_fixed40(__nv_bfloat16 v) {
-  return __float2ll_rn(__bfloat162float(v) * 0x1p40f);
+struct UpdArgs {
+  int n_inst, nq, nb, nbp;  // instances, queries per instance, beacons, beacons padded to 8
+  int box_rows;             // rows of one TMA box of queries (<= 128)
+  float* cent;
+  double* sums;
+  long long* counts;
+  int* assign_out;
+  int* err;
+};
+
+template <int D>
+struct UpdCfg {
+  static constexpr int kBoxes = D / 64;
+  static constexpr uint32_t kStageBytes = kBoxes * kQBox;
+  __host__ __device__ static size_t bmat_bytes(int nbp) { return static_cast<size_t>(kBoxes) * 2 * nbp * 128; }
+  __host__ __device__ static size_t state_bytes(int nb, int nbp) {
+    // bmat[2], acc[2] (int64), cent[2] (fp32), sums (fp64)
+    return 2 * bmat_bytes(nbp) + 2 * static_cast<size_t>(nb) * D * 8 + 2 * static_cast<size_t>(nb) * D * 4 +
+           static_cast<size_t>(nb) * D * 8;
+  }
+  static int stages(int nb, int nbp) {
+    const size_t room = kUSmemBudget - 1024 - state_bytes(nb, nbp);
+    const int n = static_cast<int>(room / kStageBytes);
+    return n < kUMaxStages ? n : kUMaxStages;
+  }
+  static size_t smem_bytes(int nb, int nbp) {
+    return 1024 + static_cast<size_t>(stages(nb, nbp)) * kStageBytes + state_bytes(nb, nbp);
+  }
+};
+
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* err) {
+  int never = 0;
+  mbar_wait(bar, parity, &never, err, kDevTimeoutDrain);
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// Contiguous global -> shared copy by the TMA unit, completing on `bar`.
+__device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
 }
 
 __device__ __forceinline__ double warp_sum_f64(double v) {
@@ -39,247 +103,596 @@ __device__ __forceinline__ double warp_sum_f64(double v) {
   return v;
 }
 
+// round(x * 2^40) of the bf16 value whose bits sit in the upper half of
+// `hi16` (lower half zero): the scale is added to the fp32 exponent field
+// (exact for |x| < 2^88; a zero or subnormal x becomes a value below 2^-80,
+// which rounds to 0 as x * 2^40 would), then one round-to-nearest conversion.
+__device__ __forceinline__ long long bf16_fixed40(uint32_t hi16) {
+  return __float2ll_rn(__uint_as_float(hi16 + (40u << 23)));
+}
+
+// Byte offset of element (row, col) in a [rows][D] bf16 tile stored as D / 64
+// boxes of [rows][64] with the 128-byte swizzle (box_bytes apart).
+__device__ __forceinline__ uint32_t sw128_offset(int row, int col, uint32_t box_bytes) {
+  return (col >> 6) * box_bytes + row * 128 + ((((col & 63) >> 3) ^ (row & 7)) << 4) + ((col & 7) << 1);
+}
+
+// Adds the kCols bf16 values at p (columns col0 ..) to s as fixed point.
+template <int kCols>
+__device__ __forceinline__ void add_fixed(long long (&s)[kCols], const unsigned char* p) {
+  if constexpr (kCols == 4) {
+    const uint2 w = *reinterpret_cast<const uint2*>(p);
+    s[0] += bf16_fixed40(w.x << 16);
+    s[1] += bf16_fixed40(w.x & 0xffff0000u);
+    s[2] += bf16_fixed40(w.y << 16);
+    s[3] += bf16_fixed40(w.y & 0xffff0000u);
+  } else {
+    const uint32_t w = *reinterpret_cast<const uint32_t*>(p);
+    s[0] += bf16_fixed40(w << 16);
+    s[1] += bf16_fixed40(w & 0xffff0000u);
+  }
+}
+
+// Exact sums of bf16 values without a 64-bit conversion per element: x is
+// split into xh = x rounded to a multiple of 2^-3, xm = the rest rounded to a
+// multiple of 2^-20 and xl = what remains (magic-number rounding, fp32 adds
+// only); each part's fp32 running sum is exact over up to 128 values with
+// |x| < 2^14 (xl is exact for |x| >= 2^-31).  `fixed40` turns the three sums
+// into round(sum * 2^40) with 32-bit conversions.
+struct Parts {
+  float h, m, l;
+};
+
+__device__ __forceinline__ void parts_add(Parts& p, float x) {
+  constexpr float kM1 = 1572864.0f;  // 1.5 * 2^20: x + kM1 rounds x to a multiple of 2^-3
+  constexpr float kM2 = 12.0f;       // 1.5 * 2^3: r + kM2 rounds r to a multiple of 2^-20
+  const float xh = __fadd_rn(__fadd_rn(x, kM1), -kM1);
+  const float r = __fadd_rn(x, -xh);
+  const float xm = __fadd_rn(__fadd_rn(r, kM2), -kM2);
+  p.h = __fadd_rn(p.h, xh);
+  p.m = __fadd_rn(p.m, xm);
+  p.l = __fadd_rn(p.l, __fadd_rn(r, -xm));
+}
+
+__device__ __forceinline__ long long fixed40(const Parts& p) {
+  const long long h = static_cast<long long>(__float2int_rn(p.h * 8.0f)) << 37;
+  const long long m = static_cast<long long>(__float2int_rn(p.m * 1048576.0f)) << 20;
+  const long long l = static_cast<long long>(__float2int_rn(p.l * 274877906944.0f)) << 2;
+  return h + m + l;
+}
+
+// Adds the kCols bf16 values at p (columns col0 ..) to the part sums.
+template <int kCols>
+__device__ __forceinline__ void add_parts(Parts (&s)[kCols], const unsigned char* p) {
+  if constexpr (kCols == 4) {
+    const uint2 w = *reinterpret_cast<const uint2*>(p);
+    parts_add(s[0], __uint_as_float(w.x << 16));
+    parts_add(s[1], __uint_as_float(w.x & 0xffff0000u));
+    parts_add(s[2], __uint_as_float(w.y << 16));
+    parts_add(s[3], __uint_as_float(w.y & 0xffff0000u));
+  } else {
+    const uint32_t w = *reinterpret_cast<const uint32_t*>(p);
+    parts_add(s[0], __uint_as_float(w << 16));
+    parts_add(s[1], __uint_as_float(w & 0xffff0000u));
+  }
+}
+
 template <int D>
-__global__ void __launch_bounds__(kUpdThreads) update_kernel(const __nv_bfloat16* __restrict__ q_new, int nq, int nb,
-                                                              float* __restrict__ cent, double* __restrict__ sums,
-                                                              long long* __restrict__ counts,
-                                                              int* __restrict__ assign_out) {
-  constexpr int kPer = D / 4;  // dims per screening thread
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  long long* acc = reinterpret_cast<long long*>(smem_raw);  // [nb][D]
-  float* chat = reinterpret_cast<float*>(acc + nb * D);     // [nb][D] unit centroids
-  __shared__ int asg[kPass];
-  __shared__ short order[kPass];
-  __shared__ int refine_idx[kPass];
-  __shared__ int n_refine;
-  __shared__ int bucket_start[kMaxBeacons + 1];
-  __shared__ int bucket_fill[kMaxBeacons];
-  __shared__ int add_cnt[kMaxBeacons];
-  __shared__ int bvalid[kMaxBeacons];
-  __shared__ double cn64[kMaxBeacons];
-  __shared__ int degenerate;
+__global__ void __launch_bounds__(kUThreads, 1)
+    update_kernel(const __grid_constant__ CUtensorMap qmap, UpdArgs a, int n_stages) {
+  using C = UpdCfg<D>;
+  constexpr int kCols = D / 32;  // columns per lane in the accumulation
+  extern __shared__ unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[kUMaxStages], empty_bar[kUMaxStages];
+  __shared__ __align__(8) uint64_t accfull[2], accfree[2], bready[2], bfree[2], drain_bar;
+  __shared__ __align__(8) uint64_t accdone[2], accclear[2], cbar[2], sbar, sfull[2], sempty[2];
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ int abort_sh;
+  __shared__ int order_t[2][kQTile];  // row | beacon << 8, sorted by beacon (by tile parity)
+  __shared__ int refine_t[2][kQTile];
+  __shared__ int n_refine[2], n_asg_sh[2];
+  __shared__ int cnt_w[2][4][kMaxBeacons];
+  __shared__ int add_cnt[2][kMaxBeacons];
+  __shared__ int bvalid[2][kMaxBeacons];
+  __shared__ double cninv[2][kMaxBeacons];
+  __shared__ long long cnt_old[2][kMaxBeacons];
+  __shared__ double rcp_sh[kMaxBeacons];
+  __shared__ int degenerate[2];
 
-  const int e = blockIdx.x;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const float* cent_e = cent + static_cast<size_t>(e) * nb * D;
-  const __nv_bfloat16* q_e = q_new + static_cast<size_t>(e) * nq * D;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nq = a.nq, nb = a.nb, nbp = a.nbp;
+  const int cells = nb * D;
+  const int n_my = blockIdx.x < a.n_inst ? (a.n_inst - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
+  const int T = (nq + kQTile - 1) / kQTile;  // tiles per instance
+  const int ncols1 = 2 * nbp;                 // screening columns (hi, lo)
+  const int acc_cols = ncols1 + kQTile;       // + the Q Q^T block
+  const uint32_t bbox = static_cast<uint32_t>(ncols1) * 128;  // bytes of one 64-column box of bmat
 
-  for (int idx = tid; idx < nb * D; idx += kUpdThreads) {
-    chat[idx] = cent_e[idx];
-    acc[idx] = 0;
+  unsigned char* base = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  unsigned char* stage_smem = base;                                             // [n_stages][kBoxes][128 x 128 B]
+  unsigned char* bmat = base + static_cast<size_t>(n_stages) * C::kStageBytes;  // [2][kBoxes][2 nbp x 128 B]
+  long long* acc = reinterpret_cast<long long*>(bmat + 2 * C::bmat_bytes(nbp));  // [2][nb][D]
+  float* cent_sm = reinterpret_cast<float*>(acc + 2 * cells);                     // [2][nb][D]
+  double* sums_sm = reinterpret_cast<double*>(cent_sm + 2 * cells);               // [nb][D]
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < n_stages; ++i) {
+      mbar_init(&full_bar[i], 1);
+      mbar_init(&empty_bar[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&accfull[i], 1);
+      mbar_init(&accfree[i], 4);  // the four screening warps
+      mbar_init(&bready[i], 1);
+      mbar_init(&bfree[i], 1);
+      mbar_init(&accdone[i], 1);
+      mbar_init(&accclear[i], 1);
+      mbar_init(&cbar[i], 1);
+      mbar_init(&sfull[i], 1);
+      mbar_init(&sempty[i], 1);
+    }
+    mbar_init(&sbar, 1);
+    mbar_init(&drain_bar, 1);
+    abort_sh = 0;
+    n_refine[0] = n_refine[1] = 0;
+    fence_mbar_init();
   }
-  if (tid < kMaxBeacons) add_cnt[tid] = 0;
-  if (tid == 0) degenerate = 0;
-  __syncthreads();
-
-  // one warp per beacon: qualification, fp64 norm, unit-length fp32 copy
-  for (int b = warp; b < nb; b += kUpdWarps) {
-    float n2 = 0.f;
-    double n2d = 0.0;
-    int nz = 0;
-    for (int i = lane; i < D; i += 32) {
-      const float c = chat[b * D + i];
-      n2 = fmaf(c, c, n2);
-      n2d = fma(static_cast<double>(c), static_cast<double>(c), n2d);
-      nz |= (c != 0.f);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      n2 += __shfl_xor_sync(0xffffffffu, n2, o);
-      nz |= __shfl_xor_sync(0xffffffffu, nz, o);
-    }
-    n2d = warp_sum_f64(n2d);
-    const int ok = (counts[static_cast<size_t>(e) * nb + b] > 0) && nz;
-    const float inv = rsqrtf(n2);
-    for (int i = lane; i < D; i += 32) chat[b * D + i] *= inv;
-    if (lane == 0) {
-      bvalid[b] = ok;
-      cn64[b] = sqrt(n2d);
-      if (ok && !(n2 > 1e-30f && n2 < 1e30f)) atomicExch(&degenerate, 1);
-    }
+  for (int c = threadIdx.x; c < 2 * cells; c += kUThreads) acc[c] = 0;
+  if (threadIdx.x < 2 * kMaxBeacons) add_cnt[threadIdx.x >> 5][threadIdx.x & 31] = 0;
+  if (warp == 1) {
+    tmem_alloc(&tmem_base_sh, 512);
+    tmem_relinquish();
   }
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_sh;
+  volatile int* abort_flag = &abort_sh;
 
-  const int quad = tid >> 2, sub = tid & 3;
-  for (int p0 = 0; p0 < nq; p0 += kPass) {
-    const int rows = min(kPass, nq - p0);
-    if (tid == 0) n_refine = 0;
-    if (tid < kMaxBeacons) bucket_fill[tid] = 0;
-    __syncthreads();
-
-    // ---- screening: 64 queries per block-wide step, 4 threads each (warp-uniform trip count)
-    for (int n0 = 0; n0 < rows; n0 += kUpdThreads / 4) {
-      const int n = n0 + quad;
-      const bool active = n < rows;
-      const __nv_bfloat16* qrow = q_e + static_cast<size_t>(p0 + (active ? n : rows - 1)) * D + 4 * sub;
-      float qv[kPer];
-      unsigned nz = 0;
-      float qa = 0.f, qb = 0.f;
-#pragma unroll
-      for (int k = 0; k < kPer / 4; ++k) {
-        const uint2 raw = __ldg(reinterpret_cast<const uint2*>(qrow + 16 * k));
-        nz |= (raw.x | raw.y) & 0x7fff7fffu;
-        const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&raw.x));
-        const float2 c = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&raw.y));
-        qv[4 * k + 0] = a.x;
-        qv[4 * k + 1] = a.y;
-        qv[4 * k + 2] = c.x;
-        qv[4 * k + 3] = c.y;
-        qa = fmaf(a.x, a.x, fmaf(a.y, a.y, qa));
-        qb = fmaf(c.x, c.x, fmaf(c.y, c.y, qb));
-      }
-      float qn2 = qa + qb;
-      qn2 += __shfl_xor_sync(0xffffffffu, qn2, 1);
-      qn2 += __shfl_xor_sync(0xffffffffu, qn2, 2);
-      nz |= __shfl_xor_sync(0xffffffffu, nz, 1);
-      nz |= __shfl_xor_sync(0xffffffffu, nz, 2);
-      float best = -INFINITY, second = -INFINITY;
-      int bi = -1;
-      for (int b = 0; b < nb; ++b) {
-        if (!bvalid[b]) continue;
-        const float* cb = chat + b * D + 4 * sub;
-        float d0 = 0.f, d1 = 0.f, d2 = 0.f, d3 = 0.f;
-#pragma unroll
-        for (int k = 0; k < kPer / 4; ++k) {
-          const float4 c4 = *reinterpret_cast<const float4*>(cb + 16 * k);
-          d0 = fmaf(qv[4 * k + 0], c4.x, d0);
-          d1 = fmaf(qv[4 * k + 1], c4.y, d1);
-          d2 = fmaf(qv[4 * k + 2], c4.z, d2);
-          d3 = fmaf(qv[4 * k + 3], c4.w, d3);
-        }
-        float dot = (d0 + d1) + (d2 + d3);
-        dot += __shfl_xor_sync(0xffffffffu, dot, 1);
-        dot += __shfl_xor_sync(0xffffffffu, dot, 2);
-        if (dot > best) {
-          second = best;
-          best = dot;
-          bi = b;
-        } else if (dot > second) {
-          second = dot;
+  if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    if (lane == 0 && n_my > 0) {
+      const uint64_t once = l2_policy_evict_first();
+      prefetch_tmap(&qmap);
+      int g = 0;
+      bool ok = true;
+      for (int i = 0; ok && i < n_my; ++i) {
+        const int e = blockIdx.x + i * gridDim.x;
+        for (int t = 0; t < T; ++t, ++g) {
+          const int st = g % n_stages;
+          if (g >= n_stages &&
+              !mbar_wait(&empty_bar[st], ((g / n_stages) - 1) & 1, abort_flag, a.err, kDevTimeoutProducer)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full_bar[st], static_cast<uint32_t>(C::kBoxes * a.box_rows * 128));
+          for (int b = 0; b < C::kBoxes; ++b)
+            tma_load_2d(stage_smem + st * C::kStageBytes + b * kQBox, &qmap, &full_bar[st], b * 64,
+                        e * nq + t * kQTile, once);
         }
       }
-      if (active && sub == 0) {
-        int a;
-        if (nz == 0 || bi < 0) {
-          a = -1;
-        } else if (degenerate || !(qn2 > 1e-30f && qn2 < 1e30f) || !(best - second > 1e-4f * sqrtf(qn2))) {
-          a = -2;  // decided exactly below
-          refine_idx[atomicAdd(&n_refine, 1)] = n;
-        } else {
-          a = bi;
+      if (!ok || *abort_flag)
+        for (int j = (g > n_stages ? g - n_stages : 0); j < g; ++j)
+          drain_wait(&full_bar[j % n_stages], (j / n_stages) & 1, a.err);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0 && n_my > 0) {
+      const uint32_t idesc1 = idesc_bf16_f32(128, ncols1), idesc2 = idesc_bf16_f32(128, kQTile);
+      int g = 0;
+      bool ok = true;
+      for (int i = 0; ok && i < n_my; ++i) {
+        const int pb = i & 1;
+        if (!mbar_wait(&bready[pb], (i >> 1) & 1, abort_flag, a.err, kDevTimeoutMma)) break;
+        for (int t = 0; t < T; ++t, ++g) {
+          const int st = g % n_stages, ab = g & 1;
+          if (!mbar_wait(&full_bar[st], (g / n_stages) & 1, abort_flag, a.err, kDevTimeoutMma) ||
+              (g >= 2 && !mbar_wait(&accfree[ab], ((g >> 1) - 1) & 1, abort_flag, a.err, kDevTimeoutMma))) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d = tmem + ab * acc_cols;
+          const uint32_t q_addr = smem_u32(stage_smem + st * C::kStageBytes);
+          const uint32_t b_addr = smem_u32(bmat + pb * C::bmat_bytes(nbp));
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t qoff = (kk >> 2) * kQBox + (kk & 3) * 32;
+            const uint32_t boff = (kk >> 2) * bbox + (kk & 3) * 32;
+            mma_bf16_ss(d, sdesc_kmajor_sw128(q_addr + qoff), sdesc_kmajor_sw128(b_addr + boff), idesc1, kk > 0);
+          }
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t qoff = (kk >> 2) * kQBox + (kk & 3) * 32;
+            mma_bf16_ss(d + ncols1, sdesc_kmajor_sw128(q_addr + qoff), sdesc_kmajor_sw128(q_addr + qoff), idesc2,
+                        kk > 0);
+          }
+          mma_commit(&accfull[ab]);
         }
-        asg[n] = a;
+        if (ok) mma_commit(&bfree[pb]);  // this instance's centroid operand is no longer read
       }
+      mma_commit(&drain_bar);
+      drain_wait(&drain_bar, 0, a.err);
     }
-    __syncthreads();
+    __syncwarp();
+  } else if (warp < 2 + kScreeners) {
+    // ---------------------------------------------------------------- screeners
+    const int ws = warp - 2;          // 0 .. 3
+    const int quarter = warp & 3;     // TMEM lane quarter (warps 2..5 cover all four)
+    const int ts = threadIdx.x - 64;  // 0 .. 127
+    const uint32_t lane_addr = static_cast<uint32_t>(quarter * 32) << 16;
+    const int n = quarter * 32 + lane;  // this thread's query row in the tile
+    const int col0 = lane * kCols;
+    const unsigned lt = (1u << lane) - 1u;
+    int g = 0;
+    for (int i = 0; i < n_my; ++i) {
+      const int e = blockIdx.x + i * gridDim.x;
+      const int pb = i & 1;
+      long long* acc_i = acc + pb * cells;
+      const float* cent_i = cent_sm + pb * cells;
+      // re-decided rows go straight into acc_i: wait until the fold two instances back cleared it
+      if (i >= 2) mbar_wait(&accclear[pb], ((i >> 1) - 1) & 1, abort_flag, a.err, kDevTimeoutEpilogue);
+      for (int t = 0; t < T; ++t, ++g) {
+        const int st = g % n_stages, ab = g & 1, ob = g & 1;
+        const int rows = min(kQTile, nq - t * kQTile);
+        const unsigned char* qs = stage_smem + st * C::kStageBytes;
+        int* assign_t = a.assign_out ? a.assign_out + static_cast<size_t>(e) * nq + t * kQTile : nullptr;
 
-    // ---- exact fp64 decisions for close calls: one warp per query
-    for (int t = warp; t < n_refine; t += kUpdWarps) {
-      const int n = refine_idx[t];
-      const __nv_bfloat16* qrow = q_e + static_cast<size_t>(p0 + n) * D;
-      double x[D / 32];
+        // ---- dots and norm of this thread's query from tensor memory
+        bool have = !*abort_flag && mbar_wait(&accfull[ab], (g >> 1) & 1, abort_flag, a.err, kDevTimeoutEpilogue);
+        have = __all_sync(0xffffffffu, have);
+        float best = -INFINITY, second = -INFINITY, qn2 = 0.f;
+        int bi = -1;
+        if (have) {
+          tc_fence_after();
+          const uint32_t d = tmem + ab * acc_cols + lane_addr;
+          float v[32];
+          tmem_ld32(d + ncols1 + quarter * 32, v);  // Q Q^T columns of this quarter: the diagonal is v[lane]
+          tmem_wait_ld();
 #pragma unroll
-      for (int k = 0; k < D / 32; ++k) x[k] = __bfloat162float(qrow[lane + 32 * k]);
-      double qq = 0.0;
+          for (int k = 0; k < 32; ++k) qn2 = (k == lane) ? v[k] : qn2;
+          for (int c0 = 0; c0 < nbp; c0 += 8) {
+            uint32_t h[8], l[8];
+            asm volatile(
+                "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                : "=r"(h[0]), "=r"(h[1]), "=r"(h[2]), "=r"(h[3]), "=r"(h[4]), "=r"(h[5]), "=r"(h[6]), "=r"(h[7])
+                : "r"(d + c0));
+            asm volatile(
+                "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                : "=r"(l[0]), "=r"(l[1]), "=r"(l[2]), "=r"(l[3]), "=r"(l[4]), "=r"(l[5]), "=r"(l[6]), "=r"(l[7])
+                : "r"(d + nbp + c0));
+            tmem_wait_ld();
 #pragma unroll
-      for (int k = 0; k < D / 32; ++k) qq = fma(x[k], x[k], qq);
-      const double nqd = sqrt(warp_sum_f64(qq));
-      double b1 = -INFINITY;
-      int best_b = -1;
-      for (int b = 0; b < nb; ++b) {
-        if (!bvalid[b]) continue;
-        double dt = 0.0;
-#pragma unroll
-        for (int k = 0; k < D / 32; ++k) dt = fma(x[k], static_cast<double>(cent_e[b * D + lane + 32 * k]), dt);
-        const double cs = warp_sum_f64(dt) / (nqd * cn64[b]);
-        if (cs > b1) {
-          b1 = cs;
-          best_b = b;
-        }
-      }
-      if (lane == 0) asg[n] = best_b;
-    }
-    __syncthreads();
-
-    // ---- bucket the pass's queries by beacon (order inside a bucket is irrelevant)
-    for (int n = tid; n < rows; n += kUpdThreads) {
-      const int b = asg[n];
-      if (b >= 0) atomicAdd(&bucket_fill[b], 1);
-      if (assign_out) assign_out[static_cast<size_t>(e) * nq + p0 + n] = b;
-    }
-    __syncthreads();
-    if (tid == 0) {
-      int run = 0;
-      for (int b = 0; b < nb; ++b) {
-        bucket_start[b] = run;
-        run += bucket_fill[b];
-        add_cnt[b] += bucket_fill[b];
-        bucket_fill[b] = 0;
-      }
-      bucket_start[nb] = run;
-    }
-    __syncthreads();
-    for (int n = tid; n < rows; n += kUpdThreads) {
-      const int b = asg[n];
-      if (b >= 0) order[bucket_start[b] + atomicAdd(&bucket_fill[b], 1)] = static_cast<short>(n);
-    }
-    __syncthreads();
-
-    // ---- exact sums: thread (group g, column col) owns cells (b, col) of beacons b = g mod kGroups
-    {
-      constexpr int kGroups = kUpdThreads / D;
-      const int col = tid % D, g = tid / D;
-      const __nv_bfloat16* qc = q_e + static_cast<size_t>(p0) * D + col;
-      for (int b = g; b < nb; b += kGroups) {
-        const int r0 = bucket_start[b], r1 = bucket_start[b + 1];
-        if (r0 == r1) continue;
-        long long s0 = 0, s1 = 0;
-        int r = r0;
-        for (; r + 8 <= r1; r += 8) {  // eight independent loads in flight
-          __nv_bfloat16 v[8];
-#pragma unroll
-          for (int u = 0; u < 8; ++u) v[u] = qc[static_cast<size_t>(order[r + u]) * D];
-#pragma unroll
-          for (int u = 0; u < 8; u += 2) {
-            s0 += to_fixed40(v[u]);
-            s1 += to_fixed40(v[u + 1]);
+            for (int u = 0; u < 8; ++u) {
+              const int b = c0 + u;
+              if (b < nb && bvalid[pb][b]) {
+                const float dot = __uint_as_float(h[u]) + __uint_as_float(l[u]);
+                if (dot > best) {
+                  second = best;
+                  best = dot;
+                  bi = b;
+                } else if (dot > second) {
+                  second = dot;
+                }
+              }
+            }
           }
         }
-        for (; r < r1; ++r) s0 += to_fixed40(qc[static_cast<size_t>(order[r]) * D]);
-        acc[b * D + col] += s0 + s1;
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&accfree[ab]);
+
+        // ---- decision; close calls go to the exact list; counts per beacon by ballot
+        int my_b = -1, my_pos = 0;
+        if (have && n < rows) {
+          if (bi >= 0 && (degenerate[pb] || !(qn2 > 1e-30f && qn2 < 1e30f) ||
+                          !(best - second > kMarginRel * sqrtf(qn2)))) {
+            refine_t[ob][atomicAdd(&n_refine[ob], 1)] = n;
+          } else {
+            my_b = bi;
+            if (assign_t) assign_t[n] = bi;
+          }
+        }
+        for (int b = 0; b < nb; ++b) {
+          const unsigned m = __ballot_sync(0xffffffffu, my_b == b);
+          if (lane == b) cnt_w[ob][quarter][b] = __popc(m);
+          if (my_b == b) my_pos = __popc(m & lt);
+        }
+        named_barrier(1, 32 * kScreeners);
+
+        // ---- sorted row list for the accumulators (its buffer is free once they are done with tile g - 2)
+        if (g >= 2) mbar_wait(&sempty[ob], ((g >> 1) - 1) & 1, abort_flag, a.err, kDevTimeoutEpilogue);
+        if (ts == 0) n_refine[ob ^ 1] = 0;  // the next tile's list; its previous readers finished a tile ago
+        {
+          int tot = 0, mine = 0;
+          if (lane < nb)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const int c = cnt_w[ob][q][lane];
+              tot += c;
+              mine += (q < quarter) ? c : 0;
+            }
+          int incl = tot;
+#pragma unroll
+          for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += y;
+          }
+          const int off = incl - tot + mine;  // where this warp's rows of beacon `lane` start
+          const int my_off = __shfl_sync(0xffffffffu, off, my_b < 0 ? 0 : my_b);
+          if (my_b >= 0) order_t[ob][my_off + my_pos] = n | (my_b << 8);
+          if (quarter == 0) {
+            if (lane == 31) n_asg_sh[ob] = incl;
+            if (lane < nb && tot > 0) atomicAdd(&add_cnt[pb][lane], tot);  // refinements add concurrently
+          }
+        }
+
+        // ---- exact decisions for close calls, one warp per query; the row is added here
+        const int nr = n_refine[ob];
+        for (int k = ws; k < nr; k += kScreeners) {
+          const int r = refine_t[ob][k];
+          double x[D / 32];
+#pragma unroll
+          for (int j = 0; j < D / 32; ++j)
+            x[j] = __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(qs + sw128_offset(r, lane + 32 * j, kQBox)));
+          double qq = 0.0;
+#pragma unroll
+          for (int j = 0; j < D / 32; ++j) qq = fma(x[j], x[j], qq);
+          qq = warp_sum_f64(qq);
+          double b1 = -INFINITY;
+          int best_b = -1;
+          if (qq > 0.0)
+            for (int b = 0; b < nb; ++b) {
+              if (!bvalid[pb][b]) continue;
+              double dt = 0.0;
+#pragma unroll
+              for (int j = 0; j < D / 32; ++j) dt = fma(x[j], static_cast<double>(cent_i[b * D + lane + 32 * j]), dt);
+              const double cs = warp_sum_f64(dt) * cninv[pb][b];
+              if (cs > b1) {
+                b1 = cs;
+                best_b = b;
+              }
+            }
+          if (lane == 0) {
+            if (assign_t) assign_t[r] = best_b;
+            if (best_b >= 0) atomicAdd(&add_cnt[pb][best_b], 1);
+          }
+          if (best_b >= 0) {
+            long long sr[kCols];
+#pragma unroll
+            for (int c = 0; c < kCols; ++c) sr[c] = 0;
+            add_fixed<kCols>(sr, qs + sw128_offset(r, col0, kQBox));
+#pragma unroll
+            for (int c = 0; c < kCols; ++c)
+              atomicAdd(reinterpret_cast<unsigned long long*>(&acc_i[best_b * D + col0 + c]),
+                        static_cast<unsigned long long>(sr[c]));
+          }
+        }
+        named_barrier(1, 32 * kScreeners);
+        if (ts == 0) mbar_arrive(&sfull[ob]);
       }
     }
-    __syncthreads();
+  } else if (warp < 2 + kScreeners + kAccum) {
+    // ---------------------------------------------------------------- accumulators
+    const int wa = warp - 2 - kScreeners;               // 0 .. 7
+    const int ta = threadIdx.x - 32 * (2 + kScreeners);  // 0 .. 255
+    const int col0 = lane * kCols;
+    const int chunk = (col0 & 63) >> 3;
+    const uint32_t lane_off = (col0 >> 6) * kQBox + ((col0 & 7) << 1);
+    int g = 0;
+    for (int i = 0; i < n_my; ++i) {
+      const int pb = i & 1;
+      long long* acc_i = acc + pb * cells;
+      if (i >= 2) mbar_wait(&accclear[pb], ((i >> 1) - 1) & 1, abort_flag, a.err, kDevTimeoutEpilogue);
+      for (int t = 0; t < T; ++t, ++g) {
+        const int st = g % n_stages, ob = g & 1;
+        const unsigned char* qs = stage_smem + st * C::kStageBytes + lane_off;
+        const bool ready = mbar_wait(&sfull[ob], (g >> 1) & 1, abort_flag, a.err, kDevTimeoutEpilogue);
+        const int n_asg = ready ? n_asg_sh[ob] : 0;
+        const int* ord = order_t[ob];
+        const int p1 = (wa + 1) * n_asg / kAccum;
+        int p = wa * n_asg / kAccum;
+        auto row_ptr = [&](int en) {
+          const int r = en & 0xff;
+          return qs + r * 128 + ((chunk ^ (r & 7)) << 4);
+        };
+        Parts s[kCols];
+#pragma unroll
+        for (int c = 0; c < kCols; ++c) s[c] = Parts{0.f, 0.f, 0.f};
+        int cur = -1;
+        auto flush = [&]() {
+#pragma unroll
+          for (int c = 0; c < kCols; ++c) {
+            atomicAdd(reinterpret_cast<unsigned long long*>(&acc_i[cur * D + col0 + c]),
+                      static_cast<unsigned long long>(fixed40(s[c])));
+            s[c] = Parts{0.f, 0.f, 0.f};
+          }
+        };
+        while (p < p1) {
+          if (p + 4 <= p1) {
+            const int e0 = ord[p], e3 = ord[p + 3];
+            if ((e0 >> 8) == cur && (e3 >> 8) == cur) {  // sorted: the four rows share the beacon
+              const int e1 = ord[p + 1], e2 = ord[p + 2];
+              add_parts<kCols>(s, row_ptr(e0));
+              add_parts<kCols>(s, row_ptr(e1));
+              add_parts<kCols>(s, row_ptr(e2));
+              add_parts<kCols>(s, row_ptr(e3));
+              p += 4;
+              continue;
+            }
+          }
+          const int en = ord[p];
+          const int b = en >> 8;
+          if (b != cur) {
+            if (cur >= 0) flush();
+            cur = b;
+          }
+          add_parts<kCols>(s, row_ptr(en));
+          ++p;
+        }
+        if (cur >= 0) flush();
+        named_barrier(2, 32 * kAccum);
+        if (ta == 0) {
+          mbar_arrive(&empty_bar[st]);  // the stage's queries are no longer read
+          mbar_arrive(&sempty[ob]);
+          if (t == T - 1) mbar_arrive(&accdone[pb]);  // this instance's sums are complete
+        }
+      }
+    }
+  } else {
+    // ---------------------------------------------------------------- bookkeeping
+    const int wk = warp - 2 - kScreeners - kAccum;  // 0 .. 3
+    const int tk = threadIdx.x - 32 * (2 + kScreeners + kAccum);
+    const uint32_t cbytes = static_cast<uint32_t>(cells) * 4, sbytes = static_cast<uint32_t>(cells) * 8;
+    auto inst = [&](int idx) { return blockIdx.x + idx * gridDim.x; };
+    auto issue_cent = [&](int idx) {  // centroids of instance idx into cent_sm[idx & 1]
+      fence_proxy_async_smem();
+      mbar_arrive_expect_tx(&cbar[idx & 1], cbytes);
+      bulk_copy_g2s(cent_sm + (idx & 1) * cells, a.cent + static_cast<size_t>(inst(idx)) * cells, cbytes,
+                    &cbar[idx & 1]);
+    };
+    auto issue_sums = [&](int idx) {
+      fence_proxy_async_smem();
+      mbar_arrive_expect_tx(&sbar, sbytes);
+      bulk_copy_g2s(sums_sm, a.sums + static_cast<size_t>(inst(idx)) * cells, sbytes, &sbar);
+    };
+    auto build = [&](int idx) {
+      const int pb = idx & 1;
+      const int e = inst(idx);
+      if (tk < nb) cnt_old[pb][tk] = a.counts[static_cast<size_t>(e) * nb + tk];
+      if (tk == 0) degenerate[pb] = 0;
+      mbar_wait(&cbar[pb], (idx >> 1) & 1, abort_flag, a.err, kDevTimeoutEpilogue);
+      if (idx >= 2) mbar_wait(&bfree[pb], ((idx >> 1) - 1) & 1, abort_flag, a.err, kDevTimeoutEpilogue);
+      named_barrier(3, 32 * kKeepers);
+      const float* cs = cent_sm + pb * cells;
+      unsigned char* bm = bmat + pb * C::bmat_bytes(nbp);
+      for (int b = wk; b < nbp; b += kKeepers) {
+        float c[D / 32];
+        float n2 = 0.f;
+        double n2d = 0.0;
+        int nz = 0;
+#pragma unroll
+        for (int k = 0; k < D / 32; ++k) {
+          c[k] = b < nb ? cs[b * D + lane + 32 * k] : 0.f;
+          n2 = fmaf(c[k], c[k], n2);
+          n2d = fma(static_cast<double>(c[k]), static_cast<double>(c[k]), n2d);
+          nz |= (c[k] != 0.f);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          n2 += __shfl_xor_sync(0xffffffffu, n2, o);
+          nz |= __shfl_xor_sync(0xffffffffu, nz, o);
+        }
+        n2d = warp_sum_f64(n2d);
+        const bool ok = b < nb && cnt_old[pb][b] > 0 && nz;
+        const float inv = ok ? rsqrtf(n2) : 0.f;
+#pragma unroll
+        for (int k = 0; k < D / 32; ++k) {
+          const int col = lane + 32 * k;
+          const float u = c[k] * inv;
+          const __nv_bfloat16 hi = __float2bfloat16_rn(u);
+          const __nv_bfloat16 lo = __float2bfloat16_rn(u - __bfloat162float(hi));
+          *reinterpret_cast<__nv_bfloat16*>(bm + sw128_offset(b, col, bbox)) = hi;
+          *reinterpret_cast<__nv_bfloat16*>(bm + sw128_offset(nbp + b, col, bbox)) = lo;
+        }
+        if (lane == 0 && b < nb) {
+          bvalid[pb][b] = ok;
+          cninv[pb][b] = ok ? __drcp_rn(sqrt(n2d)) : 0.0;
+          if (ok && !(n2 > 1e-30f && n2 < 1e30f)) degenerate[pb] = 1;
+        }
+      }
+      fence_proxy_async_smem();  // generic-proxy writes, read next by the tensor cores
+      named_barrier(3, 32 * kKeepers);
+      if (tk == 0) mbar_arrive(&bready[pb]);
+    };
+    auto fold = [&](int idx) {
+      const int pb = idx & 1;
+      const int e = inst(idx);
+      long long* acc_i = acc + pb * cells;
+      mbar_wait(&accdone[pb], (idx >> 1) & 1, abort_flag, a.err, kDevTimeoutEpilogue);
+      mbar_wait(&sbar, idx & 1, abort_flag, a.err, kDevTimeoutEpilogue);
+      if (tk < nb) rcp_sh[tk] = __drcp_rn(static_cast<double>(cnt_old[pb][tk] + add_cnt[pb][tk]));
+      named_barrier(3, 32 * kKeepers);
+      for (int c = tk; c < cells; c += 32 * kKeepers) {
+        const int b = c / D;
+        if (add_cnt[pb][b] > 0) {
+          const size_t gi = static_cast<size_t>(e) * cells + c;
+          const double s_new = __dadd_rn(sums_sm[c], static_cast<double>(acc_i[c]) * 0x1p-40);
+          a.sums[gi] = s_new;
+          a.cent[gi] = __double2float_rn(__dmul_rn(s_new, rcp_sh[b]));
+        }
+        acc_i[c] = 0;
+      }
+      named_barrier(3, 32 * kKeepers);
+      if (tk < nb) {
+        if (add_cnt[pb][tk] > 0) a.counts[static_cast<size_t>(e) * nb + tk] = cnt_old[pb][tk] + add_cnt[pb][tk];
+        add_cnt[pb][tk] = 0;
+      }
+      named_barrier(3, 32 * kKeepers);
+      if (tk == 0) {
+        mbar_arrive(&accclear[pb]);
+        if (idx + 1 < n_my) issue_sums(idx + 1);
+        if (idx + 2 < n_my) issue_cent(idx + 2);
+      }
+    };
+
+    if (n_my > 0) {
+      if (tk == 0) {
+        issue_cent(0);
+        issue_sums(0);
+        if (n_my > 1) issue_cent(1);
+      }
+      build(0);
+      for (int i = 0; i < n_my; ++i) {
+        if (i + 1 < n_my) build(i + 1);
+        fold(i);
+      }
+    }
   }
 
-  // ---- fold the call into the running state
-  for (int idx = tid; idx < nb * D; idx += kUpdThreads) {
-    const int b = idx / D;
-    const int add = add_cnt[b];
-    if (add == 0) continue;
-    const size_t g = static_cast<size_t>(e) * nb * D + idx;
-    const double s_new = __dadd_rn(sums[g], static_cast<double>(acc[idx]) * 0x1p-40);
-    sums[g] = s_new;
-    const long long cnt = counts[static_cast<size_t>(e) * nb + b] + add;
-    cent[g] = __double2float_rn(__dmul_rn(s_new, __drcp_rn(static_cast<double>(cnt))));
-  }
+  tc_fence_before();
   __syncthreads();
-  if (tid < nb) counts[static_cast<size_t>(e) * nb + tid] += add_cnt[tid];
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
 }
 
 }  // namespace
 
-cudaError_t launch_update(const Shape& s, const __nv_bfloat16* q_new, int n_new, float* cent, double* sums,
-                          long long* counts, int* assign_out, cudaStream_t st) {
-  const int nq = s.G * n_new;
-  const int nb = s.nb;
-  const size_t smem = static_cast<size_t>(nb) * s.d * (sizeof(long long) + sizeof(float));
+cudaError_t launch_update(const Shape& s, const CUtensorMap& qmap, int box_rows, int n_new, float* cent,
+                          double* sums, long long* counts, int* assign_out, int* err, cudaStream_t st) {
+  UpdArgs a;
+  a.n_inst = s.n_inst;
+  a.nq = s.G * n_new;
+  a.box_rows = box_rows;
+  a.nb = s.nb;
+  a.nbp = (s.nb + 7) / 8 * 8;
+  a.cent = cent;
+  a.sums = sums;
+  a.counts = counts;
+  a.assign_out = assign_out;
+  a.err = err;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int grid = s.n_inst < sms ? s.n_inst : sms;
   if (s.d == 128) {
-    cudaFuncSetAttribute(update_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-    update_kernel<128><<<s.n_inst, kUpdThreads, smem, st>>>(q_new, nq, nb, cent, sums, counts, assign_out);
+    using C = UpdCfg<128>;
+    const size_t smem = C::smem_bytes(a.nb, a.nbp);
+    cudaError_t e =
+        cudaFuncSetAttribute(update_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    update_kernel<128><<<grid, kUThreads, smem, st>>>(qmap, a, C::stages(a.nb, a.nbp));
   } else {
-    cudaFuncSetAttribute(update_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-    update_kernel<64><<<s.n_inst, kUpdThreads, smem, st>>>(q_new, nq, nb, cent, sums, counts, assign_out);
+    using C = UpdCfg<64>;
+    const size_t smem = C::smem_bytes(a.nb, a.nbp);
+    cudaError_t e =
+        cudaFuncSetAttribute(update_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    update_kernel<64><<<grid, kUThreads, smem, st>>>(qmap, a, C::stages(a.nb, a.nbp));
   }
   return cudaGetLastError();
 }
