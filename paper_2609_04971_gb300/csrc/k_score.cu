@@ -233,8 +233,9 @@ __global__ void __launch_bounds__(kScThreads, 1)
   const int str_slot = ring;                         // pass-1 streaming slots; +2, +3: pass-2 slots
   const uint32_t qbox = static_cast<uint32_t>(s.n_obs_pad) * 128;
 
-  unsigned char* base = reinterpret_cast<unsigned char*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  // 1024-byte aligned (the 128-byte swizzle pattern repeats every 1024 bytes);
+  // offset from the __shared__ array itself so that accesses stay shared-space
+  unsigned char* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   unsigned char* q_smem = base;                         // [2 buffers][kBoxes][n_obs_pad rows x 128 B]
   unsigned char* k_smem = base + 2 * C::kBoxes * qbox;  // [n_stages][kBoxes][128 rows x 128 B]
   float2* recv = reinterpret_cast<float2*>(k_smem + n_stages * C::kBoxes * kBoxBytes);  // [2][csize][N]

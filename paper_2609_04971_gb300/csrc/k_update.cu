@@ -10,13 +10,14 @@
 // c_hi = bf16(c / |c|) and c_lo = bf16(c / |c| - c_hi), so dot_b = D1[:, b] +
 // D1[:, nbp + b] carries the unit-centroid dot to about 2^-16 |q| (bf16 x bf16
 // products are exact, the accumulation is fp32); D2 = Q x Q^T gives |q|^2 on
-// its diagonal.  When best and second-best dots differ by at most 4e-4 |q|
-// (several times their error bound), the query is re-decided exactly: the
-// beacon maximising (q . c_b) / |c_b| with fp64 products, warp-parallel fp64
-// sums and a correctly rounded fp64 1 / |c_b|; this agrees with the cosine
-// (q . c_b) / (|q| |c_b|) evaluated sequentially in fp64 except at ties below
-// ~1e-15 (the lowest beacon wins ties).  Zero queries and instances without a
-// valid beacon give -1.
+// its diagonal.  When best and second-best dots differ by at most 1e-4 |q|
+// (about twice the bound on their difference's error: 2^-17 |q| per dot from
+// the hi/lo split, 128 fp32 accumulation steps), the query is re-decided
+// exactly: the beacon maximising (q . c_b) / |c_b| in double-float arithmetic
+// (exact products, TwoSum accumulation, 1 / |c_b| rounded from fp64), which
+// agrees with the cosine (q . c_b) / (|q| |c_b|) evaluated in fp64 except at
+// ties below ~1e-12 (the lowest beacon wins ties).  Zero queries and instances
+// without a valid beacon give -1.
 //
 // Sums: int64 fixed point with 40 fractional bits.  A tile's screened rows
 // are sorted by beacon (ballot counting sort); each accumulator warp takes an
@@ -28,11 +29,11 @@
 // added once to the fp64 running sum, and c = fp32(sum * (1 / count)) in
 // fp64, within one fp32 ulp of fp32(sum / count).
 //
-// Warp roles (18 warps): warp 0 TMA producer; warp 1 TMEM allocation and MMA
+// Warp roles (26 warps): warp 0 TMA producer; warp 1 TMEM allocation and MMA
 // issue; warps 2..5 screeners (one per TMEM lane quarter: decisions, the
-// sorted row list of the tile, exact re-decisions); warps 6..13 accumulators
+// sorted row list of the tile, exact re-decisions); warps 6..21 accumulators
 // (the sums of a tile, while the screeners work on the next one; the row
-// lists are double-buffered); warps 14..17 bookkeeping: they build the
+// lists are double-buffered); warps 22..25 bookkeeping: they build the
 // unit-centroid operand of the next instance and fold the finished one into
 // the running state, from centroids and sums brought in by bulk copies
 // (accumulators double-buffered by instance).  All waits are bounded.
@@ -43,14 +44,15 @@ namespace bkv {
 namespace {
 
 constexpr int kScreeners = 4;
-constexpr int kAccum = 8;
+constexpr int kAccum = 16;
 constexpr int kKeepers = 4;
 constexpr int kUThreads = 32 * (2 + kScreeners + kAccum + kKeepers);
 constexpr int kQTile = 128;                 // queries per tile (MMA M)
 constexpr uint32_t kQBox = 128 * 128;       // [128 rows][64 bf16] swizzled box slot
 constexpr int kUMaxStages = 8;
 constexpr size_t kUSmemBudget = 216 * 1024;
-constexpr float kMarginRel = 4e-4f;
+constexpr float kMarginRel = 1e-4f;
+constexpr int kGroup = 4;  // rows an accumulator lane sums per step when they share a beacon
 
 struct UpdArgs {
   int n_inst, nq, nb, nbp;  // instances, queries per instance, beacons, beacons padded to 8
@@ -133,26 +135,48 @@ __device__ __forceinline__ void add_fixed(long long (&s)[kCols], const unsigned 
   }
 }
 
+// Double-float arithmetic (an unevaluated sum hi + lo of two fp32 values,
+// about 48 significant bits) for the exact re-decisions: fp64 is slow on
+// this part.  TwoSum (Knuth) and the FMA-based exact product.
+struct DF {
+  float hi, lo;
+};
+
+__device__ __forceinline__ DF df_add(DF a, DF b) {
+  const float s = __fadd_rn(a.hi, b.hi);
+  const float bb = __fadd_rn(s, -a.hi);
+  const float err = __fadd_rn(__fadd_rn(a.hi, -__fadd_rn(s, -bb)), __fadd_rn(b.hi, -bb));
+  const float lo = __fadd_rn(__fadd_rn(a.lo, b.lo), err);
+  const float t = __fadd_rn(s, lo);
+  return DF{t, __fadd_rn(lo, -__fadd_rn(t, -s))};
+}
+
+__device__ __forceinline__ DF df_two_prod(float a, float b) {
+  const float p = __fmul_rn(a, b);
+  return DF{p, __fmaf_rn(a, b, -p)};
+}
+
+__device__ __forceinline__ DF df_mul(DF a, DF b) {
+  const float p = __fmul_rn(a.hi, b.hi);
+  float e = __fmaf_rn(a.hi, b.hi, -p);
+  e = __fmaf_rn(a.hi, b.lo, e);
+  e = __fmaf_rn(a.lo, b.hi, e);
+  const float t = __fadd_rn(p, e);
+  return DF{t, __fadd_rn(e, -__fadd_rn(t, -p))};
+}
+
+__device__ __forceinline__ bool df_gt(DF a, DF b) { return a.hi > b.hi || (a.hi == b.hi && a.lo > b.lo); }
+
 // Exact sums of bf16 values without a 64-bit conversion per element: x is
 // split into xh = x rounded to a multiple of 2^-3, xm = the rest rounded to a
 // multiple of 2^-20 and xl = what remains (magic-number rounding, fp32 adds
-// only); each part's fp32 running sum is exact over up to 128 values with
-// |x| < 2^14 (xl is exact for |x| >= 2^-31).  `fixed40` turns the three sums
-// into round(sum * 2^40) with 32-bit conversions.
+// only, two columns per paired-fp32 instruction); each part's fp32 running
+// sum is exact over up to 128 values with |x| < 2^14 (xl is exact for
+// |x| >= 2^-31).  `fixed40` turns the three sums into round(sum * 2^40) with
+// 32-bit conversions.
 struct Parts {
   float h, m, l;
 };
-
-__device__ __forceinline__ void parts_add(Parts& p, float x) {
-  constexpr float kM1 = 1572864.0f;  // 1.5 * 2^20: x + kM1 rounds x to a multiple of 2^-3
-  constexpr float kM2 = 12.0f;       // 1.5 * 2^3: r + kM2 rounds r to a multiple of 2^-20
-  const float xh = __fadd_rn(__fadd_rn(x, kM1), -kM1);
-  const float r = __fadd_rn(x, -xh);
-  const float xm = __fadd_rn(__fadd_rn(r, kM2), -kM2);
-  p.h = __fadd_rn(p.h, xh);
-  p.m = __fadd_rn(p.m, xm);
-  p.l = __fadd_rn(p.l, __fadd_rn(r, -xm));
-}
 
 __device__ __forceinline__ long long fixed40(const Parts& p) {
   const long long h = static_cast<long long>(__float2int_rn(p.h * 8.0f)) << 37;
@@ -161,20 +185,42 @@ __device__ __forceinline__ long long fixed40(const Parts& p) {
   return h + m + l;
 }
 
-// Adds the kCols bf16 values at p (columns col0 ..) to the part sums.
-template <int kCols>
-__device__ __forceinline__ void add_parts(Parts (&s)[kCols], const unsigned char* p) {
-  if constexpr (kCols == 4) {
-    const uint2 w = *reinterpret_cast<const uint2*>(p);
-    parts_add(s[0], __uint_as_float(w.x << 16));
-    parts_add(s[1], __uint_as_float(w.x & 0xffff0000u));
-    parts_add(s[2], __uint_as_float(w.y << 16));
-    parts_add(s[3], __uint_as_float(w.y & 0xffff0000u));
-  } else {
-    const uint32_t w = *reinterpret_cast<const uint32_t*>(p);
-    parts_add(s[0], __uint_as_float(w << 16));
-    parts_add(s[1], __uint_as_float(w & 0xffff0000u));
-  }
+// The same split for two adjacent columns at once, on packed f32x2 values
+// (low word: the first column), with Blackwell's paired fp32 adds.
+struct Parts2 {
+  unsigned long long h, m, l;
+};
+
+__device__ __forceinline__ unsigned long long f2_add(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ unsigned long long f2_sub(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+// w holds two bf16 values (low half: the first column).
+__device__ __forceinline__ void parts2_add(Parts2& p, uint32_t w) {
+  constexpr unsigned long long kM1 = 0x49C0000049C00000ull;  // {1.5 * 2^20, 1.5 * 2^20}
+  constexpr unsigned long long kM2 = 0x4140000041400000ull;  // {12, 12}
+  const unsigned long long x = static_cast<unsigned long long>(w << 16) |
+                               (static_cast<unsigned long long>(w & 0xffff0000u) << 32);
+  const unsigned long long xh = f2_sub(f2_add(x, kM1), kM1);
+  const unsigned long long r = f2_sub(x, xh);
+  const unsigned long long xm = f2_sub(f2_add(r, kM2), kM2);
+  p.h = f2_add(p.h, xh);
+  p.m = f2_add(p.m, xm);
+  p.l = f2_add(p.l, f2_sub(r, xm));
+}
+
+// Column `second` (0 or 1) of a packed pair of part sums.
+__device__ __forceinline__ Parts parts2_get(const Parts2& p, int second) {
+  const int sh = second ? 32 : 0;
+  return Parts{__uint_as_float(static_cast<uint32_t>(p.h >> sh)), __uint_as_float(static_cast<uint32_t>(p.m >> sh)),
+               __uint_as_float(static_cast<uint32_t>(p.l >> sh))};
 }
 
 template <int D>
@@ -194,7 +240,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
   __shared__ int cnt_w[2][4][kMaxBeacons];
   __shared__ int add_cnt[2][kMaxBeacons];
   __shared__ int bvalid[2][kMaxBeacons];
-  __shared__ double cninv[2][kMaxBeacons];
+  __shared__ DF cninv[2][kMaxBeacons];  // 1 / |c_b| as a double-float
   __shared__ long long cnt_old[2][kMaxBeacons];
   __shared__ double rcp_sh[kMaxBeacons];
   __shared__ int degenerate[2];
@@ -208,11 +254,14 @@ __global__ void __launch_bounds__(kUThreads, 1)
   const int acc_cols = ncols1 + kQTile;       // + the Q Q^T block
   const uint32_t bbox = static_cast<uint32_t>(ncols1) * 128;  // bytes of one 64-column box of bmat
 
-  unsigned char* base = reinterpret_cast<unsigned char*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  // 1024-byte aligned (the 128-byte swizzle pattern repeats every 1024 bytes);
+  // offset from the __shared__ array itself so that accesses stay shared-space
+  unsigned char* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   unsigned char* stage_smem = base;                                             // [n_stages][kBoxes][128 x 128 B]
   unsigned char* bmat = base + static_cast<size_t>(n_stages) * C::kStageBytes;  // [2][kBoxes][2 nbp x 128 B]
-  long long* acc = reinterpret_cast<long long*>(bmat + 2 * C::bmat_bytes(nbp));  // [2][nb][D]
+  // [2][nb][D]; column 4 l + c of a beacon row (l = lane, c < D / 32) sits at
+  // c * 32 + l, so that the 64-bit updates of a warp hit consecutive words
+  long long* acc = reinterpret_cast<long long*>(bmat + 2 * C::bmat_bytes(nbp));
   float* cent_sm = reinterpret_cast<float*>(acc + 2 * cells);                     // [2][nb][D]
   double* sums_sm = reinterpret_cast<double*>(cent_sm + 2 * cells);               // [nb][D]
 
@@ -433,24 +482,26 @@ __global__ void __launch_bounds__(kUThreads, 1)
         const int nr = n_refine[ob];
         for (int k = ws; k < nr; k += kScreeners) {
           const int r = refine_t[ob][k];
-          double x[D / 32];
+          float x[D / 32];
+          int nz = 0;
 #pragma unroll
-          for (int j = 0; j < D / 32; ++j)
+          for (int j = 0; j < D / 32; ++j) {
             x[j] = __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(qs + sw128_offset(r, lane + 32 * j, kQBox)));
-          double qq = 0.0;
-#pragma unroll
-          for (int j = 0; j < D / 32; ++j) qq = fma(x[j], x[j], qq);
-          qq = warp_sum_f64(qq);
-          double b1 = -INFINITY;
+            nz |= x[j] != 0.f;
+          }
+          DF b1{-INFINITY, 0.f};
           int best_b = -1;
-          if (qq > 0.0)
+          if (__any_sync(0xffffffffu, nz))  // a zero query stays unassigned
             for (int b = 0; b < nb; ++b) {
               if (!bvalid[pb][b]) continue;
-              double dt = 0.0;
+              DF dt{0.f, 0.f};
 #pragma unroll
-              for (int j = 0; j < D / 32; ++j) dt = fma(x[j], static_cast<double>(cent_i[b * D + lane + 32 * j]), dt);
-              const double cs = warp_sum_f64(dt) * cninv[pb][b];
-              if (cs > b1) {
+              for (int j = 0; j < D / 32; ++j) dt = df_add(dt, df_two_prod(x[j], cent_i[b * D + lane + 32 * j]));
+#pragma unroll
+              for (int o = 16; o > 0; o >>= 1)
+                dt = df_add(dt, DF{__shfl_xor_sync(0xffffffffu, dt.hi, o), __shfl_xor_sync(0xffffffffu, dt.lo, o)});
+              const DF cs = df_mul(dt, cninv[pb][b]);
+              if (best_b < 0 || df_gt(cs, b1)) {
                 b1 = cs;
                 best_b = b;
               }
@@ -466,7 +517,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
             add_fixed<kCols>(sr, qs + sw128_offset(r, col0, kQBox));
 #pragma unroll
             for (int c = 0; c < kCols; ++c)
-              atomicAdd(reinterpret_cast<unsigned long long*>(&acc_i[best_b * D + col0 + c]),
+              atomicAdd(reinterpret_cast<unsigned long long*>(&acc_i[best_b * D + c * 32 + lane]),
                         static_cast<unsigned long long>(sr[c]));
           }
         }
@@ -476,8 +527,8 @@ __global__ void __launch_bounds__(kUThreads, 1)
     }
   } else if (warp < 2 + kScreeners + kAccum) {
     // ---------------------------------------------------------------- accumulators
-    const int wa = warp - 2 - kScreeners;               // 0 .. 7
-    const int ta = threadIdx.x - 32 * (2 + kScreeners);  // 0 .. 255
+    const int wa = warp - 2 - kScreeners;               // 0 .. kAccum - 1
+    const int ta = threadIdx.x - 32 * (2 + kScreeners);  // 0 .. 32 * kAccum - 1
     const int col0 = lane * kCols;
     const int chunk = (col0 & 63) >> 3;
     const uint32_t lane_off = (col0 >> 6) * kQBox + ((col0 & 7) << 1);
@@ -498,30 +549,35 @@ __global__ void __launch_bounds__(kUThreads, 1)
           const int r = en & 0xff;
           return qs + r * 128 + ((chunk ^ (r & 7)) << 4);
         };
-        Parts s[kCols];
+        constexpr int kPairs = kCols / 2;
+        Parts2 s[kPairs];
 #pragma unroll
-        for (int c = 0; c < kCols; ++c) s[c] = Parts{0.f, 0.f, 0.f};
+        for (int h = 0; h < kPairs; ++h) s[h] = Parts2{0ull, 0ull, 0ull};
         int cur = -1;
         auto flush = [&]() {
 #pragma unroll
-          for (int c = 0; c < kCols; ++c) {
-            atomicAdd(reinterpret_cast<unsigned long long*>(&acc_i[cur * D + col0 + c]),
-                      static_cast<unsigned long long>(fixed40(s[c])));
-            s[c] = Parts{0.f, 0.f, 0.f};
+          for (int c = 0; c < kCols; ++c)
+            atomicAdd(reinterpret_cast<unsigned long long*>(&acc_i[cur * D + c * 32 + lane]),
+                      static_cast<unsigned long long>(fixed40(parts2_get(s[c >> 1], c & 1))));
+#pragma unroll
+          for (int h = 0; h < kPairs; ++h) s[h] = Parts2{0ull, 0ull, 0ull};
+        };
+        auto add_row = [&](const unsigned char* rp) {
+          if constexpr (kCols == 4) {
+            const uint2 v = *reinterpret_cast<const uint2*>(rp);
+            parts2_add(s[0], v.x);
+            parts2_add(s[1 % kPairs], v.y);
+          } else {
+            parts2_add(s[0], *reinterpret_cast<const uint32_t*>(rp));
           }
         };
         while (p < p1) {
-          if (p + 4 <= p1) {
-            const int e0 = ord[p], e3 = ord[p + 3];
-            if ((e0 >> 8) == cur && (e3 >> 8) == cur) {  // sorted: the four rows share the beacon
-              const int e1 = ord[p + 1], e2 = ord[p + 2];
-              add_parts<kCols>(s, row_ptr(e0));
-              add_parts<kCols>(s, row_ptr(e1));
-              add_parts<kCols>(s, row_ptr(e2));
-              add_parts<kCols>(s, row_ptr(e3));
-              p += 4;
-              continue;
-            }
+          if (p + kGroup <= p1 && (ord[p] >> 8) == cur && (ord[p + kGroup - 1] >> 8) == cur) {
+            // sorted: the group's rows share the beacon
+#pragma unroll
+            for (int r = 0; r < kGroup; ++r) add_row(row_ptr(ord[p + r]));
+            p += kGroup;
+            continue;
           }
           const int en = ord[p];
           const int b = en >> 8;
@@ -529,7 +585,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
             if (cur >= 0) flush();
             cur = b;
           }
-          add_parts<kCols>(s, row_ptr(en));
+          add_row(row_ptr(en));
           ++p;
         }
         if (cur >= 0) flush();
@@ -599,7 +655,9 @@ __global__ void __launch_bounds__(kUThreads, 1)
         }
         if (lane == 0 && b < nb) {
           bvalid[pb][b] = ok;
-          cninv[pb][b] = ok ? __drcp_rn(sqrt(n2d)) : 0.0;
+          const double inv = ok ? __drcp_rn(sqrt(n2d)) : 0.0;
+          const float inv_hi = __double2float_rn(inv);
+          cninv[pb][b] = DF{inv_hi, __double2float_rn(inv - static_cast<double>(inv_hi))};
           if (ok && !(n2 > 1e-30f && n2 < 1e30f)) degenerate[pb] = 1;
         }
       }
@@ -616,14 +674,15 @@ __global__ void __launch_bounds__(kUThreads, 1)
       if (tk < nb) rcp_sh[tk] = __drcp_rn(static_cast<double>(cnt_old[pb][tk] + add_cnt[pb][tk]));
       named_barrier(3, 32 * kKeepers);
       for (int c = tk; c < cells; c += 32 * kKeepers) {
-        const int b = c / D;
+        const int b = c / D, col = c - b * D;
+        const int ai = b * D + (col % kCols) * 32 + col / kCols;  // the accumulator cell of (b, col)
         if (add_cnt[pb][b] > 0) {
           const size_t gi = static_cast<size_t>(e) * cells + c;
-          const double s_new = __dadd_rn(sums_sm[c], static_cast<double>(acc_i[c]) * 0x1p-40);
+          const double s_new = __dadd_rn(sums_sm[c], static_cast<double>(acc_i[ai]) * 0x1p-40);
           a.sums[gi] = s_new;
           a.cent[gi] = __double2float_rn(__dmul_rn(s_new, rcp_sh[b]));
         }
-        acc_i[c] = 0;
+        acc_i[ai] = 0;  // the cell this thread read: no other thread touches it
       }
       named_barrier(3, 32 * kKeepers);
       if (tk < nb) {
