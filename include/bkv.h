@@ -172,6 +172,19 @@ int bkv_set_state(bkv_ctx* ctx, const float* centroids, const double* sums, cons
 int bkv_sync(bkv_ctx* ctx);
 
 /*
+ * Diagnostic with no counterpart in the paper: checks the expiry path of the
+ * library's bounded device waits.  After a bkv_sync of earlier work, launches
+ * on the context's stream one kernel that waits on a barrier nothing
+ * completes, through the same wait routine the other kernels use, with the
+ * limit limit_ns (1e3 .. 1e10 ns) instead of the kernels' 1 s; the wait
+ * expires, the kernel records the timeout in the device error word and
+ * returns.  Returns what bkv_sync then reports: BKV_ETIMEOUT when the path
+ * works, with the error word cleared and the context usable; BKV_EINVAL for
+ * a NULL context or a limit out of range; BKV_ECUDA on a CUDA error.
+ */
+int bkv_selftest_wait_timeout(bkv_ctx* ctx, int64_t limit_ns);
+
+/*
  * Per-kernel timing (tracing).  While enabled, every kernel launch made by
  * this context is bracketed by CUDA events on the context's stream.
  * bkv_profile_read synchronises the stream, then writes for each kernel k

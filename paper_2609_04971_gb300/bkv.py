@@ -67,6 +67,7 @@ def load_library(path: str | None = None, build: bool = True):
             "bkv_get_state": (ctypes.c_int, [_P, _P, _P, _P]),
             "bkv_set_state": (ctypes.c_int, [_P, _P, _P, _P]),
             "bkv_sync": (ctypes.c_int, [_P]),
+            "bkv_selftest_wait_timeout": (ctypes.c_int, [_P, ctypes.c_int64]),
             "bkv_compress_static": (ctypes.c_int, [ctypes.POINTER(BkvConfig), _P, _P, _P, _P, ctypes.c_int32,
                                                    ctypes.c_int32, ctypes.c_int64, _P, _P, _P, _P, _P, _P,
                                                    ctypes.c_char_p, ctypes.c_size_t]),
@@ -175,6 +176,16 @@ def bkv_set_state(ctx, centroids, sums, counts) -> None:
 
 def bkv_sync(ctx) -> None:
     _check(_l().bkv_sync(ctx), "bkv_sync", ctx)
+
+
+def bkv_selftest_wait_timeout(ctx, limit_ns: int) -> int:
+    """Runs one device wait that is meant to expire after limit_ns (see
+    include/bkv.h) and returns the status code bkv_sync reports for it
+    (BKV_ETIMEOUT when the expiry path works); raises on other errors."""
+    rc = _l().bkv_selftest_wait_timeout(ctx, int(limit_ns))
+    if rc not in (BKV_OK, BKV_ETIMEOUT):
+        _check(rc, "bkv_selftest_wait_timeout", ctx)
+    return rc
 
 
 def bkv_profile_enable(ctx, on: bool = True) -> None:

@@ -461,6 +461,16 @@ int bkv_profile_read(bkv_ctx* ctx, double* ms, int64_t* launches, int32_t n_kern
   return BKV_OK;
 }
 
+int bkv_selftest_wait_timeout(bkv_ctx* ctx, int64_t limit_ns) {
+  if (!ctx) return BKV_EINVAL;
+  if (limit_ns < 1000 || limit_ns > 10000000000LL) return fail(ctx, BKV_EINVAL, "limit_ns must be in 1e3..1e10");
+  int rc = bkv_sync(ctx);  // report earlier work first
+  if (rc != BKV_OK) return rc;
+  cudaError_t e = bkv::launch_selftest_wait(ctx->err, static_cast<unsigned long long>(limit_ns), ctx->stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "selftest launch");
+  return bkv_sync(ctx);
+}
+
 int bkv_sync(bkv_ctx* ctx) {
   if (!ctx) return BKV_EINVAL;
   cudaError_t e = cudaStreamSynchronize(ctx->stream);

@@ -18,6 +18,7 @@ enum DevErr : int {
   kDevTimeoutEpilogue = 3,
   kDevTimeoutDrain = 4,
   kDevTimeoutCluster = 5,
+  kDevTimeoutSelftest = 6,
 };
 
 // Every spin-wait gives up after this long and reports a timeout.
@@ -84,20 +85,25 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t pari
 }
 
 // Waits for the phase with the given parity to complete.  Gives up (returns
-// false) after kWaitLimitNs, or as soon as *abort is set by another warp; on
-// its own timeout it sets *abort and records `code` in the error word.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* err, int code) {
+// false) after limit_ns, or as soon as *abort is set by another warp; on its
+// own timeout it sets *abort and records `code` in the error word.
+__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, volatile int* abort, int* err, int code,
+                                              uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   while (true) {
     if (mbar_try_wait_sleep(bar, parity)) return true;
     if (*abort) return false;
-    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+    if (globaltimer_ns() - t0 > limit_ns) {
       *abort = 1;
       record_error(err, code);
       return false;
     }
   }
+}
+
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int* err, int code) {
+  return mbar_wait_for(bar, parity, abort, err, code, kWaitLimitNs);
 }
 
 // ------------------------------------------------------------------ clusters

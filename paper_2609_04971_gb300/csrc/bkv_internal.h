@@ -64,4 +64,7 @@ cudaError_t launch_select_gather(const Shape& s, const float* r, int L, int budg
 
 cudaError_t launch_keep_all(const Shape& s, int L, int budget, int* kept, cudaStream_t st);
 
+// ---- diagnostics (k_selftest.cu): a bounded wait that expires after limit_ns
+cudaError_t launch_selftest_wait(int* err, unsigned long long limit_ns, cudaStream_t st);
+
 }  // namespace bkv

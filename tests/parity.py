@@ -150,59 +150,17 @@ def check_instance(run: GpuRun, k: int, L: int | None = None, budget: int | None
             np.testing.assert_array_equal(run.counts0[e], st["counts"])
         # ---- update, from the GPU's seed state
         pre = dict(cent=run.cent0[e].copy(), sums=run.sums0[e].copy(), counts=run.counts0[e].copy())
-        st = {kk: v.copy() for kk, v in pre.items()}
-        a_o, margin = O.update(q_new, st, lib=lib)
-        a_g = run.assign[e]
-        diff = np.flatnonzero(a_o != a_g)
-        if diff.size:
-            bad = diff[margin[diff] >= ASSIGN_TIE]
-            assert bad.size == 0, f"instance {e}: {bad.size} assignments differ beyond ties, e.g. query " \
-                                  f"{bad[0]}: gpu {a_g[bad[0]]} oracle {a_o[bad[0]]} margin {margin[bad[0]]:.3e}"
-            rep.assign_ties += diff.size
-            st = {kk: v.copy() for kk, v in pre.items()}
-            O.update(q_new, st, override=a_g, lib=lib)
-        np.testing.assert_array_equal(run.counts1[e], st["counts"])
-        np.testing.assert_allclose(run.sums1[e], st["sums"], rtol=1e-12, atol=1e-12)
-        ref = st["cent"].astype(np.float64)
-        scale = np.maximum(np.linalg.norm(ref, axis=1, keepdims=True), 1.0)
-        cerr = float(np.max(np.abs(run.cent1[e].astype(np.float64) - ref) / scale)) if ref.size else 0.0
-        assert cerr <= CENT_TOL, f"instance {e}: centroid error {cerr:.3e}"
+        post = dict(cent=run.cent1[e], sums=run.sums1[e], counts=run.counts1[e])
+        ties, cerr = check_update(q_new, pre, run.assign[e], post, lib, tag=f"instance {e}")
+        rep.assign_ties += ties
         rep.max_cent_err = cerr
 
     # ---- compress, on the GPU's beacon state
-    K0 = run.K_before[k]
-    V0 = run.V_before[k]
-    kept_g = run.kept[e]
-    if L <= budget:
-        np.testing.assert_array_equal(kept_g[:L], np.arange(L))
-        assert np.all(kept_g[L:] == -1)
-        np.testing.assert_array_equal(run.K_after[k], K0)
-        return rep
-    qobs, valid = O.build_qobs(run.cent1[e], run.counts1[e], q_recent, np.asarray(inp["recent_pos"], np.int64),
-                               inp["t_pos"], wl.rope_theta, lib)
-    s_o = O.score(qobs, valid, K0[:L], lib)
-    if run.scores is not None:
-        s_g = run.scores[e][:L].astype(np.float64)
-        rel = np.abs(s_g - s_o) / np.maximum(s_o, 1e-300)
-        rep.max_score_rel = float(rel.max())
-        assert rep.max_score_rel <= SCORE_RTOL, \
-            f"instance {e}: score rel err {rep.max_score_rel:.3e} at key {int(rel.argmax())}"
-    kept_o, bd = O.select(s_o, budget, W, wl.n_prefix, lib)
-    assert kept_g.shape[0] == budget
-    assert np.all(np.diff(kept_g) > 0), f"instance {e}: kept indices not strictly ascending"
-    keep_set = set(range(wl.n_prefix)) | set(range(L - W, L))
-    assert keep_set <= set(kept_g.tolist()), f"instance {e}: keep set not retained"
-    assert kept_g.min() >= 0 and kept_g.max() < L
-    sym = set(kept_g.tolist()) ^ set(kept_o.tolist())
-    if sym:
-        b = bd[0]
-        for j in sym:
-            assert j not in keep_set
-            assert abs(s_o[j] - b) <= TIE_RTOL * b, \
-                f"instance {e}: key {j} kept by only one side with margin {abs(s_o[j] - b) / b:.3e} (> 1e-5)"
-        rep.boundary_swaps += len(sym) // 2
-    np.testing.assert_array_equal(run.K_after[k][:budget], K0[kept_g], err_msg=f"instance {e}: K compaction")
-    np.testing.assert_array_equal(run.V_after[k][:budget], V0[kept_g], err_msg=f"instance {e}: V compaction")
+    rel, swaps = check_compress(wl, run.cent1[e], run.counts1[e], q_recent, inp["recent_pos"], inp["t_pos"],
+                                run.K_before[k], run.V_before[k], run.K_after[k], run.V_after[k], run.kept[e],
+                                None if run.scores is None else run.scores[e], L, budget, lib, tag=f"instance {e}")
+    rep.max_score_rel = rel
+    rep.boundary_swaps += swaps
     return rep
 
 
@@ -212,3 +170,68 @@ def check_run(run: GpuRun, L=None, budget=None) -> Report:
     for k in range(len(run.sample)):
         rep.merge(check_instance(run, k, L=L, budget=budget, lib=lib))
     return rep
+
+
+def check_update(q_new: np.ndarray, pre: dict, assign_g: np.ndarray, post: dict, lib, tag: str = "") -> tuple:
+    """One beacon update of one instance from state `pre` (fp32 centroids, fp64 sums, int64 counts):
+    the GPU's assignments must equal the oracle's except at oracle ties (runner-up within 1e-12), and
+    the GPU's state `post` must equal the oracle's state after the GPU's own assignments.
+    Returns (ties, centroid error)."""
+    st = {kk: v.copy() for kk, v in pre.items()}
+    a_o, margin = O.update(q_new, st, lib=lib)
+    diff = np.flatnonzero(a_o != assign_g)
+    ties = 0
+    if diff.size:
+        bad = diff[margin[diff] >= ASSIGN_TIE]
+        assert bad.size == 0, f"{tag}: {bad.size} assignments differ beyond ties, e.g. query " \
+                              f"{bad[0]}: gpu {assign_g[bad[0]]} oracle {a_o[bad[0]]} margin {margin[bad[0]]:.3e}"
+        ties = diff.size
+        st = {kk: v.copy() for kk, v in pre.items()}
+        O.update(q_new, st, override=assign_g, lib=lib)
+    np.testing.assert_array_equal(post["counts"], st["counts"], err_msg=f"{tag}: counts")
+    np.testing.assert_allclose(post["sums"], st["sums"], rtol=1e-12, atol=1e-12, err_msg=f"{tag}: sums")
+    ref = st["cent"].astype(np.float64)
+    scale = np.maximum(np.linalg.norm(ref, axis=1, keepdims=True), 1.0)
+    cerr = float(np.max(np.abs(post["cent"].astype(np.float64) - ref) / scale)) if ref.size else 0.0
+    assert cerr <= CENT_TOL, f"{tag}: centroid error {cerr:.3e}"
+    return ties, cerr
+
+
+def check_compress(wl: Workload, cent: np.ndarray, counts: np.ndarray, q_recent: np.ndarray, recent_pos, t_pos: int,
+                   K0: np.ndarray, V0: np.ndarray, K1: np.ndarray, V1: np.ndarray, kept_g: np.ndarray,
+                   scores_g: np.ndarray | None, L: int, budget: int, lib, tag: str = "") -> tuple:
+    """One compress of one instance on the beacon state (cent, counts): scores within 1e-3, the kept set
+    equal up to boundary ties, K / V rows byte-equal to the kept pre-compress rows.  K0 / V0 and K1 / V1
+    are the instance's uint16 rows before and after.  Returns (max score rel err, boundary swaps)."""
+    W = wl.window
+    if L <= budget:
+        np.testing.assert_array_equal(kept_g[:L], np.arange(L))
+        assert np.all(kept_g[L:] == -1)
+        np.testing.assert_array_equal(K1, K0)
+        return 0.0, 0
+    qobs, valid = O.build_qobs(cent, counts, q_recent, np.asarray(recent_pos, np.int64), t_pos, wl.rope_theta, lib)
+    s_o = O.score(qobs, valid, K0[:L], lib)
+    rel_max = 0.0
+    if scores_g is not None:
+        s_g = scores_g[:L].astype(np.float64)
+        rel = np.abs(s_g - s_o) / np.maximum(s_o, 1e-300)
+        rel_max = float(rel.max())
+        assert rel_max <= SCORE_RTOL, f"{tag}: score rel err {rel_max:.3e} at key {int(rel.argmax())}"
+    kept_o, bd = O.select(s_o, budget, W, wl.n_prefix, lib)
+    assert kept_g.shape[0] == budget
+    assert np.all(np.diff(kept_g) > 0), f"{tag}: kept indices not strictly ascending"
+    keep_set = set(range(wl.n_prefix)) | set(range(L - W, L))
+    assert keep_set <= set(kept_g.tolist()), f"{tag}: keep set not retained"
+    assert kept_g.min() >= 0 and kept_g.max() < L
+    sym = set(kept_g.tolist()) ^ set(kept_o.tolist())
+    swaps = 0
+    if sym:
+        b = bd[0]
+        for j in sym:
+            assert j not in keep_set
+            assert abs(s_o[j] - b) <= TIE_RTOL * b, \
+                f"{tag}: key {j} kept by only one side with margin {abs(s_o[j] - b) / b:.3e} (> 1e-5)"
+        swaps = len(sym) // 2
+    np.testing.assert_array_equal(K1[:budget], K0[kept_g], err_msg=f"{tag}: K compaction")
+    np.testing.assert_array_equal(V1[:budget], V0[kept_g], err_msg=f"{tag}: V compaction")
+    return rel_max, swaps

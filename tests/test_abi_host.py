@@ -85,3 +85,7 @@ def test_byte_accounting_matches_closed_form():
     assert wl.n_obs == 40 and n_obs_padded(wl.n_obs) == 48
     assert LLAMA_8B.n_obs == 48 and QWEN3_14B.n_obs == 56 and TINY.n_obs == 20
     assert n_obs_padded(QWEN3_14B.n_obs) == 64 and n_obs_padded(TINY.n_obs) == 32
+
+
+def test_selftest_rejects_null_context(lib):
+    assert lib.bkv_selftest_wait_timeout(None, 1_000_000) == bkv.BKV_EINVAL
