@@ -114,8 +114,13 @@ int bkv_init_beacons(bkv_ctx* ctx, const void* q_init, int32_t n_init);
  * is assigned to argmax_b cos(q, c_b) over the beacons with count > 0 and a
  * non-zero centroid, using the centroids as they were when the call started
  * (ties go to the lowest b; a zero query is skipped).  Then for each beacon
- * sums_b += sum of its assigned queries (exact), counts_b += their number and
- * c_b = fp32(sums_b / counts_b).
+ * sums_b += sum of its assigned queries, counts_b += their number and
+ * c_b = fp32(sums_b / counts_b).  Query elements must be finite with
+ * |x| < 2^14, and one call's sum for a beacon must stay below 2^23 in every
+ * element (int64 fixed point with 40 fractional bits); that sum is then
+ * exact, except that elements below 2^-31 in magnitude are rounded to
+ * multiples of 2^-38.  Assignments equal the exact cosine argmax except at
+ * ties below about 1e-12 relative.
  *   q_new       bf16 [n_layers][batch][n_q_heads][n_new][head_dim], pre-RoPE.
  *   assign_out  int32 [n_layers][batch][n_q_heads][n_new] or NULL: the beacon
  *               chosen for each query, -1 when it was skipped.
