@@ -60,8 +60,16 @@ extern "C" {
 #define BKV_ETIMEOUT (-4) /* a bounded device-side wait expired (kernel aborted) */
 #define BKV_ESTATE (-5)   /* call order violated (e.g. update before init)       */
 
-/* bkv_config.flags: no option is defined yet; pass 0. */
+/* bkv_config.flags (bitwise OR). */
 #define BKV_F_NONE 0u
+/*
+ * Mean aggregation (the mean form of Eq. 6, the paper's ablation of its max
+ * pooling, Section 4.3): Score[j] = the mean of the softmax weights of key j
+ * over the group's valid observation queries instead of their maximum (0
+ * when no query is valid).  Selection, the keep set and compaction are
+ * unchanged.
+ */
+#define BKV_F_MEAN_AGG 1u
 
 typedef struct bkv_ctx bkv_ctx;
 
@@ -81,7 +89,7 @@ typedef struct {
   int32_t n_beacons, window, n_prefix;
   int32_t capacity;
   double rope_theta;
-  uint32_t flags; /* reserved, must be 0 */
+  uint32_t flags; /* BKV_F_* options; unknown bits are rejected */
 } bkv_config;
 
 /*
@@ -135,7 +143,8 @@ int bkv_update_beacons(bkv_ctx* ctx, const void* q_new, int32_t n_new, int32_t* 
  * its G query heads, query (h, w) rotated to position recent_pos[w], and its
  * beacons with count > 0 rotated to t_pos; each is rounded to bf16 after the
  * rotation.  Score[j] = max over those queries of the softmax weight of key
- * j over all L cached keys (Eq. 4, Eq. 6 max form; logits q.k / sqrt(d)).
+ * j over all L cached keys (Eq. 4, Eq. 6 max form; logits q.k / sqrt(d)), or
+ * their mean under BKV_F_MEAN_AGG.
  * Kept rows = [0, n_prefix) U [L - window, L) U the (budget - n_prefix -
  * window) other rows with the largest Score (ties to the lower index), in
  * ascending order (Eq. 7, Algorithm 2).  Row i of K and V then holds what row

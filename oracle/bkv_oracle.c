@@ -333,26 +333,29 @@ int bkvo_build_qobs(const float* cent, const int64_t* counts, int nb, const uint
 }
 
 /* ------------------------------------------------------------------ */
-/* Scoring (Eq. 4; Eq. 6 max form; group max of Section 4.3, App. D.2) */
+/* Scoring (Eq. 4; Eq. 6 max or mean form; group of Section 4.3)     */
 /* ------------------------------------------------------------------ */
 
 /*
  * For every valid observation query q and cached key j:
  *   logit_qj = (q . k_j) / sqrt(d)
  *   w_qj     = exp(logit_qj) / sum_l exp(logit_ql)      (softmax over all L keys)
- * Score[j]   = max over valid q of w_qj.
+ * Score[j]   = max over valid q of w_qj            (mean == 0, Eq. 6 max form)
+ *            = (1 / #valid) * sum over valid q of w_qj   (mean != 0, Eq. 6 mean form)
  * The normaliser is evaluated as lse_q = m_q + log(sum_l exp(logit_ql - m_q)),
  * m_q = max_l logit_ql, so that exp does not overflow.
  * Score[j] = 0 for every j when no query is valid.
  */
-void bkvo_score(const double* qobs, const int32_t* valid, int M, const uint16_t* K, int L, int d,
-                double* score) {
+void bkvo_score_agg(const double* qobs, const int32_t* valid, int M, const uint16_t* K, int L, int d, int mean,
+                    double* score) {
   double* k = widen_rows(K, L, d);
   double* lg = (double*)malloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
   double inv_sqrt_d = 1.0 / sqrt((double)d);
+  int n_valid = 0;
   for (int j = 0; j < L; ++j) score[j] = 0.0;
   for (int q = 0; q < M; ++q) {
     if (!valid[q]) continue;
+    ++n_valid;
     double m = -INFINITY;
     for (int j = 0; j < L; ++j) {
       lg[j] = dot_seq(qobs + (size_t)q * d, k + (size_t)j * d, d) * inv_sqrt_d;
@@ -363,11 +366,21 @@ void bkvo_score(const double* qobs, const int32_t* valid, int M, const uint16_t*
     double lse = m + log(s);
     for (int j = 0; j < L; ++j) {
       double w = exp(lg[j] - lse);
-      if (w > score[j]) score[j] = w;
+      if (mean)
+        score[j] = score[j] + w;
+      else if (w > score[j])
+        score[j] = w;
     }
   }
+  if (mean && n_valid > 0)
+    for (int j = 0; j < L; ++j) score[j] = score[j] / (double)n_valid;
   free(lg);
   free(k);
+}
+
+void bkvo_score(const double* qobs, const int32_t* valid, int M, const uint16_t* K, int L, int d,
+                double* score) {
+  bkvo_score_agg(qobs, valid, M, K, L, d, 0, score);
 }
 
 /* ------------------------------------------------------------------ */

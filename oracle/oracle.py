@@ -52,6 +52,7 @@ _SIGS = {
     "bkvo_rope": (None, [_P, _I, _I64, _D, _P]),
     "bkvo_build_qobs": (_I, [_P, _P, _I, _P, _I, _I, _P, _I64, _I, _D, _P, _P]),
     "bkvo_score": (None, [_P, _P, _I, _P, _I, _I, _P]),
+    "bkvo_score_agg": (None, [_P, _P, _I, _P, _I, _I, _I, _P]),
     "bkvo_select": (_I, [_P, _I, _I, _I, _I, _P, _P]),
     "bkvo_gather": (None, [_P, _P, _P, _I, _I]),
     "bkvo_step_many": (_I, [_P, _I, _I, _I, _I, _I, _I, _I, _P, _I, _P, _P, _I64, _D, _I, _I,
@@ -184,14 +185,15 @@ def build_qobs(cent, counts, q_recent_bits, recent_pos, t_pos: int, theta: float
     return qobs[:m].copy(), valid[:m].copy()
 
 
-def score(qobs: np.ndarray, valid: np.ndarray, k_bits: np.ndarray, lib=None) -> np.ndarray:
-    """Eq. 4 softmax weights, max over the group's valid queries (Eq. 6, Section 4.3)."""
+def score(qobs: np.ndarray, valid: np.ndarray, k_bits: np.ndarray, lib=None, mean: bool = False) -> np.ndarray:
+    """Eq. 4 softmax weights, max (or, with mean=True, mean) over the group's valid queries
+    (Eq. 6, Section 4.3)."""
     qo = _c(qobs, np.float64)
     va = _c(valid, np.int32)
     k = _c(k_bits, np.uint16)
     L, d = k.shape
     out = np.zeros(max(L, 1), np.float64)
-    (lib or load()).bkvo_score(_p(qo), _p(va), qo.shape[0], _p(k), L, d, _p(out))
+    (lib or load()).bkvo_score_agg(_p(qo), _p(va), qo.shape[0], _p(k), L, d, int(bool(mean)), _p(out))
     return out[:L].copy()
 
 

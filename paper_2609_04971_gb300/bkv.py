@@ -26,6 +26,11 @@ BKV_ESTATE = -5
 KERNEL_NAMES = ("fps_init", "update", "qobs", "score", "select_gather", "keep_all")
 
 
+# bkv_config.flags options (include/bkv.h)
+BKV_F_NONE = 0
+BKV_F_MEAN_AGG = 1
+
+
 class BkvConfig(ctypes.Structure):
     _fields_ = [
         ("n_layers", ctypes.c_int32), ("batch", ctypes.c_int32), ("n_q_heads", ctypes.c_int32),
@@ -233,17 +238,19 @@ class BeaconKV:
     """
 
     def __init__(self, *, n_layers, batch, n_q_heads, n_kv_heads, head_dim, n_beacons, window, capacity,
-                 rope_theta=0.0, n_prefix=0, stream=None):
+                 rope_theta=0.0, n_prefix=0, stream=None, mean_agg=False):
+        flags = BKV_F_MEAN_AGG if mean_agg else BKV_F_NONE
         self.cfg = BkvConfig(n_layers, batch, n_q_heads, n_kv_heads, head_dim, n_beacons, window, n_prefix,
-                             capacity, float(rope_theta), 0)
+                             capacity, float(rope_theta), flags)
         self.ctx = bkv_create(self.cfg, stream)
         self.n_inst = n_layers * batch * n_kv_heads
 
     @classmethod
-    def for_workload(cls, wl, stream=None, capacity=None) -> "BeaconKV":
+    def for_workload(cls, wl, stream=None, capacity=None, mean_agg=False) -> "BeaconKV":
         return cls(n_layers=wl.n_layers, batch=wl.batch, n_q_heads=wl.n_q_heads, n_kv_heads=wl.n_kv_heads,
                    head_dim=wl.head_dim, n_beacons=wl.n_beacons, window=wl.window,
-                   capacity=capacity or wl.capacity, rope_theta=wl.rope_theta, n_prefix=wl.n_prefix, stream=stream)
+                   capacity=capacity or wl.capacity, rope_theta=wl.rope_theta, n_prefix=wl.n_prefix, stream=stream,
+                   mean_agg=mean_agg)
 
     def close(self):
         if self.ctx:

@@ -49,7 +49,8 @@ struct ScoreArgs {
   int L;
   float scale_log2;        // log2(e) / sqrt(d)
   const uint32_t* valid;   // [n_inst][4] bitmask of valid scoring rows
-  float* r_out;            // [n_inst][cap] log2-domain scores (max_q logit - lse)
+  bool mean;               // mean over the valid queries instead of the maximum
+  float* r_out;            // [n_inst][cap] log2-domain scores (log2 of the aggregated weight)
   float* scores_out;       // [n_inst][cap] probabilities, or nullptr
   int* err;                // device error word
 };
@@ -58,6 +59,9 @@ struct ScoreArgs {
 // of n_obs_pad rows.
 cudaError_t launch_score(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32, const CUtensorMap& qmap,
                          const ScoreArgs& a, cudaStream_t st);
+// The mean form (a.mean), compiled in its own translation unit; launch_score forwards to it.
+cudaError_t launch_score_mean(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32,
+                              const CUtensorMap& qmap, const ScoreArgs& a, cudaStream_t st);
 
 cudaError_t launch_select_gather(const Shape& s, const float* r, int L, int budget, __nv_bfloat16* K,
                                  __nv_bfloat16* V, int* kept, cudaStream_t st);

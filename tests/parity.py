@@ -50,6 +50,7 @@ class GpuRun:
     K_after: np.ndarray
     V_after: np.ndarray
     sample: np.ndarray     # instance ids copied to the host
+    mean_agg: bool = False  # Eq. 6 mean form instead of the max
 
 
 def _inst_rows(t: torch.Tensor, wl: Workload) -> torch.Tensor:
@@ -59,7 +60,7 @@ def _inst_rows(t: torch.Tensor, wl: Workload) -> torch.Tensor:
 
 
 def run_gpu(wl: Workload, seed: int = 0, sample=None, with_scores: bool = True, inputs: dict | None = None,
-            L: int | None = None, budget: int | None = None) -> GpuRun:
+            L: int | None = None, budget: int | None = None, mean_agg: bool = False) -> GpuRun:
     dev = torch.device("cuda")
     inp = inputs or synth.step_inputs(wl, seed, dev)
     L = wl.L if L is None else L
@@ -68,7 +69,7 @@ def run_gpu(wl: Workload, seed: int = 0, sample=None, with_scores: bool = True, 
     sample = np.arange(n_inst) if sample is None else np.asarray(sample)
     sidx = torch.as_tensor(sample, device=dev)
 
-    bk = BeaconKV.for_workload(wl)
+    bk = BeaconKV.for_workload(wl, mean_agg=mean_agg)
     try:
         bk.init_beacons(inp["q_init"])
         c0, s0, n0 = [x.cpu().numpy() for x in bk.state()]
@@ -93,7 +94,8 @@ def run_gpu(wl: Workload, seed: int = 0, sample=None, with_scores: bool = True, 
                   assign=assign.view(n_inst, -1).cpu().numpy(), cent1=c1, sums1=s1, counts1=n1,
                   kept=kept.view(n_inst, -1).cpu().numpy(),
                   scores=None if scores is None else scores.view(n_inst, -1).cpu().numpy(),
-                  K_before=K_before, V_before=V_before, K_after=K_after, V_after=V_after, sample=sample)
+                  K_before=K_before, V_before=V_before, K_after=K_after, V_after=V_after, sample=sample,
+                  mean_agg=mean_agg)
 
 
 @dataclasses.dataclass
@@ -158,7 +160,8 @@ def check_instance(run: GpuRun, k: int, L: int | None = None, budget: int | None
     # ---- compress, on the GPU's beacon state
     rel, swaps = check_compress(wl, run.cent1[e], run.counts1[e], q_recent, inp["recent_pos"], inp["t_pos"],
                                 run.K_before[k], run.V_before[k], run.K_after[k], run.V_after[k], run.kept[e],
-                                None if run.scores is None else run.scores[e], L, budget, lib, tag=f"instance {e}")
+                                None if run.scores is None else run.scores[e], L, budget, lib, tag=f"instance {e}",
+                                mean=run.mean_agg)
     rep.max_score_rel = rel
     rep.boundary_swaps += swaps
     return rep
@@ -199,7 +202,7 @@ def check_update(q_new: np.ndarray, pre: dict, assign_g: np.ndarray, post: dict,
 
 def check_compress(wl: Workload, cent: np.ndarray, counts: np.ndarray, q_recent: np.ndarray, recent_pos, t_pos: int,
                    K0: np.ndarray, V0: np.ndarray, K1: np.ndarray, V1: np.ndarray, kept_g: np.ndarray,
-                   scores_g: np.ndarray | None, L: int, budget: int, lib, tag: str = "") -> tuple:
+                   scores_g: np.ndarray | None, L: int, budget: int, lib, tag: str = "", mean: bool = False) -> tuple:
     """One compress of one instance on the beacon state (cent, counts): scores within 1e-3, the kept set
     equal up to boundary ties, K / V rows byte-equal to the kept pre-compress rows.  K0 / V0 and K1 / V1
     are the instance's uint16 rows before and after.  Returns (max score rel err, boundary swaps)."""
@@ -210,7 +213,7 @@ def check_compress(wl: Workload, cent: np.ndarray, counts: np.ndarray, q_recent:
         np.testing.assert_array_equal(K1, K0)
         return 0.0, 0
     qobs, valid = O.build_qobs(cent, counts, q_recent, np.asarray(recent_pos, np.int64), t_pos, wl.rope_theta, lib)
-    s_o = O.score(qobs, valid, K0[:L], lib)
+    s_o = O.score(qobs, valid, K0[:L], lib, mean=mean)
     rel_max = 0.0
     if scores_g is not None:
         s_g = scores_g[:L].astype(np.float64)

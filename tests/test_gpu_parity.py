@@ -126,3 +126,15 @@ def test_deterministic_across_runs():
     np.testing.assert_array_equal(a.scores, b.scores)
     np.testing.assert_array_equal(a.cent1, b.cent1)
     np.testing.assert_array_equal(a.K_after, b.K_after)
+
+
+# ---------------------------------------------------------------- Eq. 6 mean form (BKV_F_MEAN_AGG)
+@pytest.mark.parametrize("wl,seed", [
+    (TINY.scaled(name="mean_tiny"), 11),
+    (QWEN3_4B.scaled(name="mean_qwen3_4b_1L_b2", n_layers=1, batch=2), 12),
+    (QWEN3_4B.scaled(name="mean_ragged_L300_B17", n_layers=1, batch=1, L=300, budget=17), 13),
+    (QWEN3_4B.scaled(name="mean_long_L20000", n_layers=1, batch=1, L=20000, budget=9000), 14),
+    (LLAMA_8B.scaled(name="mean_w0", n_layers=1, batch=1, L=400, budget=200, window=0), 15),
+], ids=lambda x: getattr(x, "name", str(x)))
+def test_mean_aggregation(wl, seed):
+    _run(wl, seed=seed, mean_agg=True)

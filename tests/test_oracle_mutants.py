@@ -23,6 +23,8 @@ SRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), 
 _SCORE = [(TS.test_score_matches_scipy_softmax_max, dict(M=3, L=50, d=8)),
           (TS.test_score_two_key_logistic_closed_form, {}), (TS.test_golden_worked_case, {}),
           (TS.test_score_single_query_sums_to_one_and_ranks_by_dot, {})]
+_MEAN = [(TS.test_score_mean_matches_scipy_softmax_mean, dict(M=4, L=77, d=8)),
+         (TS.test_score_mean_closed_forms_and_bounds, {}), (TS.test_score_mean_duplicated_query_weights, {})]
 _ROPE = [(TN.test_rope_is_complex_rotation_of_rotate_half_pairs, {}),
          (TN.test_rope_preserves_norm_and_relative_position, {})]
 _FPS = [(TB.test_fps_matches_maxmin_brute_force, dict(seed=s)) for s in range(6)] + [
@@ -35,7 +37,10 @@ _SEL = [(TS.test_select_matches_lexsort_and_invariants, dict(L=130, budget=100, 
 MUTANTS = [
     ("drop_inv_sqrt_d", "* inv_sqrt_d;", "* 1.0;", _SCORE),
     ("no_max_shift_in_lse", "double lse = m + log(s);", "double lse = log(s);", _SCORE),
-    ("mean_instead_of_max", "if (w > score[j]) score[j] = w;", "score[j] = score[j] + w / M;", _SCORE),
+    ("sum_instead_of_max", "else if (w > score[j])\n        score[j] = w;", "else\n        score[j] = score[j] + w;", _SCORE),
+    ("mean_over_all_rows", "score[j] = score[j] / (double)n_valid;", "score[j] = score[j] / (double)M;", _MEAN),
+    ("mean_takes_max", "      if (mean)\n        score[j] = score[j] + w;", "      if (mean && w > score[j])\n        score[j] = w;",
+     _MEAN),
     ("rope_sign", "y[i] = x1 * cs - x2 * sn;", "y[i] = x1 * cs + x2 * sn;", _ROPE),
     ("rope_interleaved_pairs", "double x1 = x[i], x2 = x[i + h];", "double x1 = x[2 * i], x2 = x[2 * i + 1];",
      _ROPE),

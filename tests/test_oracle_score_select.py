@@ -1,4 +1,4 @@
-"""Pins of the oracle's scoring (Eq. 4, Eq. 6 max, group max), selection (Eq. 7 and
+"""Pins of the oracle's scoring (Eq. 4, Eq. 6 max and mean forms, group aggregation), selection (Eq. 7 and
 the keep set of Algorithm 2) and compaction (Eq. 8).
 
 Independent routes: scipy.special.softmax, numpy lexsort, numpy fancy indexing,
@@ -102,6 +102,48 @@ def test_score_permutation_of_queries(olib):
     a = O.score(q, np.ones(7, np.int32), k, olib)
     b = O.score(q[perm], np.ones(7, np.int32), k, olib)
     np.testing.assert_array_equal(a, b)
+
+
+# ------------------------------------------------------------------ score, mean form of Eq. 6
+@pytest.mark.parametrize("M,L,d", [(1, 9, 4), (4, 77, 8), (7, 260, 32)])
+def test_score_mean_matches_scipy_softmax_mean(olib, M, L, d):
+    rng = np.random.default_rng(7 * M + L)
+    q, k = _rand_case(rng, M, L, d)
+    valid = np.ones(M, np.int32)
+    valid[M // 2] = 0 if M > 1 else 1
+    got = O.score(q, valid, k, olib, mean=True)
+    w = softmax(q @ O.bf16_to_f64(k).T / math.sqrt(d), axis=1)
+    want = w[valid.astype(bool)].mean(axis=0)
+    np.testing.assert_allclose(got, want, rtol=1e-12, atol=0)
+
+
+def test_score_mean_closed_forms_and_bounds(olib):
+    rng = np.random.default_rng(35)
+    q, k = _rand_case(rng, 5, 140, 16)
+    one = np.array([0, 0, 1, 0, 0], np.int32)
+    # one valid query: mean == max == that query's softmax row, which sums to one
+    m1 = O.score(q, one, k, olib, mean=True)
+    np.testing.assert_array_equal(m1, O.score(q, one, k, olib))
+    assert m1.sum() == pytest.approx(1.0, rel=1e-12)
+    # every query's row sums to one, so the mean does too; and the mean never exceeds the max
+    allv = np.ones(5, np.int32)
+    mean = O.score(q, allv, k, olib, mean=True)
+    assert mean.sum() == pytest.approx(1.0, rel=1e-12)
+    assert np.all(mean <= O.score(q, allv, k, olib) * (1 + 1e-15))
+    # identical keys: every weight is 1 / L
+    kk = np.tile(k[:1], (33, 1))
+    np.testing.assert_allclose(O.score(q, allv, kk, olib, mean=True), 1.0 / 33, rtol=1e-13)
+    # no valid query: all zero
+    np.testing.assert_array_equal(O.score(q, np.zeros(5, np.int32), k, olib, mean=True), 0.0)
+
+
+def test_score_mean_duplicated_query_weights(olib):
+    """Duplicating a query counts it twice in the mean (unlike the max)."""
+    rng = np.random.default_rng(36)
+    q, k = _rand_case(rng, 2, 60, 8)
+    w = softmax(q @ O.bf16_to_f64(k).T / math.sqrt(8), axis=1)
+    got = O.score(np.vstack([q, q[:1]]), np.ones(3, np.int32), k, olib, mean=True)
+    np.testing.assert_allclose(got, (2 * w[0] + w[1]) / 3, rtol=1e-12)
 
 
 # ------------------------------------------------------------------ select
