@@ -21,7 +21,9 @@
  *
  * Readings of points the paper leaves open (each is listed in the design doc):
  *   - beacons are kept per KV head and fed by all G query heads of its group;
- *     they are maintained as running-mean centroids seeded by FPS;
+ *     they are maintained as running-mean centroids seeded by FPS; in the
+ *     Continual FPS mode they are instead each query head's fill-and-compress
+ *     buffer (Eq. 9), whose FPS decisions are taken in fp32 as in the kernels;
  *   - cosine with a zero vector is 0 (FPS) / the query is skipped (assignment);
  *   - argmin / argmax ties go to the lowest index;
  *   - RoPE uses the rotate-half pairing (i, i + d/2) with
@@ -178,6 +180,134 @@ int bkvo_fps(const uint16_t* q, int N, int d, int m, int32_t* picks, double* gap
   free(S);
   free(x);
   return m;
+}
+
+/* ------------------------------------------------------------------ */
+/* Continual FPS (Section 4.2, Eq. 9; Algorithm 2 decode branch)       */
+/* ------------------------------------------------------------------ */
+
+/*
+ * Algorithm 1 with every similarity taken in fp32, the precision of the
+ * buffer kernels (the argmins are integer decisions; both sides take them in
+ * the same precision, and the pins compare them with the fp64 bkvo_fps):
+ *   dot32(a, b) = fmaf(a_{d-1}, b_{d-1}, ... fmaf(a_0, b_0, 0.f))    (i increasing)
+ *   n_a         = sqrtf(dot32(a, a))
+ *   cos32(a, b) = dot32(a, b) / (n_a * n_b), or 0 when a norm is 0
+ *   avg_i       = (sum over j = 0 .. N-1 of cos32(q_i, q_j), fp32, j increasing) / N
+ * then the same first pick, S_j and farthest-point loop as bkvo_fps, ties to
+ * the lowest index.  gap[k] is the runner-up distance of the k-th argmin.
+ */
+static float dot32(const float* a, const float* b, int d) {
+  float s = 0.f;
+  for (int i = 0; i < d; ++i) s = fmaf(a[i], b[i], s);
+  return s;
+}
+
+int bkvo_fps32(const uint16_t* q, int N, int d, int m, int32_t* picks, double* gap) {
+  if (m > N) m = N;
+  if (m <= 0) return 0;
+  float* x = (float*)malloc(sizeof(float) * (size_t)N * (size_t)d);
+  for (size_t i = 0; i < (size_t)N * (size_t)d; ++i) x[i] = (float)bkvo_bf16_to_f64(q[i]);
+  float* nrm = (float*)malloc(sizeof(float) * (size_t)N);
+  float* cs = (float*)malloc(sizeof(float) * (size_t)N * (size_t)N);
+  float* S = (float*)malloc(sizeof(float) * (size_t)N);
+  char* sel = (char*)calloc((size_t)N, 1);
+  for (int i = 0; i < N; ++i) nrm[i] = sqrtf(dot32(x + (size_t)i * d, x + (size_t)i * d, d));
+  for (int i = 0; i < N; ++i)
+    for (int j = 0; j < N; ++j) {
+      const float den = nrm[i] * nrm[j];
+      cs[(size_t)i * N + j] = (nrm[i] == 0.f || nrm[j] == 0.f)
+                                  ? 0.f
+                                  : dot32(x + (size_t)i * d, x + (size_t)j * d, d) / den;
+    }
+  int p = -1;
+  float best = INFINITY, second = INFINITY;
+  for (int i = 0; i < N; ++i) {
+    float sum = 0.f;
+    for (int j = 0; j < N; ++j) sum = sum + cs[(size_t)i * N + j];
+    const float avg = sum / (float)N;
+    if (avg < best) {
+      second = best;
+      best = avg;
+      p = i;
+    } else if (avg < second) {
+      second = avg;
+    }
+  }
+  if (p < 0) p = 0; /* only reachable with non-finite inputs */
+  picks[0] = p;
+  gap[0] = (double)second - (double)best;
+  sel[p] = 1;
+  for (int j = 0; j < N; ++j) S[j] = cs[(size_t)j * N + p];
+  for (int k = 1; k < m; ++k) {
+    int r = -1;
+    float b1 = INFINITY, b2 = INFINITY;
+    for (int j = 0; j < N; ++j) {
+      if (sel[j]) continue;
+      if (S[j] < b1) {
+        b2 = b1;
+        b1 = S[j];
+        r = j;
+      } else if (S[j] < b2) {
+        b2 = S[j];
+      }
+    }
+    if (r < 0) { /* only reachable with non-finite inputs */
+      m = k;
+      break;
+    }
+    picks[k] = r;
+    gap[k] = (double)b2 - (double)b1;
+    sel[r] = 1;
+    for (int j = 0; j < N; ++j) {
+      if (sel[j]) continue;
+      const float c = cs[(size_t)j * N + r];
+      if (c > S[j]) S[j] = c;
+    }
+  }
+  free(sel);
+  free(S);
+  free(cs);
+  free(nrm);
+  free(x);
+  return m;
+}
+
+/*
+ * The fill-and-compress buffer of one query head (Eq. 9): every new query is
+ * appended in order; when the buffer holds b_max queries it is replaced by
+ * its FPS selection of b_min queries, in pick order.
+ *   buf     bf16 [b_max][d], rows [0, *size) in use; updated in place.
+ *   q_new   bf16 [n_new][d].
+ *   events  if not NULL, receives for each compression its b_min picks
+ *           (indices into the full buffer) and gaps, events_cap compressions at most.
+ * Returns the number of compressions.
+ */
+int bkvo_cfps_update(uint16_t* buf, int32_t* size, int b_min, int b_max, const uint16_t* q_new, int n_new, int d,
+                     int32_t* ev_picks, double* ev_gaps, int events_cap) {
+  int n_ev = 0;
+  int32_t* picks = (int32_t*)malloc(sizeof(int32_t) * (size_t)(b_min > 0 ? b_min : 1));
+  double* gaps = (double*)malloc(sizeof(double) * (size_t)(b_min > 0 ? b_min : 1));
+  uint16_t* tmp = (uint16_t*)malloc(sizeof(uint16_t) * (size_t)b_max * (size_t)d);
+  for (int n = 0; n < n_new; ++n) {
+    memcpy(buf + (size_t)(*size) * d, q_new + (size_t)n * d, sizeof(uint16_t) * (size_t)d);
+    *size += 1;
+    if (*size >= b_max) {
+      int got = bkvo_fps32(buf, *size, d, b_min, picks, gaps);
+      for (int k = 0; k < got; ++k) memcpy(tmp + (size_t)k * d, buf + (size_t)picks[k] * d, sizeof(uint16_t) * (size_t)d);
+      memcpy(buf, tmp, sizeof(uint16_t) * (size_t)got * (size_t)d);
+      if (ev_picks && n_ev < events_cap) {
+        memcpy(ev_picks + (size_t)n_ev * b_min, picks, sizeof(int32_t) * (size_t)got);
+        memcpy(ev_gaps + (size_t)n_ev * b_min, gaps, sizeof(double) * (size_t)got);
+      }
+      ++n_ev;
+      *size = got;
+    }
+  }
+  free(tmp);
+  free(gaps);
+  free(picks);
+  return n_ev;
 }
 
 /* ------------------------------------------------------------------ */

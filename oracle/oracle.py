@@ -53,6 +53,8 @@ _SIGS = {
     "bkvo_build_qobs": (_I, [_P, _P, _I, _P, _I, _I, _P, _I64, _I, _D, _P, _P]),
     "bkvo_score": (None, [_P, _P, _I, _P, _I, _I, _P]),
     "bkvo_score_agg": (None, [_P, _P, _I, _P, _I, _I, _I, _P]),
+    "bkvo_fps32": (_I, [_P, _I, _I, _I, _P, _P]),
+    "bkvo_cfps_update": (_I, [_P, _P, _I, _I, _P, _I, _I, _P, _P, _I]),
     "bkvo_select": (_I, [_P, _I, _I, _I, _I, _P, _P]),
     "bkvo_gather": (None, [_P, _P, _P, _I, _I]),
     "bkvo_step_many": (_I, [_P, _I, _I, _I, _I, _I, _I, _I, _P, _I, _P, _P, _I64, _D, _I, _I,
@@ -119,6 +121,35 @@ def fps(q_bits: np.ndarray, m: int, lib=None):
     gaps = np.zeros(max(m, 1), np.float64)
     got = (lib or load()).bkvo_fps(_p(q), n, d, m, _p(picks), _p(gaps))
     return picks[:got].copy(), gaps[:got].copy()
+
+
+def fps32(q_bits: np.ndarray, m: int, lib=None):
+    """Algorithm 1 with the similarities in fp32 (sequential fused dot products), the
+    precision of the Continual FPS kernels.  Returns (picks, gaps)."""
+    q = _c(q_bits, np.uint16)
+    n, d = q.shape
+    picks = np.full(max(m, 1), -1, np.int32)
+    gaps = np.zeros(max(m, 1), np.float64)
+    got = (lib or load()).bkvo_fps32(_p(q), n, d, m, _p(picks), _p(gaps))
+    return picks[:got].copy(), gaps[:got].copy()
+
+
+def cfps_update(buf_bits: np.ndarray, size: int, b_min: int, b_max: int, q_new_bits: np.ndarray, lib=None):
+    """Continual FPS (Eq. 9) of one query head: append each new query; at b_max queries
+    compress the buffer to its FPS selection of b_min.  buf_bits: uint16 [>= size, d].
+    Returns (buffer uint16 [b_max, d] with rows [0, size) in use, size, picks [events, b_min],
+    gaps [events, b_min])."""
+    d = q_new_bits.shape[-1]
+    buf = np.zeros((b_max, d), np.uint16)
+    buf[:size] = buf_bits[:size]
+    q = _c(q_new_bits.reshape(-1, d), np.uint16)
+    n_new = q.shape[0]
+    cap = n_new // max(b_max - b_min, 1) + 2
+    ev_p = np.full((cap, max(b_min, 1)), -1, np.int32)
+    ev_g = np.zeros((cap, max(b_min, 1)), np.float64)
+    sz = np.array([size], np.int32)
+    n_ev = (lib or load()).bkvo_cfps_update(_p(buf), _p(sz), b_min, b_max, _p(q), n_new, d, _p(ev_p), _p(ev_g), cap)
+    return buf, int(sz[0]), ev_p[:n_ev].copy(), ev_g[:n_ev].copy()
 
 
 def init_beacons(q_bits: np.ndarray, nb: int, lib=None):
