@@ -70,6 +70,29 @@ extern "C" {
  * unchanged.
  */
 #define BKV_F_MEAN_AGG 1u
+/*
+ * Continual FPS beacons (Section 4.2, Eq. 9; Algorithm 2), the paper's own
+ * beacon maintenance, instead of running-mean centroids.  n_beacons is then
+ * B_Q^min per QUERY head and every query head keeps a buffer of at most
+ * B_Q^max = n_beacons + window pre-RoPE queries:
+ *   bkv_init_beacons    buffer = FPS (Algorithm 1, fp64 similarities) of the
+ *                       head's n_init prompt queries down to n_beacons rows;
+ *   bkv_update_beacons  each new query is appended in order; whenever the
+ *                       buffer holds B_Q^max rows it is replaced by its FPS
+ *                       selection of n_beacons rows (Eq. 9);
+ *   bkv_compress        the beacons of head h are the FPS selection of
+ *                       min(n_beacons, size) buffer rows, rotated to t_pos;
+ *                       the group scores with its G * n_beacons beacons and
+ *                       G * window recent queries; after an eviction each
+ *                       buffer becomes the FPS selection of n_beacons rows of
+ *                       (its beacons, then its window queries in order).
+ * The FPS of the buffer steps takes its similarities in fp32: fused
+ * multiply-add dot products in element order, cos = dot / (|a| |b|) (0 for a
+ * zero vector), the averages summed in row order, ties to the lowest row.
+ * Requires n_beacons >= 1, window >= 1, n_beacons + window <= 32 and
+ * G * (n_beacons + window) <= 128.  The centroid state functions do not apply.
+ */
+#define BKV_F_CONTINUAL_FPS 2u
 
 typedef struct bkv_ctx bkv_ctx;
 
@@ -131,7 +154,8 @@ int bkv_init_beacons(bkv_ctx* ctx, const void* q_init, int32_t n_init);
  * ties below about 1e-12 relative.
  *   q_new       bf16 [n_layers][batch][n_q_heads][n_new][head_dim], pre-RoPE.
  *   assign_out  int32 [n_layers][batch][n_q_heads][n_new] or NULL: the beacon
- *               chosen for each query, -1 when it was skipped.
+ *               chosen for each query, -1 when it was skipped (all -1 under
+ *               BKV_F_CONTINUAL_FPS, which assigns nothing).
  * n_new == 0 is a no-op.  BKV_ESTATE if bkv_init_beacons / bkv_set_state was
  * never called.
  */
@@ -179,6 +203,17 @@ int bkv_get_state(bkv_ctx* ctx, float* centroids, double* sums, int64_t* counts)
 int bkv_set_state(bkv_ctx* ctx, const float* centroids, const double* sums, const int64_t* counts);
 
 /*
+ * Continual FPS contexts: copies the buffers to / from caller DEVICE memory.
+ *   buffers  bf16 [n_layers][batch][n_q_heads][n_beacons + window][head_dim];
+ *            rows [0, size) of each head are in use, in buffer order.
+ *   sizes    int32 [n_layers][batch][n_q_heads], each in 0..n_beacons + window - 1.
+ * bkv_set_cfps_state needs both and marks the state as initialised.
+ * BKV_EINVAL on a context without BKV_F_CONTINUAL_FPS.
+ */
+int bkv_get_cfps_state(bkv_ctx* ctx, void* buffers, int32_t* sizes);
+int bkv_set_cfps_state(bkv_ctx* ctx, const void* buffers, const int32_t* sizes);
+
+/*
  * Waits for the context's stream, then reads and clears the device error
  * word.  Returns BKV_OK, BKV_ETIMEOUT (a kernel gave up a bounded wait and
  * its outputs are invalid) or BKV_ECUDA.
@@ -212,7 +247,8 @@ int bkv_selftest_wait_timeout(bkv_ctx* ctx, int64_t limit_ns);
 #define BKV_K_SCORE 3
 #define BKV_K_SELECT_GATHER 4
 #define BKV_K_KEEP_ALL 5
-#define BKV_NUM_KERNELS 6
+#define BKV_K_CFPS 6 /* Continual FPS buffer update, beacon selection and merge */
+#define BKV_NUM_KERNELS 7
 int bkv_profile_enable(bkv_ctx* ctx, int on);
 int bkv_profile_read(bkv_ctx* ctx, double* ms, int64_t* launches, int32_t n_kernels);
 

@@ -23,12 +23,13 @@ BKV_ECUDA = -3
 BKV_ETIMEOUT = -4
 BKV_ESTATE = -5
 
-KERNEL_NAMES = ("fps_init", "update", "qobs", "score", "select_gather", "keep_all")
+KERNEL_NAMES = ("fps_init", "update", "qobs", "score", "select_gather", "keep_all", "cfps")
 
 
 # bkv_config.flags options (include/bkv.h)
 BKV_F_NONE = 0
 BKV_F_MEAN_AGG = 1
+BKV_F_CONTINUAL_FPS = 2
 
 
 class BkvConfig(ctypes.Structure):
@@ -71,6 +72,8 @@ def load_library(path: str | None = None, build: bool = True):
                                             _P, _P]),
             "bkv_get_state": (ctypes.c_int, [_P, _P, _P, _P]),
             "bkv_set_state": (ctypes.c_int, [_P, _P, _P, _P]),
+            "bkv_get_cfps_state": (ctypes.c_int, [_P, _P, _P]),
+            "bkv_set_cfps_state": (ctypes.c_int, [_P, _P, _P]),
             "bkv_sync": (ctypes.c_int, [_P]),
             "bkv_selftest_wait_timeout": (ctypes.c_int, [_P, ctypes.c_int64]),
             "bkv_compress_static": (ctypes.c_int, [ctypes.POINTER(BkvConfig), _P, _P, _P, _P, ctypes.c_int32,
@@ -179,6 +182,16 @@ def bkv_set_state(ctx, centroids, sums, counts) -> None:
                               _ptr(counts, torch.int64, "counts")), "bkv_set_state", ctx)
 
 
+def bkv_get_cfps_state(ctx, buffers=None, sizes=None) -> None:
+    _check(_l().bkv_get_cfps_state(ctx, _ptr(buffers, torch.bfloat16, "buffers"), _ptr(sizes, torch.int32, "sizes")),
+           "bkv_get_cfps_state", ctx)
+
+
+def bkv_set_cfps_state(ctx, buffers, sizes) -> None:
+    _check(_l().bkv_set_cfps_state(ctx, _ptr(buffers, torch.bfloat16, "buffers"), _ptr(sizes, torch.int32, "sizes")),
+           "bkv_set_cfps_state", ctx)
+
+
 def bkv_sync(ctx) -> None:
     _check(_l().bkv_sync(ctx), "bkv_sync", ctx)
 
@@ -238,19 +251,19 @@ class BeaconKV:
     """
 
     def __init__(self, *, n_layers, batch, n_q_heads, n_kv_heads, head_dim, n_beacons, window, capacity,
-                 rope_theta=0.0, n_prefix=0, stream=None, mean_agg=False):
-        flags = BKV_F_MEAN_AGG if mean_agg else BKV_F_NONE
+                 rope_theta=0.0, n_prefix=0, stream=None, mean_agg=False, continual_fps=False):
+        flags = (BKV_F_MEAN_AGG if mean_agg else BKV_F_NONE) | (BKV_F_CONTINUAL_FPS if continual_fps else BKV_F_NONE)
         self.cfg = BkvConfig(n_layers, batch, n_q_heads, n_kv_heads, head_dim, n_beacons, window, n_prefix,
                              capacity, float(rope_theta), flags)
         self.ctx = bkv_create(self.cfg, stream)
         self.n_inst = n_layers * batch * n_kv_heads
 
     @classmethod
-    def for_workload(cls, wl, stream=None, capacity=None, mean_agg=False) -> "BeaconKV":
+    def for_workload(cls, wl, stream=None, capacity=None, mean_agg=False, continual_fps=False) -> "BeaconKV":
         return cls(n_layers=wl.n_layers, batch=wl.batch, n_q_heads=wl.n_q_heads, n_kv_heads=wl.n_kv_heads,
                    head_dim=wl.head_dim, n_beacons=wl.n_beacons, window=wl.window,
                    capacity=capacity or wl.capacity, rope_theta=wl.rope_theta, n_prefix=wl.n_prefix, stream=stream,
-                   mean_agg=mean_agg)
+                   mean_agg=mean_agg, continual_fps=continual_fps)
 
     def close(self):
         if self.ctx:
@@ -287,6 +300,19 @@ class BeaconKV:
 
     def set_state(self, cent, sums, counts):
         bkv_set_state(self.ctx, cent, sums, counts)
+
+    def cfps_state(self):
+        """Continual FPS buffers: (bf16 [L, B, Hq, n_beacons + window, d], int32 sizes [L, B, Hq])."""
+        c = self.cfg
+        dev = torch.device("cuda", torch.cuda.current_device())
+        buf = torch.empty(c.n_layers, c.batch, c.n_q_heads, c.n_beacons + c.window, c.head_dim, dtype=torch.bfloat16,
+                          device=dev)
+        sizes = torch.empty(c.n_layers, c.batch, c.n_q_heads, dtype=torch.int32, device=dev)
+        bkv_get_cfps_state(self.ctx, buf, sizes)
+        return buf, sizes
+
+    def set_cfps_state(self, buf, sizes):
+        bkv_set_cfps_state(self.ctx, buf, sizes)
 
     def sync(self):
         bkv_sync(self.ctx)

@@ -26,6 +26,12 @@ struct bkv_ctx {
   double* sums = nullptr;
   long long* counts = nullptr;
   bool state_ready = false;
+  // Continual FPS (BKV_F_CONTINUAL_FPS): per-query-head buffers; cent / counts then hold each
+  // compress's beacons ([n_inst][G * n_beacons] rows, count 1 or 0) for the scoring-query build
+  bool cfps = false;
+  int b_min = 0, b_max = 0, n_heads = 0;
+  __nv_bfloat16* cbuf = nullptr;  // [n_heads][b_max][d]
+  int* csize = nullptr;           // [n_heads]
   // scratch
   __nv_bfloat16* qobs = nullptr;  // [n_inst][n_obs_pad][d]
   uint32_t* valid = nullptr;      // [n_inst][4]
@@ -152,11 +158,14 @@ int validate_config(const bkv_config* cfg, std::string& why) {
   if (cfg->n_prefix < 0) return bad("n_prefix must be >= 0");
   if (cfg->capacity < 1 || cfg->capacity > bkv::kMaxCapacity) return bad("capacity must be in 1..32768");
   if (!(cfg->rope_theta >= 0.0) || !std::isfinite(cfg->rope_theta)) return bad("rope_theta must be finite and >= 0");
-  if (cfg->flags & ~BKV_F_MEAN_AGG) return bad("flags holds an unknown option");
+  if (cfg->flags & ~(BKV_F_MEAN_AGG | BKV_F_CONTINUAL_FPS)) return bad("flags holds an unknown option");
   const long long G = cfg->n_q_heads / cfg->n_kv_heads;
-  const long long n_obs = G * cfg->window + cfg->n_beacons;
+  const bool cfps = (cfg->flags & BKV_F_CONTINUAL_FPS) != 0;
+  if (cfps && (cfg->n_beacons < 1 || cfg->window < 1 || cfg->n_beacons + cfg->window > bkv::kCfpsMaxRows))
+    return bad("continual FPS needs n_beacons >= 1, window >= 1 and n_beacons + window <= 32");
+  const long long n_obs = G * cfg->window + (cfps ? G * cfg->n_beacons : cfg->n_beacons);
   if (n_obs < 1 || n_obs > bkv::kMaxObs) {
-    snprintf(buf, sizeof buf, "G * window + n_beacons = %lld must be in 1..128", n_obs);
+    snprintf(buf, sizeof buf, "scoring queries per KV head (G * window + beacons) = %lld must be in 1..128", n_obs);
     why = buf;
     return BKV_EINVAL;
   }
@@ -182,6 +191,8 @@ void free_all(bkv_ctx* c) {
   cudaFree(c->cent);
   cudaFree(c->sums);
   cudaFree(c->counts);
+  cudaFree(c->cbuf);
+  cudaFree(c->csize);
   cudaFree(c->qobs);
   cudaFree(c->valid);
   cudaFree(c->rscore);
@@ -221,8 +232,12 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
   s.G = cfg->n_q_heads / cfg->n_kv_heads;
   s.n_inst = cfg->n_layers * cfg->batch * cfg->n_kv_heads;
   s.d = cfg->head_dim;
-  s.nb = cfg->n_beacons;
+  c->cfps = (cfg->flags & BKV_F_CONTINUAL_FPS) != 0;
+  s.nb = c->cfps ? s.G * cfg->n_beacons : cfg->n_beacons;  // beacon scoring rows per instance
   s.W = cfg->window;
+  c->b_min = cfg->n_beacons;
+  c->b_max = cfg->n_beacons + cfg->window;
+  c->n_heads = c->cfps ? cfg->n_layers * cfg->batch * cfg->n_q_heads : 0;
   s.n_prefix = cfg->n_prefix;
   s.cap = cfg->capacity;
   s.n_obs = s.G * s.W + s.nb;
@@ -232,9 +247,12 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
 
   const size_t ni = static_cast<size_t>(s.n_inst);
   cudaError_t e = cudaSuccess;
+  const size_t nh = static_cast<size_t>(c->n_heads);
   if ((e = dmalloc(&c->cent, ni * s.nb * s.d)) != cudaSuccess ||
-      (e = dmalloc(&c->sums, ni * s.nb * s.d)) != cudaSuccess ||
+      (e = dmalloc(&c->sums, c->cfps ? 0 : ni * s.nb * s.d)) != cudaSuccess ||
       (e = dmalloc(&c->counts, ni * s.nb)) != cudaSuccess ||
+      (e = dmalloc(&c->cbuf, nh * c->b_max * s.d)) != cudaSuccess ||
+      (e = dmalloc(&c->csize, nh)) != cudaSuccess ||
       (e = dmalloc(&c->qobs, ni * s.n_obs_pad * s.d)) != cudaSuccess ||
       (e = dmalloc(&c->valid, ni * 4)) != cudaSuccess ||
       (e = dmalloc(&c->rscore, ni * s.cap)) != cudaSuccess ||
@@ -247,7 +265,8 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
     return code;
   }
   if ((e = cudaMemsetAsync(c->cent, 0, sizeof(float) * ni * s.nb * s.d + 0, c->stream)) != cudaSuccess ||
-      (e = cudaMemsetAsync(c->sums, 0, sizeof(double) * ni * s.nb * s.d, c->stream)) != cudaSuccess ||
+      (e = cudaMemsetAsync(c->sums, 0, sizeof(double) * (c->cfps ? 1 : ni * s.nb * s.d), c->stream)) != cudaSuccess ||
+      (e = cudaMemsetAsync(c->csize, 0, sizeof(int) * (nh ? nh : 1), c->stream)) != cudaSuccess ||
       (e = cudaMemsetAsync(c->counts, 0, sizeof(long long) * ni * s.nb, c->stream)) != cudaSuccess ||
       (e = cudaMemsetAsync(c->err, 0, sizeof(int), c->stream)) != cudaSuccess) {
     free_all(c);
@@ -280,6 +299,24 @@ int bkv_init_beacons(bkv_ctx* ctx, const void* q_init, int32_t n_init) {
     return BKV_OK;
   }
   if (!q_init || !aligned16(q_init)) return fail(ctx, BKV_EINVAL, "q_init must be a non-NULL 16-byte aligned pointer");
+  if (ctx->cfps) {
+    // per query head: FPS of its n_init prompt queries down to n_beacons rows (the buffer)
+    if (n_init < ctx->b_min || n_init > bkv::kMaxFpsRows)
+      return fail(ctx, BKV_EINVAL, "n_init = %d must be in n_beacons..4096", n_init);
+    Shape hs = s;
+    hs.n_inst = ctx->n_heads;
+    hs.G = 1;
+    hs.nb = ctx->b_min;
+    ProfScope ps(ctx, BKV_K_FPS);
+    cudaError_t e = bkv::launch_fps_init(hs, static_cast<const __nv_bfloat16*>(q_init), n_init, ctx->cent, nullptr,
+                                         ctx->counts, ctx->stream);
+    if (e == cudaSuccess)
+      e = bkv::launch_cfps_seed(s.d, ctx->cent, ctx->n_heads, ctx->b_min, ctx->b_max, ctx->cbuf, ctx->csize,
+                                ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "continual FPS seeding launch");
+    ctx->state_ready = true;
+    return BKV_OK;
+  }
   const long long N = 1LL * s.G * n_init;
   if (n_init < 1 || N < s.nb || N > bkv::kMaxFpsRows)
     return fail(ctx, BKV_EINVAL, "G * n_init = %lld must be in n_beacons..4096", N);
@@ -309,6 +346,27 @@ int bkv_update_beacons(bkv_ctx* ctx, const void* q_new, int32_t n_new, int32_t* 
     return BKV_OK;
   }
   if (!ctx->state_ready) return fail(ctx, BKV_ESTATE, "update before bkv_init_beacons / bkv_set_state");
+  if (ctx->cfps) {
+    if (assign_out) {  // nothing is assigned in this mode
+      cudaError_t e =
+          cudaMemsetAsync(assign_out, 0xff, sizeof(int32_t) * s.n_inst * s.G * static_cast<size_t>(n_new), ctx->stream);
+      if (e != cudaSuccess) return cuda_fail(ctx, e, "assign_out memset");
+    }
+    bkv::CfpsArgs ca{};
+    ca.mode = bkv::kCfpsUpdate;
+    ca.H = ctx->n_heads;
+    ca.b_min = ctx->b_min;
+    ca.b_max = ctx->b_max;
+    ca.q = static_cast<const __nv_bfloat16*>(q_new);
+    ca.n_q = n_new;
+    ca.buf = ctx->cbuf;
+    ca.size = ctx->csize;
+    ca.bcn = ctx->cent;
+    ca.bcnt = ctx->counts;
+    ProfScope ps(ctx, BKV_K_CFPS);
+    cudaError_t e = bkv::launch_cfps(s.d, ca, ctx->stream);
+    return e == cudaSuccess ? BKV_OK : cuda_fail(ctx, e, "continual FPS update launch");
+  }
   // a tile is at most 128 queries of one instance: boxes no taller than that
   const uint64_t q_rows = static_cast<uint64_t>(s.n_inst) * s.G * n_new;
   uint64_t box_rows = (static_cast<uint64_t>(s.G) * n_new + 7) / 8 * 8;
@@ -369,6 +427,20 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
                         cudaMemcpyHostToDevice, ctx->stream);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "rope table upload");
   }
+  bkv::CfpsArgs ca{};
+  if (ctx->cfps) {  // this compress's beacons: FPS of each head's buffer, into cent / counts
+    ca.H = ctx->n_heads;
+    ca.b_min = ctx->b_min;
+    ca.b_max = ctx->b_max;
+    ca.buf = ctx->cbuf;
+    ca.size = ctx->csize;
+    ca.bcn = ctx->cent;
+    ca.bcnt = ctx->counts;
+    ca.mode = bkv::kCfpsBeacons;
+    ProfScope ps(ctx, BKV_K_CFPS);
+    e = bkv::launch_cfps(s.d, ca, ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "continual FPS beacon launch");
+  }
   {
     ProfScope ps(ctx, BKV_K_QOBS);
     e = bkv::launch_qobs(s, static_cast<const __nv_bfloat16*>(q_recent), ctx->cent, ctx->counts, ctx->rope, rotate,
@@ -403,11 +475,20 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
                                   static_cast<__nv_bfloat16*>(V), kept_idx_out, ctx->stream);
   }
   if (e != cudaSuccess) return cuda_fail(ctx, e, "select_gather launch");
+  if (ctx->cfps) {  // after the eviction: buffer = FPS of (beacons, then the window queries)
+    ca.mode = bkv::kCfpsMerge;
+    ca.q = static_cast<const __nv_bfloat16*>(q_recent);
+    ca.n_q = s.W;
+    ProfScope ps(ctx, BKV_K_CFPS);
+    e = bkv::launch_cfps(s.d, ca, ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "continual FPS merge launch");
+  }
   return BKV_OK;
 }
 
 int bkv_get_state(bkv_ctx* ctx, float* centroids, double* sums, int64_t* counts) {
   if (!ctx) return BKV_EINVAL;
+  if (ctx->cfps) return fail(ctx, BKV_EINVAL, "a continual FPS context has no centroid state");
   const Shape& s = ctx->shape;
   const size_t n = static_cast<size_t>(s.n_inst) * s.nb;
   cudaError_t e = cudaSuccess;
@@ -425,6 +506,7 @@ int bkv_get_state(bkv_ctx* ctx, float* centroids, double* sums, int64_t* counts)
 
 int bkv_set_state(bkv_ctx* ctx, const float* centroids, const double* sums, const int64_t* counts) {
   if (!ctx) return BKV_EINVAL;
+  if (ctx->cfps) return fail(ctx, BKV_EINVAL, "a continual FPS context has no centroid state");
   const Shape& s = ctx->shape;
   if (!centroids || !sums || !counts) return fail(ctx, BKV_EINVAL, "set_state needs all three arrays");
   const size_t n = static_cast<size_t>(s.n_inst) * s.nb;
@@ -436,6 +518,35 @@ int bkv_set_state(bkv_ctx* ctx, const float* centroids, const double* sums, cons
       (e = cudaMemcpyAsync(ctx->counts, counts, sizeof(int64_t) * n, cudaMemcpyDeviceToDevice, ctx->stream)) !=
           cudaSuccess)
     return cuda_fail(ctx, e, "set_state copy");
+  ctx->state_ready = true;
+  return BKV_OK;
+}
+
+int bkv_get_cfps_state(bkv_ctx* ctx, void* buffers, int32_t* sizes) {
+  if (!ctx) return BKV_EINVAL;
+  if (!ctx->cfps) return fail(ctx, BKV_EINVAL, "not a continual FPS context");
+  const size_t nh = static_cast<size_t>(ctx->n_heads);
+  cudaError_t e = cudaSuccess;
+  if (buffers && (e = cudaMemcpyAsync(buffers, ctx->cbuf, sizeof(__nv_bfloat16) * nh * ctx->b_max * ctx->shape.d,
+                                      cudaMemcpyDeviceToDevice, ctx->stream)) != cudaSuccess)
+    return cuda_fail(ctx, e, "get_cfps_state buffers");
+  if (sizes && (e = cudaMemcpyAsync(sizes, ctx->csize, sizeof(int32_t) * nh, cudaMemcpyDeviceToDevice, ctx->stream)) !=
+                   cudaSuccess)
+    return cuda_fail(ctx, e, "get_cfps_state sizes");
+  return BKV_OK;
+}
+
+int bkv_set_cfps_state(bkv_ctx* ctx, const void* buffers, const int32_t* sizes) {
+  if (!ctx) return BKV_EINVAL;
+  if (!ctx->cfps) return fail(ctx, BKV_EINVAL, "not a continual FPS context");
+  if (!buffers || !sizes) return fail(ctx, BKV_EINVAL, "set_cfps_state needs buffers and sizes");
+  const size_t nh = static_cast<size_t>(ctx->n_heads);
+  cudaError_t e;
+  if ((e = cudaMemcpyAsync(ctx->cbuf, buffers, sizeof(__nv_bfloat16) * nh * ctx->b_max * ctx->shape.d,
+                           cudaMemcpyDeviceToDevice, ctx->stream)) != cudaSuccess ||
+      (e = cudaMemcpyAsync(ctx->csize, sizes, sizeof(int32_t) * nh, cudaMemcpyDeviceToDevice, ctx->stream)) !=
+          cudaSuccess)
+    return cuda_fail(ctx, e, "set_cfps_state");
   ctx->state_ready = true;
   return BKV_OK;
 }

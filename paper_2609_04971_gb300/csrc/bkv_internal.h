@@ -28,7 +28,26 @@ constexpr int kMaxWindow = 64;
 constexpr int kMaxCapacity = 32768;
 constexpr int kMaxFpsRows = 4096;
 
-// ---- beacon maintenance (k_fps.cu, k_update.cu)
+// ---- Continual FPS buffers (k_cfps.cu)
+constexpr int kCfpsMaxRows = 32;  // b_max = n_beacons + window per query head
+enum { kCfpsUpdate = 0, kCfpsBeacons = 1, kCfpsMerge = 2 };
+struct CfpsArgs {
+  int mode;                 // kCfpsUpdate / kCfpsBeacons / kCfpsMerge
+  int H;                    // query heads: n_layers * batch * n_q_heads
+  int b_min, b_max;         // n_beacons, n_beacons + window
+  const __nv_bfloat16* q;   // update: q_new [H][n_q][d]; merge: q_recent [H][n_q][d]; beacons: unused
+  int n_q;                  // n_new (update) or window (merge)
+  __nv_bfloat16* buf;       // [H][b_max][d] buffers
+  int* size;                // [H] rows in use
+  float* bcn;               // [H][b_min][d] beacons of a compress (fp32 copies of bf16 queries)
+  long long* bcnt;          // [H][b_min] 1 for a beacon, 0 for an empty slot
+};
+cudaError_t launch_cfps(int d, const CfpsArgs& a, cudaStream_t st);
+// Buffers seeded with b_min fp32 rows per head (FPS picks of the prompt), size b_min.
+cudaError_t launch_cfps_seed(int d, const float* rows, int H, int b_min, int b_max, __nv_bfloat16* buf, int* size,
+                             cudaStream_t st);
+
+// ---- beacon maintenance (k_fps.cu, k_update.cu); fps_init's sums may be NULL
 cudaError_t launch_fps_init(const Shape& s, const __nv_bfloat16* q_init, int n_init, float* cent, double* sums,
                             long long* counts, cudaStream_t st);
 

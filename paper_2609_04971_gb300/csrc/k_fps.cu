@@ -161,7 +161,7 @@ __global__ void __launch_bounds__(kFpsThreads) fps_init_kernel(const __nv_bfloat
     const int k = idx / D, i = idx % D;
     const __nv_bfloat16 v = x[static_cast<size_t>(picks[k]) * D + i];
     cent[(static_cast<size_t>(e) * nb + k) * D + i] = __bfloat162float(v);
-    sums[(static_cast<size_t>(e) * nb + k) * D + i] = bf(v);
+    if (sums) sums[(static_cast<size_t>(e) * nb + k) * D + i] = bf(v);
   }
   for (int k = threadIdx.x; k < nb; k += blockDim.x) counts[static_cast<size_t>(e) * nb + k] = 1;
 }

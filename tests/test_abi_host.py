@@ -53,11 +53,21 @@ def test_strerror_and_version(lib):
 
 @pytest.mark.parametrize("field,value", [
     ("n_kv_heads", 3), ("head_dim", 96), ("n_beacons", 33), ("window", -1), ("window", 65),
-    ("capacity", 0), ("capacity", 40000), ("rope_theta", -1.0), ("flags", 2), ("flags", 0x80000000), ("n_layers", 0),
+    ("capacity", 0), ("capacity", 40000), ("rope_theta", -1.0), ("flags", 4), ("flags", 0x80000000), ("n_layers", 0),
     ("n_prefix", -2)])
 def test_create_rejects_bad_config_before_touching_the_gpu(lib, field, value):
     cfg = bkv.BkvConfig(1, 1, 4, 2, 64, 4, 8, 0, 1088, 1e4, 0)
     setattr(cfg, field, value)
+    out = ctypes.c_void_p()
+    assert lib.bkv_create(ctypes.byref(cfg), None, ctypes.byref(out)) == bkv.BKV_EINVAL
+    assert not out.value
+
+
+@pytest.mark.parametrize("n_beacons,window,n_q_heads", [(0, 8, 4), (8, 0, 4), (20, 13, 4), (16, 16, 16)])
+def test_create_rejects_bad_continual_fps_config(lib, n_beacons, window, n_q_heads):
+    """Continual FPS needs n_beacons >= 1, window >= 1, n_beacons + window <= 32 and
+    G * (n_beacons + window) <= 128 (here G = n_q_heads / 2)."""
+    cfg = bkv.BkvConfig(1, 1, n_q_heads, 2, 64, n_beacons, window, 0, 1088, 1e4, bkv.BKV_F_CONTINUAL_FPS)
     out = ctypes.c_void_p()
     assert lib.bkv_create(ctypes.byref(cfg), None, ctypes.byref(out)) == bkv.BKV_EINVAL
     assert not out.value

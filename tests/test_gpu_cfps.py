@@ -1,0 +1,135 @@
+"""Continual FPS beacons (BKV_F_CONTINUAL_FPS) through the C ABI against the oracle.
+
+Every query head is checked: the FPS seeding (fp64 similarities; picks equal up
+to ties below 1e-12), the fill-and-compress buffer after a call of many new
+queries (fp32 decisions, taken with the same operations on both sides, so the
+buffers must be identical), the compress on the resulting beacons (scores,
+kept set, compacted rows, as in tests/parity.py) and the post-eviction merge.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_04971_gb300.workloads import QWEN3_4B, TINY
+
+pytestmark = pytest.mark.gpu
+
+if torch.cuda.is_available():
+    from oracle import oracle as O
+    from paper_2609_04971_gb300 import synth
+    from paper_2609_04971_gb300.bkv import BeaconKV
+    from tests import parity as P
+
+
+def _bits(t: torch.Tensor) -> np.ndarray:
+    return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def _heads(t: torch.Tensor, d: int) -> np.ndarray:
+    """[L, B, Hq, n, d] bf16 -> uint16 [heads, n, d]."""
+    return _bits(t).reshape(-1, t.shape[-2], d)
+
+
+def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None):
+    dev = torch.device("cuda")
+    inp = synth.step_inputs(wl, seed, dev)
+    L = wl.L if L is None else L
+    budget = wl.budget if budget is None else budget
+    d, G, W = wl.head_dim, wl.group, wl.window
+    b_max = b_min + W
+    lib = O.load()
+    q_new_t = inp["q_new"] if n_new is None else inp["q_new"][..., :n_new, :].contiguous()
+    bk = BeaconKV(n_layers=wl.n_layers, batch=wl.batch, n_q_heads=wl.n_q_heads, n_kv_heads=wl.n_kv_heads, head_dim=d,
+                  n_beacons=b_min, window=W, capacity=wl.capacity, rope_theta=wl.rope_theta, n_prefix=wl.n_prefix,
+                  continual_fps=True)
+    try:
+        bk.init_beacons(inp["q_init"])
+        buf0, size0 = [x.cpu() for x in bk.cfps_state()]
+        bk.update(q_new_t)
+        buf1, size1 = [x.cpu() for x in bk.cfps_state()]
+        K, V = inp["K"], inp["V"]
+        n_inst = wl.n_inst
+        Kb = _bits(K).reshape(n_inst, wl.capacity, d)
+        Vb = _bits(V).reshape(n_inst, wl.capacity, d)
+        scores = torch.full((wl.n_layers, wl.batch, wl.n_kv_heads, wl.capacity), -1.0, device=dev)
+        kept = bk.compress(K, V, L=L, budget=budget, t_pos=inp["t_pos"], q_recent=inp["q_recent"],
+                           recent_pos=inp["recent_pos"], scores_out=scores)
+        buf2, size2 = [x.cpu() for x in bk.cfps_state()]
+        bk.sync()
+        K1 = _bits(K).reshape(n_inst, wl.capacity, d)
+        V1 = _bits(V).reshape(n_inst, wl.capacity, d)
+    finally:
+        bk.close()
+
+    q_init = _heads(inp["q_init"], d)
+    q_new = _heads(q_new_t, d)
+    q_rec = _heads(inp["q_recent"], d)
+    buf0 = buf0.view(torch.int16).numpy().view(np.uint16).reshape(-1, b_max, d)
+    buf1 = buf1.view(torch.int16).numpy().view(np.uint16).reshape(-1, b_max, d)
+    buf2 = buf2.view(torch.int16).numpy().view(np.uint16).reshape(-1, b_max, d)
+    size0, size1, size2 = (x.numpy().reshape(-1) for x in (size0, size1, size2))
+    n_heads = q_init.shape[0]
+    fps_ties = 0
+    for h in range(n_heads):
+        # ---- seeding: fp64 FPS of the head's prompt queries
+        picks, gaps = O.fps(q_init[h], b_min, lib)
+        assert size0[h] == b_min
+        if not np.array_equal(buf0[h, :b_min], q_init[h][picks]):
+            first = next(k for k in range(b_min) if not np.array_equal(buf0[h, k], q_init[h][picks[k]]))
+            assert gaps[first] < P.ASSIGN_TIE, f"head {h}: seed pick {first} differs, fp64 gap {gaps[first]:.2e}"
+            fps_ties += 1
+        # ---- update from the GPU's seed: identical fp32 decisions
+        want, wsize, _, _ = O.cfps_update(buf0[h], int(size0[h]), b_min, b_max, q_new[h], lib)
+        assert size1[h] == wsize, f"head {h}: size {size1[h]} vs {wsize}"
+        np.testing.assert_array_equal(buf1[h, :wsize], want[:wsize], err_msg=f"head {h}: buffer after update")
+
+    rel_max, swaps = 0.0, 0
+    kept_h = kept.view(n_inst, budget).cpu().numpy()
+    s_h = scores.view(n_inst, wl.capacity).cpu().numpy()
+    for e in range(n_inst):
+        # ---- this compress's beacons: FPS of each head's buffer, then its scoring queries
+        cent = np.zeros((G * b_min, d), np.float32)
+        counts = np.zeros(G * b_min, np.int64)
+        bcn = []
+        for g in range(G):
+            h = e * G + g
+            picks, _ = O.fps32(buf1[h, :size1[h]], b_min, lib)
+            rows = buf1[h][picks]
+            bcn.append(rows)
+            cent[g * b_min:g * b_min + len(picks)] = O.bf16_to_f64(rows)
+            counts[g * b_min:g * b_min + len(picks)] = 1
+        r, sw = P.check_compress(wl, cent, counts, q_rec[e * G:(e + 1) * G], inp["recent_pos"], inp["t_pos"],
+                                 Kb[e], Vb[e], K1[e], V1[e], kept_h[e], s_h[e], L, budget, lib, tag=f"instance {e}")
+        rel_max, swaps = max(rel_max, r), swaps + sw
+        # ---- merge after the eviction: FPS of (beacons, then the window queries)
+        for g in range(G):
+            h = e * G + g
+            if L > budget:
+                cand = np.vstack([bcn[g], q_rec[h]])
+                picks, _ = O.fps32(cand, b_min, lib)
+                want = cand[picks]
+            else:
+                want = buf1[h, :size1[h]]
+            assert size2[h] == len(want), f"head {h}: size after compress {size2[h]} vs {len(want)}"
+            np.testing.assert_array_equal(buf2[h, :len(want)], want, err_msg=f"head {h}: buffer after merge")
+    print(f"{wl.name}: {n_heads} heads, seed ties {fps_ties}, max score rel err {rel_max:.2e}, swaps {swaps}")
+
+
+@pytest.mark.parametrize("wl,b_min,seed", [
+    (TINY.scaled(name="cfps_tiny_d64"), 4, 21),
+    (QWEN3_4B.scaled(name="cfps_qwen3_4b_1L_b1_nb8", n_layers=1, batch=1), 8, 22),
+    (QWEN3_4B.scaled(name="cfps_qwen3_4b_1L_b1_nb16_w16", n_layers=1, batch=1, window=16), 16, 23),
+], ids=lambda x: getattr(x, "name", str(x)))
+def test_continual_fps_step(wl, b_min, seed):
+    _run_cfps(wl, seed, b_min)
+
+
+def test_continual_fps_short_call_and_no_eviction():
+    """A call too short to fill the buffer (no FPS), then a compress with L <= budget (no merge)."""
+    wl = QWEN3_4B.scaled(name="cfps_short_fits", n_layers=1, batch=1, L=256, budget=300)
+    _run_cfps(wl, 24, 8, n_new=3)
+
+
+def test_continual_fps_ragged_cache():
+    wl = QWEN3_4B.scaled(name="cfps_ragged_L1000_B700", n_layers=1, batch=2, L=1000, budget=700)
+    _run_cfps(wl, 25, 8)
