@@ -238,3 +238,36 @@ def check_compress(wl: Workload, cent: np.ndarray, counts: np.ndarray, q_recent:
     np.testing.assert_array_equal(K1[:budget], K0[kept_g], err_msg=f"{tag}: K compaction")
     np.testing.assert_array_equal(V1[:budget], V0[kept_g], err_msg=f"{tag}: V compaction")
     return rel_max, swaps
+
+
+def check_cfps_compress(wl: Workload, b_min: int, buf: np.ndarray, size: np.ndarray, q_rec: np.ndarray, recent_pos,
+                        t_pos: int, K0, V0, K1, V1, kept_g, scores_g, L: int, budget: int, buf_after: np.ndarray,
+                        size_after: np.ndarray, lib, tag: str = "", mean: bool = False) -> tuple:
+    """One compress of one instance in the Continual FPS mode.  buf / size: the G buffers of the
+    instance's query heads before the compress (uint16 [G, b_max, d], int [G]); q_rec: their window
+    queries (uint16 [G, W, d]); buf_after / size_after: the GPU's buffers after it.  The beacons are
+    the fp32 FPS selection of min(b_min, size) rows of each buffer; after an eviction each buffer must
+    be the FPS selection of b_min rows of (its beacons, then its window queries).
+    Returns (max score rel err, boundary swaps)."""
+    G, d = buf.shape[0], buf.shape[-1]
+    cent = np.zeros((G * b_min, d), np.float32)
+    counts = np.zeros(G * b_min, np.int64)
+    beacons = []
+    for g in range(G):
+        picks, _ = O.fps32(buf[g, :size[g]], b_min, lib)
+        rows = buf[g][picks]
+        beacons.append(rows)
+        cent[g * b_min:g * b_min + len(picks)] = O.bf16_to_f64(rows)
+        counts[g * b_min:g * b_min + len(picks)] = 1
+    rel, swaps = check_compress(wl, cent, counts, q_rec, recent_pos, t_pos, K0, V0, K1, V1, kept_g, scores_g, L,
+                                budget, lib, tag=tag, mean=mean)
+    for g in range(G):
+        if L > budget:
+            cand = np.vstack([beacons[g], q_rec[g]])
+            picks, _ = O.fps32(cand, b_min, lib)
+            want = cand[picks]
+        else:
+            want = buf[g, :size[g]]
+        assert size_after[g] == len(want), f"{tag} head {g}: buffer size {size_after[g]} vs {len(want)}"
+        np.testing.assert_array_equal(buf_after[g, :len(want)], want, err_msg=f"{tag} head {g}: buffer after merge")
+    return rel, swaps

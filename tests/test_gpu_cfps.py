@@ -87,31 +87,11 @@ def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None):
     kept_h = kept.view(n_inst, budget).cpu().numpy()
     s_h = scores.view(n_inst, wl.capacity).cpu().numpy()
     for e in range(n_inst):
-        # ---- this compress's beacons: FPS of each head's buffer, then its scoring queries
-        cent = np.zeros((G * b_min, d), np.float32)
-        counts = np.zeros(G * b_min, np.int64)
-        bcn = []
-        for g in range(G):
-            h = e * G + g
-            picks, _ = O.fps32(buf1[h, :size1[h]], b_min, lib)
-            rows = buf1[h][picks]
-            bcn.append(rows)
-            cent[g * b_min:g * b_min + len(picks)] = O.bf16_to_f64(rows)
-            counts[g * b_min:g * b_min + len(picks)] = 1
-        r, sw = P.check_compress(wl, cent, counts, q_rec[e * G:(e + 1) * G], inp["recent_pos"], inp["t_pos"],
-                                 Kb[e], Vb[e], K1[e], V1[e], kept_h[e], s_h[e], L, budget, lib, tag=f"instance {e}")
+        hs = slice(e * G, (e + 1) * G)
+        r, sw = P.check_cfps_compress(wl, b_min, buf1[hs], size1[hs], q_rec[hs], inp["recent_pos"], inp["t_pos"],
+                                      Kb[e], Vb[e], K1[e], V1[e], kept_h[e], s_h[e], L, budget, buf2[hs], size2[hs],
+                                      lib, tag=f"instance {e}")
         rel_max, swaps = max(rel_max, r), swaps + sw
-        # ---- merge after the eviction: FPS of (beacons, then the window queries)
-        for g in range(G):
-            h = e * G + g
-            if L > budget:
-                cand = np.vstack([bcn[g], q_rec[h]])
-                picks, _ = O.fps32(cand, b_min, lib)
-                want = cand[picks]
-            else:
-                want = buf1[h, :size1[h]]
-            assert size2[h] == len(want), f"head {h}: size after compress {size2[h]} vs {len(want)}"
-            np.testing.assert_array_equal(buf2[h, :len(want)], want, err_msg=f"head {h}: buffer after merge")
     print(f"{wl.name}: {n_heads} heads, seed ties {fps_ties}, max score rel err {rel_max:.2e}, swaps {swaps}")
 
 
