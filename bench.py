@@ -51,6 +51,10 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
+    ap.add_argument("--beacons", choices=["centroid", "continual-fps"], default="centroid",
+                    help="beacon maintenance: running-mean centroids, or the paper's Continual FPS buffers")
+    ap.add_argument("--cfps-beacons", type=int, default=8,
+                    help="Continual FPS: beacons per query head (the buffer holds this + window queries)")
     return ap.parse_args()
 
 
@@ -204,6 +208,18 @@ def reference_arm(args, wl, rank: int) -> None:
     print(json.dumps(line), flush=True)
 
 
+def cfps_bytes(wl) -> int:
+    """Algorithmic HBM bytes of the Continual FPS work of one step over all query heads: the update
+    reads the new queries and reads and writes each buffer (n_beacons + window bf16 rows); the beacon
+    selection reads the buffer and writes n_beacons fp32 rows and counts; the merge reads those and the
+    window queries and writes the buffer."""
+    d, nb, W = wl.head_dim, wl.n_beacons, wl.window
+    bmax = nb + W
+    per = (wl.n_new * d * 2 + 2 * bmax * d * 2) + (bmax * d * 2 + nb * (d * 4 + 8)) + \
+          (nb * (d * 4 + 8) + W * d * 2 + bmax * d * 2)
+    return per * wl.n_layers * wl.batch * wl.n_q_heads
+
+
 def config_block(wl, n_gpus: int) -> dict:
     return {"workload": wl.name, "layers": wl.n_layers, "batch": wl.batch, "q_heads": wl.n_q_heads,
             "kv_heads": wl.n_kv_heads, "head_dim": wl.head_dim, "L": wl.L, "budget": wl.budget,
@@ -259,6 +275,10 @@ def main():
     wl = WORKLOADS[args.config]
     if args.layers:
         wl = wl.scaled(n_layers=args.layers, name=f"{wl.name}_{args.layers}layers")
+    cfps = args.beacons == "continual-fps"
+    if cfps:  # n_beacons counts beacons per query head in this mode
+        wl = wl.scaled(n_beacons=args.cfps_beacons, name=f"{wl.name}_cfps{args.cfps_beacons}")
+        args.no_cpu_baseline = True  # the timed CPU oracle covers the centroid step
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
@@ -287,7 +307,7 @@ def main():
     new_v = V[:, :, :, budget:L].clone()
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     kept = torch.empty(wl.n_layers, wl.batch, wl.n_kv_heads, budget, dtype=torch.int32, device=dev)
-    bk = bkv.BeaconKV.for_workload(wl)
+    bk = bkv.BeaconKV.for_workload(wl, continual_fps=cfps)
     bk.init_beacons(inp["q_init"])
     bk.sync()
 
@@ -336,19 +356,27 @@ def main():
     # per-kernel roofline (algorithmic bytes per launch / measured duration per launch)
     d = wl.head_dim
     alg_bytes = {
-        "update": wl.update_bytes(),
+        "update": 0 if cfps else wl.update_bytes(),
         "qobs": wl.n_inst * wl.group * wl.window * d * 2,
         "score": wl.n_inst * L * d * 2,
         "select_gather": wl.n_inst * (budget * d * 2 * 4 + budget * 4),
     }
     kernels = {}
+    if cfps:  # three launches per step: buffer update, beacon selection, merge; accounted per step
+        ms, n = prof.get("cfps", (0.0, 0))
+        b = cfps_bytes(wl)
+        per = ms / args.steps
+        kernels["cfps"] = {"ms_per_step": per, "launches": n, "alg_bytes_per_step": b,
+                           "achieved_gbs": b / (per * 1e-3) / 1e9, "frac_of_hbm": b / (per * 1e-3) / 1e9 / hbm_gbs,
+                           "note": "per step: update (n_new queries per head) + beacon FPS + post-eviction merge"}
     for name, b in alg_bytes.items():
         ms, n = prof.get(name, (0.0, 0))
         if n:
             per = ms / n
             kernels[name] = {"ms_per_launch": per, "launches": n, "alg_bytes_per_launch": b,
                              "achieved_gbs": b / (per * 1e-3) / 1e9, "frac_of_hbm": b / (per * 1e-3) / 1e9 / hbm_gbs}
-    dom = max(kernels, key=lambda k: kernels[k]["ms_per_launch"] * kernels[k]["launches"])
+    dom = max((k for k in kernels if "ms_per_launch" in kernels[k]),
+              key=lambda k: kernels[k]["ms_per_launch"] * kernels[k]["launches"])
     kd = kernels[dom]
     traffic = traffic_from_profiles(dom, wl.n_inst)
     roofline = {"bound": "hbm", "kernel": dom, "achieved": kd["achieved_gbs"], "peak": hbm_gbs, "unit": "GB/s",
@@ -356,14 +384,20 @@ def main():
                 "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else
                 f"fallback {FALLBACK_HBM_GBS} GB/s"}
     step_roof_s = wl.roofline_seconds(hbm_gbs, bf16_tflops)
+    step_bytes, step_flops = wl.step_bytes(), wl.step_flops()
+    if cfps:
+        step_bytes = wl.compress_bytes() + cfps_bytes(wl)
+        step_flops = wl.compress_flops()
+        step_roof_s = max(step_bytes / (hbm_gbs * 1e9), step_flops / (bf16_tflops * 1e12))
     launches = sum(n for _, n in prof.values())
 
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config_block(wl, world),
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": dict(config_block(wl, world), beacon_mode=args.beacons),
         "roofline": roofline,
-        "step_roofline": {"alg_bytes": wl.step_bytes(), "alg_flops": wl.step_flops(),
+        "step_roofline": {"alg_bytes": step_bytes, "alg_flops": step_flops,
                           "roofline_ms": step_roof_s * 1e3, "frac": step_roof_s * 1e3 / ms_per_step},
         "kernels": kernels, "gpu_launches": launches, "clocks": clocks,
         "step_ms_p10_p50_p90": [float(x) for x in
