@@ -4,13 +4,17 @@
 // decode branch, its beacon freeze and its post-eviction merge.
 //
 // One warp per query head, kHeadsPerCta heads per CTA.  A head's buffer (at
-// most 32 rows) sits transposed in shared memory as bf16 [d][kPitch] with its
-// fp32 Gram matrix; lane j owns buffer row j.  The dot product of a new row
-// with row j is a fused multiply-add chain in element order, run by lane j;
-// the similarities are fp32 (cos = dot / (|a| |b|), 0 when a norm is 0) and
-// the farthest-point loop takes its argmins in the same precision and order
-// as the definition, ties to the lowest row.  These are the operations the
-// fp32 decisions of the reference are defined by, so both pick the same rows.
+// most 32 rows) sits transposed in shared memory as bf16 [d][kPitch], one
+// physical slot per column, with the fp32 cosines between slots; the buffer
+// order (which the FPS ties and the output follow) is a list of slots held
+// one per lane, so an FPS compression only permutes that list.  The dot
+// product of a new row with slot p is a fused multiply-add chain in element
+// order, run by lane p; the norms are fp32 square roots of the self dots and
+// each cosine dot / (|a| |b|) (0 when a norm is 0) is taken once, when its
+// later row arrives.  The farthest-point loop sums and compares those
+// cosines in the definition's order, ties to the lowest row.  These are the
+// operations the fp32 decisions of the reference are defined by, so both
+// pick the same rows.
 //
 // The same warp routine serves three calls:
 //   update   append the call's queries in order; whenever the buffer holds
@@ -27,22 +31,17 @@
 namespace bkv {
 namespace {
 
-constexpr int kHeadsPerCta = 8;
-constexpr int kMaxRows = kCfpsMaxRows;  // 32: one buffer row per lane
-constexpr int kChunk = 16;              // rows added to the Gram matrix per pass
+constexpr int kHeadsPerCta = 12;
+constexpr int kMaxRows = kCfpsMaxRows;  // 32: one slot per lane
+constexpr int kChunk = 8;               // rows added per pass over the elements
 constexpr int kPitch = 34;              // bf16 elements per transposed row (even; spreads banks)
 
 template <int D>
 struct WarpSmem {
-  __nv_bfloat16 xt[D][kPitch];          // buffer, transposed: xt[k][j] = element k of row j
+  __nv_bfloat16 xt[D][kPitch];          // slots, transposed: xt[k][p] = element k of slot p
   __align__(16) float xn[D][kChunk];    // the rows being added, fp32, for broadcast reads
-  float G[kMaxRows][kMaxRows + 1];      // Gram matrix of the buffer rows
-  int picks[kMaxRows];
+  float C[kMaxRows][kMaxRows + 1];      // cosines between slots
 };
-
-__device__ __forceinline__ float cos_of(float dot, float ni, float nj) {
-  return (ni == 0.f || nj == 0.f) ? 0.f : __fdiv_rn(dot, __fmul_rn(ni, nj));
-}
 
 // Warp-wide argmin of (v, lane), ties to the lower lane.
 __device__ __forceinline__ int warp_argmin(float v) {
@@ -59,138 +58,168 @@ __device__ __forceinline__ int warp_argmin(float v) {
   return i;
 }
 
-// Row `slot` of the buffer from `kPer` = D / 32 consecutive bf16 (or fp32) values per lane.
-template <int D>
-__device__ __forceinline__ void put_row(WarpSmem<D>& w, int slot, int u, const float (&v)[D / 32]) {
+// One head's buffer: the list of slots in buffer order (lane t holds row t's slot), the norm
+// of every slot (lane p holds slot p's), the set of slots in use and the number of rows.
+struct Buf {
+  int slot;
+  float nrm;
+  uint32_t used;
+  int n;
+};
+
+// A row to append: bf16 values, or fp32 values that hold bf16 numbers.
+struct RowSrc {
+  const void* p;
+  bool f32;
+};
+
+// Appends cnt <= kChunk rows, whose sources `src(u)` gives, to the end of the buffer.
+template <int D, typename Src>
+__device__ void add_rows(WarpSmem<D>& w, Buf& b, int cnt, Src src) {
   const int lane = threadIdx.x & 31;
+  int q[kChunk];  // slots of the new rows: the lowest free ones
+  uint32_t taken = b.used;
 #pragma unroll
-  for (int e = 0; e < D / 32; ++e) {
-    const int k = lane * (D / 32) + e;
-    w.xt[k][slot] = __float2bfloat16_rn(v[e]);  // exact: v holds a bf16 value
-    w.xn[k][u] = v[e];
+  for (int u = 0; u < kChunk; ++u) {
+    q[u] = u < cnt ? __ffs(~taken) - 1 : 0;
+    if (u < cnt) taken |= 1u << q[u];
   }
-}
-
-template <int D>
-__device__ __forceinline__ void load_bf16_row(const __nv_bfloat16* src, float (&v)[D / 32]) {
-  const int lane = threadIdx.x & 31;
-  if constexpr (D == 128) {
-    const uint2 p = *reinterpret_cast<const uint2*>(src + lane * 4);
-    v[0] = __uint_as_float(p.x << 16);
-    v[1] = __uint_as_float(p.x & 0xffff0000u);
-    v[2] = __uint_as_float(p.y << 16);
-    v[3] = __uint_as_float(p.y & 0xffff0000u);
-  } else {
-    const uint32_t p = *reinterpret_cast<const uint32_t*>(src + lane * 2);
-    v[0] = __uint_as_float(p << 16);
-    v[1] = __uint_as_float(p & 0xffff0000u);
-  }
-}
-
-template <int D>
-__device__ __forceinline__ void load_f32_row(const float* src, float (&v)[D / 32]) {
-  const int lane = threadIdx.x & 31;
+  // all the chunk's loads are in flight together (a global load takes about a microsecond)
+  RowSrc rs[kChunk];
 #pragma unroll
-  for (int e = 0; e < D / 32; ++e) v[e] = src[lane * (D / 32) + e];
-}
-
-// Gram entries of the staged rows [sz0, sz0 + cnt) with every row [0, sz0 + cnt).
-template <int D>
-__device__ void gram_add(WarpSmem<D>& w, int sz0, int cnt) {
-  const int j = threadIdx.x & 31;
+  for (int u = 0; u < kChunk; ++u) rs[u] = u < cnt ? src(u) : RowSrc{nullptr, false};
+  uint4 raw[kChunk];
+#pragma unroll
+  for (int u = 0; u < kChunk; ++u) {
+    raw[u] = make_uint4(0u, 0u, 0u, 0u);
+    if (rs[u].p) {
+      const char* base = static_cast<const char*>(rs[u].p);
+      if constexpr (D == 128) {
+        if (rs[u].f32)
+          asm volatile("ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%4];"
+                       : "=r"(raw[u].x), "=r"(raw[u].y), "=r"(raw[u].z), "=r"(raw[u].w) : "l"(base + lane * 16));
+        else
+          asm volatile("ld.global.nc.v2.u32 {%0,%1}, [%2];" : "=r"(raw[u].x), "=r"(raw[u].y) : "l"(base + lane * 8));
+      } else {
+        if (rs[u].f32)
+          asm volatile("ld.global.nc.v2.u32 {%0,%1}, [%2];" : "=r"(raw[u].x), "=r"(raw[u].y) : "l"(base + lane * 8));
+        else
+          asm volatile("ld.global.nc.u32 %0, [%1];" : "=r"(raw[u].x) : "l"(base + lane * 4));
+      }
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < kChunk; ++u) {
+    float v[D / 32];
+    if (rs[u].f32) {
+      const uint32_t r4[4] = {raw[u].x, raw[u].y, raw[u].z, raw[u].w};
+#pragma unroll
+      for (int e = 0; e < D / 32; ++e) v[e] = __uint_as_float(r4[e]);
+    } else {
+      const uint32_t r2[2] = {raw[u].x, raw[u].y};
+#pragma unroll
+      for (int e = 0; e < D / 32; ++e) v[e] = __uint_as_float((e & 1) ? (r2[e >> 1] & 0xffff0000u) : (r2[e >> 1] << 16));
+    }
+#pragma unroll
+    for (int e = 0; e < D / 32; ++e) {
+      const int k = lane * (D / 32) + e;
+      if (u < cnt) w.xt[k][q[u]] = __float2bfloat16_rn(v[e]);  // exact: v holds a bf16 value
+      w.xn[k][u] = u < cnt ? v[e] : 0.f;
+    }
+  }
   __syncwarp();
+  // lane p: dots of the new rows with slot p, element order
   float acc[kChunk];
 #pragma unroll
   for (int u = 0; u < kChunk; ++u) acc[u] = 0.f;
 #pragma unroll 4
   for (int k = 0; k < D; ++k) {
-    const float xj = __bfloat162float(w.xt[k][j]);
-    const float4* xr = reinterpret_cast<const float4*>(&w.xn[k][0]);
+    const float xp = __bfloat162float(w.xt[k][lane]);
+    const float4 a0 = *reinterpret_cast<const float4*>(&w.xn[k][0]);
+    const float4 a1 = *reinterpret_cast<const float4*>(&w.xn[k][4]);
+    acc[0] = __fmaf_rn(a0.x, xp, acc[0]);
+    acc[1] = __fmaf_rn(a0.y, xp, acc[1]);
+    acc[2] = __fmaf_rn(a0.z, xp, acc[2]);
+    acc[3] = __fmaf_rn(a0.w, xp, acc[3]);
+    acc[4] = __fmaf_rn(a1.x, xp, acc[4]);
+    acc[5] = __fmaf_rn(a1.y, xp, acc[5]);
+    acc[6] = __fmaf_rn(a1.z, xp, acc[6]);
+    acc[7] = __fmaf_rn(a1.w, xp, acc[7]);
+  }
+  // norms of the new slots (their self dots), then every cosine with a new row
 #pragma unroll
-    for (int q = 0; q < kChunk / 4; ++q) {
-      const float4 a = xr[q];
-      acc[4 * q + 0] = __fmaf_rn(a.x, xj, acc[4 * q + 0]);
-      acc[4 * q + 1] = __fmaf_rn(a.y, xj, acc[4 * q + 1]);
-      acc[4 * q + 2] = __fmaf_rn(a.z, xj, acc[4 * q + 2]);
-      acc[4 * q + 3] = __fmaf_rn(a.w, xj, acc[4 * q + 3]);
+  for (int u = 0; u < kChunk; ++u)
+    if (u < cnt && lane == q[u]) b.nrm = __fsqrt_rn(acc[u]);
+  const bool mine = (taken >> lane) & 1u;
+#pragma unroll
+  for (int u = 0; u < kChunk; ++u) {
+    if (u < cnt) {
+      const float nq = __shfl_sync(0xffffffffu, b.nrm, q[u]);
+      const float c = (nq == 0.f || b.nrm == 0.f) ? 0.f : __fdiv_rn(acc[u], __fmul_rn(nq, b.nrm));
+      if (mine) {
+        w.C[q[u]][lane] = c;
+        w.C[lane][q[u]] = c;
+      }
     }
   }
-  if (j < sz0 + cnt) {
 #pragma unroll
-    for (int u = 0; u < kChunk; ++u)
-      if (u < cnt) {
-        w.G[sz0 + u][j] = acc[u];
-        w.G[j][sz0 + u] = acc[u];
-      }
-  }
+  for (int u = 0; u < kChunk; ++u)
+    if (u < cnt && lane == b.n + u) b.slot = q[u];
+  b.used = taken;
+  b.n += cnt;
   __syncwarp();
 }
 
-// Algorithm 1 on the first n buffer rows; picks min(m, n) rows into w.picks.
+// Algorithm 1 on the buffer's rows; the buffer becomes its min(m, n) picks in pick order.
 template <int D>
-__device__ int fps_rows(WarpSmem<D>& w, int n, int m) {
-  const int j = threadIdx.x & 31;
+__device__ void fps_keep(WarpSmem<D>& w, Buf& b, int m) {
+  const int t = threadIdx.x & 31;
+  const int n = b.n;
   if (m > n) m = n;
-  const float nj = j < n ? __fsqrt_rn(w.G[j][j]) : 0.f;
-  float sum = 0.f;
-  for (int i = 0; i < n; ++i) {
-    const float ni = __shfl_sync(0xffffffffu, nj, i);
-    sum = __fadd_rn(sum, cos_of(w.G[i][j], ni, nj));
+  if (m <= 0) {
+    b.n = 0;
+    b.used = 0;
+    return;
   }
-  const float avg = j < n ? __fdiv_rn(sum, static_cast<float>(n)) : INFINITY;
+  const bool row = t < n;
+  const int pt = row ? b.slot : 0;
+  float sum = 0.f;
+  for (int i = 0; i < n; ++i) sum = __fadd_rn(sum, w.C[__shfl_sync(0xffffffffu, b.slot, i)][pt]);
+  const float avg = row ? __fdiv_rn(sum, static_cast<float>(n)) : INFINITY;
   int r = warp_argmin(avg);
-  if (j == 0) w.picks[0] = r;
-  bool sel = j == r;
-  float nr = __shfl_sync(0xffffffffu, nj, r);
-  float S = cos_of(w.G[r][j], nr, nj);
+  int pick = r;  // lane k ends up with the k-th pick
+  bool sel = t == r;
+  float S = w.C[__shfl_sync(0xffffffffu, b.slot, r)][pt];
   for (int k = 1; k < m; ++k) {
-    r = warp_argmin((j < n && !sel) ? S : INFINITY);
-    if (j == 0) w.picks[k] = r;
-    if (j == r) sel = true;
-    nr = __shfl_sync(0xffffffffu, nj, r);
-    const float c = cos_of(w.G[r][j], nr, nj);
+    r = warp_argmin((row && !sel) ? S : INFINITY);
+    if (t == k) pick = r;
+    if (t == r) sel = true;
+    const float c = w.C[__shfl_sync(0xffffffffu, b.slot, r)][pt];
     if (!sel && c > S) S = c;
   }
-  __syncwarp();
-  return m;
-}
-
-// The buffer becomes its rows picks[0 .. m), in that order (rows and Gram entries).
-template <int D>
-__device__ void keep_picks(WarpSmem<D>& w, int m) {
-  const int t = threadIdx.x & 31;
-  const int src = t < m ? w.picks[t] : 0;
-  for (int k = 0; k < D; ++k) {
-    const __nv_bfloat16 v = w.xt[k][src];
-    __syncwarp();
-    if (t < m) w.xt[k][t] = v;
-    __syncwarp();
-  }
-  float g[kMaxRows];
-#pragma unroll
-  for (int q = 0; q < kMaxRows; ++q) g[q] = (q < m && t < m) ? w.G[w.picks[q]][src] : 0.f;
-  __syncwarp();
-  if (t < m)
-#pragma unroll
-    for (int q = 0; q < kMaxRows; ++q)
-      if (q < m) w.G[q][t] = g[q];
+  const int ns = __shfl_sync(0xffffffffu, b.slot, pick);
+  b.slot = t < m ? ns : 0;
+  b.used = __reduce_or_sync(0xffffffffu, t < m ? (1u << ns) : 0u);
+  b.n = m;
   __syncwarp();
 }
 
+// Rows of the buffer, in order, as bf16 rows at dst.
 template <int D>
-__device__ void store_buffer(WarpSmem<D>& w, int n, __nv_bfloat16* dst) {
+__device__ void store_rows(const WarpSmem<D>& w, const Buf& b, __nv_bfloat16* dst) {
   const int lane = threadIdx.x & 31;
-  for (int t = 0; t < n; ++t) {
+  for (int t = 0; t < b.n; ++t) {
+    const int p = __shfl_sync(0xffffffffu, b.slot, t);
     if constexpr (D == 128) {
       const int k = lane * 4;
-      const uint32_t a = __bfloat16_as_ushort(w.xt[k][t]) | (static_cast<uint32_t>(__bfloat16_as_ushort(w.xt[k + 1][t])) << 16);
-      const uint32_t b =
-          __bfloat16_as_ushort(w.xt[k + 2][t]) | (static_cast<uint32_t>(__bfloat16_as_ushort(w.xt[k + 3][t])) << 16);
-      *reinterpret_cast<uint2*>(dst + static_cast<size_t>(t) * D + k) = make_uint2(a, b);
+      const uint32_t x0 = __bfloat16_as_ushort(w.xt[k][p]) | (static_cast<uint32_t>(__bfloat16_as_ushort(w.xt[k + 1][p])) << 16);
+      const uint32_t x1 =
+          __bfloat16_as_ushort(w.xt[k + 2][p]) | (static_cast<uint32_t>(__bfloat16_as_ushort(w.xt[k + 3][p])) << 16);
+      *reinterpret_cast<uint2*>(dst + static_cast<size_t>(t) * D + k) = make_uint2(x0, x1);
     } else {
       const int k = lane * 2;
-      const uint32_t a = __bfloat16_as_ushort(w.xt[k][t]) | (static_cast<uint32_t>(__bfloat16_as_ushort(w.xt[k + 1][t])) << 16);
-      *reinterpret_cast<uint32_t*>(dst + static_cast<size_t>(t) * D + k) = a;
+      const uint32_t x0 = __bfloat16_as_ushort(w.xt[k][p]) | (static_cast<uint32_t>(__bfloat16_as_ushort(w.xt[k + 1][p])) << 16);
+      *reinterpret_cast<uint32_t*>(dst + static_cast<size_t>(t) * D + k) = x0;
     }
   }
 }
@@ -205,95 +234,62 @@ __global__ void __launch_bounds__(32 * kHeadsPerCta) cfps_kernel(CfpsArgs a) {
   __nv_bfloat16* buf = a.buf + static_cast<size_t>(h) * a.b_max * D;
   float* bcn = a.bcn + static_cast<size_t>(h) * a.b_min * D;
   long long* bcnt = a.bcnt + static_cast<size_t>(h) * a.b_min;
-  float v[D / 32];
+  const __nv_bfloat16* qh = a.q ? a.q + static_cast<size_t>(h) * a.n_q * D : nullptr;
+  Buf b{0, 0.f, 0u, 0};
 
   if (a.mode == kCfpsUpdate) {
-    // rows to append, in order: the buffer's own rows (its Gram is rebuilt), then the new queries
+    // rows in order: the buffer's own rows (their cosines are rebuilt), then the new queries
     const int n_old = a.size[h];
     const int total = n_old + a.n_q;
-    const __nv_bfloat16* qn = a.q + static_cast<size_t>(h) * a.n_q * D;
-    int sz = 0, next = 0;
+    int next = 0;
     while (next < total) {
-      const int add = min(a.b_max - sz, total - next);
+      const int add = min(a.b_max - b.n, total - next);
       for (int c0 = 0; c0 < add; c0 += kChunk) {
-        const int cnt = min(kChunk, add - c0);
-        for (int u = 0; u < kChunk; ++u) {
-          const int src = next + c0 + u;
-          if (u < cnt) {
-            load_bf16_row<D>(src < n_old ? buf + static_cast<size_t>(src) * D : qn + static_cast<size_t>(src - n_old) * D,
-                             v);
-          } else {
-#pragma unroll
-            for (int e = 0; e < D / 32; ++e) v[e] = 0.f;
-          }
-          if (u < cnt) {
-            put_row<D>(w, sz + c0 + u, u, v);
-          } else {
-#pragma unroll
-            for (int e = 0; e < D / 32; ++e) w.xn[lane * (D / 32) + e][u] = 0.f;
-          }
-        }
-        gram_add<D>(w, sz + c0, cnt);
+        const int base = next + c0;
+        add_rows<D>(w, b, min(kChunk, add - c0), [&](int u) {
+          const int src = base + u;
+          return RowSrc{src < n_old ? buf + static_cast<size_t>(src) * D : qh + static_cast<size_t>(src - n_old) * D,
+                        false};
+        });
       }
-      sz += add;
       next += add;
-      if (sz == a.b_max) {
-        const int m = fps_rows<D>(w, sz, a.b_min);
-        keep_picks<D>(w, m);
-        sz = m;
-      }
+      if (b.n == a.b_max) fps_keep<D>(w, b, a.b_min);
     }
-    store_buffer<D>(w, sz, buf);
-    if (lane == 0) a.size[h] = sz;
+    store_rows<D>(w, b, buf);
+    if (lane == 0) a.size[h] = b.n;
     return;
   }
 
-  // beacons / merge: gather the candidate rows (at most b_max of them)
-  int n = 0;
+  // beacons: the buffer's rows; merge: this compress's beacons, then the head's window queries
+  int n = 0, nbc = 0;
   if (a.mode == kCfpsBeacons) {
     n = a.size[h];
   } else {
-    int nbc = 0;
     for (int t = 0; t < a.b_min; ++t) nbc += bcnt[t] != 0;
     n = nbc + a.n_q;
   }
-  const __nv_bfloat16* qr = a.q ? a.q + static_cast<size_t>(h) * a.n_q * D : nullptr;
-  const int nbc = n - (a.mode == kCfpsMerge ? a.n_q : 0);
   for (int c0 = 0; c0 < n; c0 += kChunk) {
-    const int cnt = min(kChunk, n - c0);
-    for (int u = 0; u < kChunk; ++u) {
+    add_rows<D>(w, b, min(kChunk, n - c0), [&](int u) {
       const int src = c0 + u;
-      if (u < cnt) {
-        if (a.mode == kCfpsBeacons) {
-          load_bf16_row<D>(buf + static_cast<size_t>(src) * D, v);
-        } else if (src < nbc) {
-          load_f32_row<D>(bcn + static_cast<size_t>(src) * D, v);
-        } else {
-          load_bf16_row<D>(qr + static_cast<size_t>(src - nbc) * D, v);
-        }
-        put_row<D>(w, src, u, v);
-      } else {
-#pragma unroll
-        for (int e = 0; e < D / 32; ++e) w.xn[lane * (D / 32) + e][u] = 0.f;
-      }
-    }
-    gram_add<D>(w, c0, cnt);
+      if (a.mode == kCfpsBeacons) return RowSrc{buf + static_cast<size_t>(src) * D, false};
+      if (src < nbc) return RowSrc{bcn + static_cast<size_t>(src) * D, true};
+      return RowSrc{qh + static_cast<size_t>(src - nbc) * D, false};
+    });
   }
-  const int m = n > 0 ? fps_rows<D>(w, n, a.b_min) : 0;
+  fps_keep<D>(w, b, a.b_min);
   if (a.mode == kCfpsBeacons) {
     for (int t = 0; t < a.b_min; ++t) {
-      const int row = t < m ? w.picks[t] : 0;
+      const int p = __shfl_sync(0xffffffffu, b.slot, t < b.n ? t : 0);
 #pragma unroll
       for (int e = 0; e < D / 32; ++e) {
         const int k = lane * (D / 32) + e;
-        bcn[static_cast<size_t>(t) * D + k] = t < m ? __bfloat162float(w.xt[k][row]) : 0.f;
+        bcn[static_cast<size_t>(t) * D + k] = t < b.n ? __bfloat162float(w.xt[k][p]) : 0.f;
       }
-      if (lane == 0) bcnt[t] = t < m ? 1 : 0;
+      if (lane == 0) bcnt[t] = t < b.n ? 1 : 0;
     }
   } else {
-    keep_picks<D>(w, m);
-    store_buffer<D>(w, m, buf);
-    if (lane == 0) a.size[h] = m;
+    store_rows<D>(w, b, buf);
+    if (lane == 0) a.size[h] = b.n;
   }
 }
 
