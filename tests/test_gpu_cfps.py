@@ -30,7 +30,7 @@ def _heads(t: torch.Tensor, d: int) -> np.ndarray:
     return _bits(t).reshape(-1, t.shape[-2], d)
 
 
-def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None):
+def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False):
     dev = torch.device("cuda")
     inp = synth.step_inputs(wl, seed, dev)
     L = wl.L if L is None else L
@@ -41,7 +41,7 @@ def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None):
     q_new_t = inp["q_new"] if n_new is None else inp["q_new"][..., :n_new, :].contiguous()
     bk = BeaconKV(n_layers=wl.n_layers, batch=wl.batch, n_q_heads=wl.n_q_heads, n_kv_heads=wl.n_kv_heads, head_dim=d,
                   n_beacons=b_min, window=W, capacity=wl.capacity, rope_theta=wl.rope_theta, n_prefix=wl.n_prefix,
-                  continual_fps=True)
+                  continual_fps=True, mean_agg=mean_agg)
     try:
         bk.init_beacons(inp["q_init"])
         buf0, size0 = [x.cpu() for x in bk.cfps_state()]
@@ -90,7 +90,7 @@ def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None):
         hs = slice(e * G, (e + 1) * G)
         r, sw = P.check_cfps_compress(wl, b_min, buf1[hs], size1[hs], q_rec[hs], inp["recent_pos"], inp["t_pos"],
                                       Kb[e], Vb[e], K1[e], V1[e], kept_h[e], s_h[e], L, budget, buf2[hs], size2[hs],
-                                      lib, tag=f"instance {e}")
+                                      lib, tag=f"instance {e}", mean=mean_agg)
         rel_max, swaps = max(rel_max, r), swaps + sw
     print(f"{wl.name}: {n_heads} heads, seed ties {fps_ties}, max score rel err {rel_max:.2e}, swaps {swaps}")
 
@@ -113,3 +113,38 @@ def test_continual_fps_short_call_and_no_eviction():
 def test_continual_fps_ragged_cache():
     wl = QWEN3_4B.scaled(name="cfps_ragged_L1000_B700", n_layers=1, batch=2, L=1000, budget=700)
     _run_cfps(wl, 25, 8)
+
+
+def test_continual_fps_with_mean_aggregation():
+    wl = QWEN3_4B.scaled(name="cfps_mean_1L_b1", n_layers=1, batch=1, L=900, budget=500)
+    _run_cfps(wl, 26, 8, mean_agg=True)
+
+
+def test_continual_fps_state_round_trip():
+    """bkv_set_cfps_state restores buffers that bkv_get_cfps_state saved: an update from the restored
+    state gives the same buffers as from the original."""
+    wl = QWEN3_4B.scaled(name="cfps_state", n_layers=1, batch=1)
+    dev = torch.device("cuda")
+    inp = synth.step_inputs(wl, 27, dev)
+    kw = dict(n_layers=1, batch=1, n_q_heads=wl.n_q_heads, n_kv_heads=wl.n_kv_heads, head_dim=wl.head_dim,
+              n_beacons=8, window=wl.window, capacity=wl.capacity, rope_theta=wl.rope_theta, continual_fps=True)
+    a, b = BeaconKV(**kw), BeaconKV(**kw)
+    try:
+        a.init_beacons(inp["q_init"])
+        a.update(inp["q_new"][..., :37, :].contiguous())
+        buf, sizes = a.cfps_state()
+        b.set_cfps_state(buf, sizes)
+        rest = inp["q_new"][..., 37:, :].contiguous()
+        a.update(rest)
+        b.update(rest)
+        (ba, sa), (bb, sb) = a.cfps_state(), b.cfps_state()
+        torch.cuda.synchronize()
+        assert torch.equal(sa, sb)
+        for h in range(sa.numel()):
+            n = int(sa.view(-1)[h])
+            assert torch.equal(ba.view(-1, ba.shape[-2], ba.shape[-1])[h, :n], bb.view(-1, bb.shape[-2], bb.shape[-1])[h, :n])
+        with pytest.raises(Exception):
+            a.state()      # no centroid state in this mode
+    finally:
+        a.close()
+        b.close()
