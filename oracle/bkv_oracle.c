@@ -19,7 +19,7 @@
  *   One "instance" is one (layer, batch, KV head); its G query heads form the
  *   GQA group.  Group query sets are flattened head-major: row = h * n + i.
  *
- * Readings of points the paper leaves open (each is listed in the design doc):
+ * Readings of points the paper leaves open:
  *   - beacons are kept per KV head and fed by all G query heads of its group;
  *     they are maintained as running-mean centroids seeded by FPS; in the
  *     Continual FPS mode they are instead each query head's fill-and-compress
@@ -29,7 +29,10 @@
  *   - RoPE uses the rotate-half pairing (i, i + d/2) with
  *     inv_freq_i = theta^(-2i/d); theta == 0 disables rotation;
  *   - scoring queries are rounded fp64 -> fp32 -> bf16 (round to nearest even);
- *   - the softmax runs over all L cached keys, with no mask;
+ *   - the softmax runs over all L cached keys, with no mask; an optional causal
+ *     mask inside the recent window takes positions: recent query w sits at
+ *     recent_pos[w], beacons at the current step t, window key j (the last W
+ *     rows) at t - (L - 1 - j), older keys before every window position;
  *   - top-k order is (score descending, index ascending).
  *
  * Parity pins for every function live in tests/test_oracle_*.py.
@@ -467,17 +470,21 @@ int bkvo_build_qobs(const float* cent, const int64_t* counts, int nb, const uint
 /* ------------------------------------------------------------------ */
 
 /*
- * For every valid observation query q and cached key j:
+ * For every valid observation query q and every cached key j visible to it:
  *   logit_qj = (q . k_j) / sqrt(d)
- *   w_qj     = exp(logit_qj) / sum_l exp(logit_ql)      (softmax over all L keys)
+ *   w_qj     = exp(logit_qj) / sum_l exp(logit_ql)      (softmax over the visible keys l)
  * Score[j]   = max over valid q of w_qj            (mean == 0, Eq. 6 max form)
  *            = (1 / #valid) * sum over valid q of w_qj   (mean != 0, Eq. 6 mean form)
+ * Without positions (qpos == NULL) every key is visible to every query: the
+ * softmax runs over all L cached keys (Eq. 4).  With positions, key j is
+ * visible to query q only if kpos[j] <= qpos[q] (causal mask); a masked
+ * weight is 0, and a valid query still counts in #valid.
  * The normaliser is evaluated as lse_q = m_q + log(sum_l exp(logit_ql - m_q)),
  * m_q = max_l logit_ql, so that exp does not overflow.
  * Score[j] = 0 for every j when no query is valid.
  */
-void bkvo_score_agg(const double* qobs, const int32_t* valid, int M, const uint16_t* K, int L, int d, int mean,
-                    double* score) {
+void bkvo_score_mask(const double* qobs, const int32_t* valid, const int64_t* qpos, int M, const uint16_t* K,
+                     const int64_t* kpos, int L, int d, int mean, double* score) {
   double* k = widen_rows(K, L, d);
   double* lg = (double*)malloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
   double inv_sqrt_d = 1.0 / sqrt((double)d);
@@ -488,9 +495,14 @@ void bkvo_score_agg(const double* qobs, const int32_t* valid, int M, const uint1
     ++n_valid;
     double m = -INFINITY;
     for (int j = 0; j < L; ++j) {
+      if (qpos && kpos[j] > qpos[q]) {
+        lg[j] = -INFINITY; /* masked: exp gives 0 below */
+        continue;
+      }
       lg[j] = dot_seq(qobs + (size_t)q * d, k + (size_t)j * d, d) * inv_sqrt_d;
       if (lg[j] > m) m = lg[j];
     }
+    if (m == -INFINITY) continue; /* sees no key: every weight is 0 */
     double s = 0.0;
     for (int j = 0; j < L; ++j) s = s + exp(lg[j] - m);
     double lse = m + log(s);
@@ -506,6 +518,11 @@ void bkvo_score_agg(const double* qobs, const int32_t* valid, int M, const uint1
     for (int j = 0; j < L; ++j) score[j] = score[j] / (double)n_valid;
   free(lg);
   free(k);
+}
+
+void bkvo_score_agg(const double* qobs, const int32_t* valid, int M, const uint16_t* K, int L, int d, int mean,
+                    double* score) {
+  bkvo_score_mask(qobs, valid, NULL, M, K, NULL, L, d, mean, score);
 }
 
 void bkvo_score(const double* qobs, const int32_t* valid, int M, const uint16_t* K, int L, int d,

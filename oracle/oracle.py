@@ -53,6 +53,7 @@ _SIGS = {
     "bkvo_build_qobs": (_I, [_P, _P, _I, _P, _I, _I, _P, _I64, _I, _D, _P, _P]),
     "bkvo_score": (None, [_P, _P, _I, _P, _I, _I, _P]),
     "bkvo_score_agg": (None, [_P, _P, _I, _P, _I, _I, _I, _P]),
+    "bkvo_score_mask": (None, [_P, _P, _P, _I, _P, _P, _I, _I, _I, _P]),
     "bkvo_fps32": (_I, [_P, _I, _I, _I, _P, _P]),
     "bkvo_cfps_update": (_I, [_P, _P, _I, _I, _P, _I, _I, _P, _P, _I]),
     "bkvo_select": (_I, [_P, _I, _I, _I, _I, _P, _P]),
@@ -216,16 +217,38 @@ def build_qobs(cent, counts, q_recent_bits, recent_pos, t_pos: int, theta: float
     return qobs[:m].copy(), valid[:m].copy()
 
 
-def score(qobs: np.ndarray, valid: np.ndarray, k_bits: np.ndarray, lib=None, mean: bool = False) -> np.ndarray:
+def score(qobs: np.ndarray, valid: np.ndarray, k_bits: np.ndarray, lib=None, mean: bool = False,
+          qpos: np.ndarray | None = None, kpos: np.ndarray | None = None) -> np.ndarray:
     """Eq. 4 softmax weights, max (or, with mean=True, mean) over the group's valid queries
-    (Eq. 6, Section 4.3)."""
+    (Eq. 6, Section 4.3).  With positions (qpos per query row, kpos per key), key j enters
+    query q's softmax only if kpos[j] <= qpos[q] (causal mask)."""
     qo = _c(qobs, np.float64)
     va = _c(valid, np.int32)
     k = _c(k_bits, np.uint16)
     L, d = k.shape
     out = np.zeros(max(L, 1), np.float64)
-    (lib or load()).bkvo_score_agg(_p(qo), _p(va), qo.shape[0], _p(k), L, d, int(bool(mean)), _p(out))
+    if qpos is None:
+        (lib or load()).bkvo_score_agg(_p(qo), _p(va), qo.shape[0], _p(k), L, d, int(bool(mean)), _p(out))
+    else:
+        qp = _c(qpos, np.int64)
+        kp = _c(kpos, np.int64)
+        assert qp.shape[0] == qo.shape[0] and kp.shape[0] == L
+        (lib or load()).bkvo_score_mask(_p(qo), _p(va), _p(qp), qo.shape[0], _p(k), _p(kp), L, d, int(bool(mean)),
+                                        _p(out))
     return out[:L].copy()
+
+
+def causal_positions(G: int, W: int, nb: int, recent_pos, t_pos: int, L: int):
+    """Positions for the causal mask inside the recent window (a reading: the paper leaves
+    AttnWeight's mask open).  Q_obs row h*W + w (recent slot w of head h) sits at recent_pos[w],
+    beacon rows at the current step t_pos; window key j (L - W <= j < L) at t_pos - (L - 1 - j);
+    older keys come before every position.  Returns (qpos int64 [G*W + nb], kpos int64 [L])."""
+    rp = np.asarray(recent_pos, np.int64)
+    qpos = np.concatenate([np.tile(rp[:W], G), np.full(nb, int(t_pos), np.int64)])
+    kpos = np.full(L, np.iinfo(np.int64).min, np.int64)
+    w0 = max(L - W, 0)
+    kpos[w0:] = int(t_pos) - (L - 1 - np.arange(w0, L, dtype=np.int64))
+    return qpos, kpos
 
 
 def select(score_: np.ndarray, budget: int, window: int, n_prefix: int, lib=None):

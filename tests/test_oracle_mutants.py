@@ -26,6 +26,8 @@ _SCORE = [(TS.test_score_matches_scipy_softmax_max, dict(M=3, L=50, d=8)),
           (TS.test_score_single_query_sums_to_one_and_ranks_by_dot, {})]
 _MEAN = [(TS.test_score_mean_matches_scipy_softmax_mean, dict(M=4, L=77, d=8)),
          (TS.test_score_mean_closed_forms_and_bounds, {}), (TS.test_score_mean_duplicated_query_weights, {})]
+_CAUSAL = [(TS.test_score_causal_matches_scipy_softmax_over_visible_keys, dict(mean=False, M=6, L=40, d=8)),
+           (TS.test_score_causal_closed_forms, {})]
 _ROPE = [(TN.test_rope_is_complex_rotation_of_rotate_half_pairs, {}),
          (TN.test_rope_preserves_norm_and_relative_position, {})]
 _FPS = [(TB.test_fps_matches_maxmin_brute_force, dict(seed=s)) for s in range(6)] + [
@@ -45,6 +47,10 @@ MUTANTS = [
     ("mean_over_all_rows", "score[j] = score[j] / (double)n_valid;", "score[j] = score[j] / (double)M;", _MEAN),
     ("mean_takes_max", "      if (mean)\n        score[j] = score[j] + w;", "      if (mean && w > score[j])\n        score[j] = w;",
      _MEAN),
+    ("causal_mask_inverted", "if (qpos && kpos[j] > qpos[q]) {", "if (qpos && kpos[j] < qpos[q]) {", _CAUSAL),
+    ("causal_mask_hides_own_position", "if (qpos && kpos[j] > qpos[q]) {", "if (qpos && kpos[j] >= qpos[q]) {", _CAUSAL),
+    ("causal_mask_ignored", "lg[j] = -INFINITY; /* masked: exp gives 0 below */\n        continue;",
+     "lg[j] = -INFINITY; /* masked: exp gives 0 below */", _CAUSAL),
     ("rope_sign", "y[i] = x1 * cs - x2 * sn;", "y[i] = x1 * cs + x2 * sn;", _ROPE),
     ("rope_interleaved_pairs", "double x1 = x[i], x2 = x[i + h];", "double x1 = x[2 * i], x2 = x[2 * i + 1];",
      _ROPE),

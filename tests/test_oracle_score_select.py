@@ -4,7 +4,7 @@ the keep set of Algorithm 2) and compaction (Eq. 8).
 Independent routes: scipy.special.softmax, numpy lexsort, numpy fancy indexing,
 closed forms (identical keys, a single query, two-key logistic), invariants
 (window kept, exact budget, ordering, key-shift invariance, duplicated and
-invalid queries) and a hand-computed worked case stored under tests/golden/.
+invalid queries, causal masks with nothing masked) and a hand-computed worked case stored under tests/golden/.
 """
 import json
 import math
@@ -144,6 +144,60 @@ def test_score_mean_duplicated_query_weights(olib):
     w = softmax(q @ O.bf16_to_f64(k).T / math.sqrt(8), axis=1)
     got = O.score(np.vstack([q, q[:1]]), np.ones(3, np.int32), k, olib, mean=True)
     np.testing.assert_allclose(got, (2 * w[0] + w[1]) / 3, rtol=1e-12)
+
+
+# ------------------------------------------------------------------ causal mask inside the window
+@pytest.mark.parametrize("mean", [False, True])
+@pytest.mark.parametrize("M,L,d", [(6, 40, 8), (9, 130, 16)])
+def test_score_causal_matches_scipy_softmax_over_visible_keys(olib, mean, M, L, d):
+    """Each valid query's softmax runs over the keys at or before its position only (scipy over
+    the visible logits); masked weights are 0 and still count in the mean."""
+    rng = np.random.default_rng(11 * M + L + mean)
+    q, k = _rand_case(rng, M, L, d)
+    valid = np.ones(M, np.int32)
+    valid[1] = 0
+    kpos = np.sort(rng.integers(0, 3 * L, L)).astype(np.int64)
+    qpos = rng.integers(kpos[0], kpos[-1] + 2, M).astype(np.int64)
+    got = O.score(q, valid, k, olib, mean=mean, qpos=qpos, kpos=kpos)
+    lg = q @ O.bf16_to_f64(k).T / math.sqrt(d)
+    w = np.zeros((M, L))
+    for i in range(M):
+        vis = kpos <= qpos[i]
+        if vis.any():
+            w[i, vis] = softmax(lg[i, vis])
+    rows = w[valid.astype(bool)]
+    want = rows.mean(axis=0) if mean else rows.max(axis=0)
+    np.testing.assert_allclose(got, want, rtol=1e-12, atol=0)
+
+
+def test_score_causal_closed_forms(olib):
+    """Keys at positions 0, 1, 2.  A query at position 0 sees only key 0 (weight 1); a zero query at
+    position 2 sees all three (weights 1/3).  Max: [1, 1/3, 1/3]; mean: [2/3, 1/6, 1/6]."""
+    d = 8
+    q = np.zeros((2, d))
+    q[0] = O.bf16_to_f64(_bits(np.linspace(-2.0, 3.0, d)))
+    k = _bits(np.random.default_rng(3).standard_normal((3, d)))
+    qpos, kpos = np.array([0, 2], np.int64), np.array([0, 1, 2], np.int64)
+    v = np.ones(2, np.int32)
+    np.testing.assert_allclose(O.score(q, v, k, olib, qpos=qpos, kpos=kpos), [1.0, 1 / 3, 1 / 3], rtol=1e-14)
+    np.testing.assert_allclose(O.score(q, v, k, olib, mean=True, qpos=qpos, kpos=kpos), [2 / 3, 1 / 6, 1 / 6],
+                               rtol=1e-14)
+
+
+def test_score_causal_without_masked_pairs_is_unmasked_and_positions_follow_the_window(olib):
+    """Every query at or after every key: bit-equal to the unmasked score.  causal_positions puts recent
+    slot w at recent_pos[w], beacons at t and window key j at t - (L - 1 - j)."""
+    rng = np.random.default_rng(5)
+    q, k = _rand_case(rng, 7, 90, 16)
+    v = np.ones(7, np.int32)
+    kpos = np.arange(90, dtype=np.int64)
+    qpos = np.full(7, 89, np.int64) + rng.integers(0, 3, 7)
+    for mean in (False, True):
+        np.testing.assert_array_equal(O.score(q, v, k, olib, mean=mean, qpos=qpos, kpos=kpos),
+                                      O.score(q, v, k, olib, mean=mean))
+    qp, kp = O.causal_positions(G=2, W=3, nb=1, recent_pos=[97, 98, 99], t_pos=99, L=10)
+    np.testing.assert_array_equal(qp, [97, 98, 99, 97, 98, 99, 99])
+    assert np.all(kp[:7] < 0) and list(kp[7:]) == [97, 98, 99]
 
 
 # ------------------------------------------------------------------ select
