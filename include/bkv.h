@@ -93,6 +93,19 @@ extern "C" {
  * G * (n_beacons + window) <= 128.  The centroid state functions do not apply.
  */
 #define BKV_F_CONTINUAL_FPS 2u
+/*
+ * Causal mask inside the recent window (AttnWeight's mask, which the paper
+ * leaves open; Algorithm 2, Section 4.3).  Positions: recent slot w sits at
+ * recent_pos[w], beacons at t_pos, and the last `window` cache rows j
+ * (L - window <= j < L) at t_pos - (L - 1 - j); older rows come before every
+ * window position.  A recent query then takes no part in the softmax of the
+ * window rows after its own position: those rows are left out of its
+ * normaliser and its weight on them is 0 (it still counts in the mean of
+ * BKV_F_MEAN_AGG).  Beacons and older rows are never masked.  Selection, the
+ * keep set and compaction are unchanged.  Applies to bkv_compress and
+ * bkv_compress_static; no effect when window = 0.
+ */
+#define BKV_F_CAUSAL_WINDOW 4u
 
 typedef struct bkv_ctx bkv_ctx;
 
@@ -264,7 +277,9 @@ int bkv_profile_read(bkv_ctx* ctx, double* ms, int64_t* launches, int32_t n_kern
  * takes everything from the caller: the shape (cfg, same limits as
  * bkv_create), the beacon state (centroids fp32 [n_inst][n_beacons][d] and
  * counts int64 [n_inst][n_beacons], device; may be NULL when n_beacons = 0)
- * and the stream.  It needs no context and allocates or frees nothing.  Its
+ * and the stream; cfg->flags may hold BKV_F_MEAN_AGG and BKV_F_CAUSAL_WINDOW
+ * (the Continual FPS mode needs a context and is rejected here).  It needs no
+ * context and allocates or frees nothing.  Its
  * scratch is one library-owned device array of 16 MiB (resident on every
  * device that loads the library until the process exits); a call whose
  * scratch exceeds it - n_inst * (4 * capacity + 2 * n_obs_pad * head_dim +

@@ -30,6 +30,7 @@ KERNEL_NAMES = ("fps_init", "update", "qobs", "score", "select_gather", "keep_al
 BKV_F_NONE = 0
 BKV_F_MEAN_AGG = 1
 BKV_F_CONTINUAL_FPS = 2
+BKV_F_CAUSAL_WINDOW = 4
 
 
 class BkvConfig(ctypes.Structure):
@@ -251,19 +252,21 @@ class BeaconKV:
     """
 
     def __init__(self, *, n_layers, batch, n_q_heads, n_kv_heads, head_dim, n_beacons, window, capacity,
-                 rope_theta=0.0, n_prefix=0, stream=None, mean_agg=False, continual_fps=False):
-        flags = (BKV_F_MEAN_AGG if mean_agg else BKV_F_NONE) | (BKV_F_CONTINUAL_FPS if continual_fps else BKV_F_NONE)
+                 rope_theta=0.0, n_prefix=0, stream=None, mean_agg=False, continual_fps=False, causal_window=False):
+        flags = ((BKV_F_MEAN_AGG if mean_agg else BKV_F_NONE) | (BKV_F_CONTINUAL_FPS if continual_fps else BKV_F_NONE)
+                 | (BKV_F_CAUSAL_WINDOW if causal_window else BKV_F_NONE))
         self.cfg = BkvConfig(n_layers, batch, n_q_heads, n_kv_heads, head_dim, n_beacons, window, n_prefix,
                              capacity, float(rope_theta), flags)
         self.ctx = bkv_create(self.cfg, stream)
         self.n_inst = n_layers * batch * n_kv_heads
 
     @classmethod
-    def for_workload(cls, wl, stream=None, capacity=None, mean_agg=False, continual_fps=False) -> "BeaconKV":
+    def for_workload(cls, wl, stream=None, capacity=None, mean_agg=False, continual_fps=False,
+                     causal_window=False) -> "BeaconKV":
         return cls(n_layers=wl.n_layers, batch=wl.batch, n_q_heads=wl.n_q_heads, n_kv_heads=wl.n_kv_heads,
                    head_dim=wl.head_dim, n_beacons=wl.n_beacons, window=wl.window,
                    capacity=capacity or wl.capacity, rope_theta=wl.rope_theta, n_prefix=wl.n_prefix, stream=stream,
-                   mean_agg=mean_agg, continual_fps=continual_fps)
+                   mean_agg=mean_agg, continual_fps=continual_fps, causal_window=causal_window)
 
     def close(self):
         if self.ctx:

@@ -158,7 +158,8 @@ int validate_config(const bkv_config* cfg, std::string& why) {
   if (cfg->n_prefix < 0) return bad("n_prefix must be >= 0");
   if (cfg->capacity < 1 || cfg->capacity > bkv::kMaxCapacity) return bad("capacity must be in 1..32768");
   if (!(cfg->rope_theta >= 0.0) || !std::isfinite(cfg->rope_theta)) return bad("rope_theta must be finite and >= 0");
-  if (cfg->flags & ~(BKV_F_MEAN_AGG | BKV_F_CONTINUAL_FPS)) return bad("flags holds an unknown option");
+  if (cfg->flags & ~(BKV_F_MEAN_AGG | BKV_F_CONTINUAL_FPS | BKV_F_CAUSAL_WINDOW))
+    return bad("flags holds an unknown option");
   const long long G = cfg->n_q_heads / cfg->n_kv_heads;
   const bool cfps = (cfg->flags & BKV_F_CONTINUAL_FPS) != 0;
   if (cfps && (cfg->n_beacons < 1 || cfg->window < 1 || cfg->n_beacons + cfg->window > bkv::kCfpsMaxRows))
@@ -461,6 +462,7 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
   sa.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(s.d)));
   sa.valid = ctx->valid;
   sa.mean = (ctx->cfg.flags & BKV_F_MEAN_AGG) != 0;
+  if (ctx->cfg.flags & BKV_F_CAUSAL_WINDOW) bkv::set_causal(sa, L, s.W, t_pos, recent_pos);
   sa.r_out = ctx->rscore;
   sa.scores_out = scores_out;
   sa.err = ctx->err;

@@ -65,22 +65,45 @@ cudaError_t launch_qobs(const Shape& s, const __nv_bfloat16* q_recent, const flo
                         const double2* rope, int rotate, __nv_bfloat16* qobs, uint32_t* valid, cudaStream_t st);
 
 struct ScoreArgs {
-  int L;
-  float scale_log2;        // log2(e) / sqrt(d)
-  const uint32_t* valid;   // [n_inst][4] bitmask of valid scoring rows
-  bool mean;               // mean over the valid queries instead of the maximum
-  float* r_out;            // [n_inst][cap] log2-domain scores (log2 of the aggregated weight)
-  float* scores_out;       // [n_inst][cap] probabilities, or nullptr
-  int* err;                // device error word
+  int L = 0;
+  float scale_log2 = 0.f;          // log2(e) / sqrt(d)
+  const uint32_t* valid = nullptr; // [n_inst][4] bitmask of valid scoring rows
+  bool mean = false;               // mean over the valid queries instead of the maximum
+  bool causal = false;             // causal mask inside the recent window (set_causal)
+  int win0 = 0;                    // first window row, L - W
+  int thr[kMaxWindow] = {};        // recent slot w sees window row j only if j <= thr[w]
+  float* r_out = nullptr;          // [n_inst][cap] log2-domain scores (log2 of the aggregated weight)
+  float* scores_out = nullptr;     // [n_inst][cap] probabilities, or nullptr
+  int* err = nullptr;              // device error word
 };
+// Causal mask inside the recent window: recent slot w sits at recent_pos[w] and window row j
+// (L - W <= j < L) at t_pos - (L - 1 - j), so slot w sees window row j only if
+// j <= L - 1 - (t_pos - recent_pos[w]); beacons (at t_pos) and older rows are never masked.
+inline void set_causal(ScoreArgs& a, int L, int W, long long t_pos, const int64_t* recent_pos) {
+  a.causal = W > 0;
+  a.win0 = L - W;
+  for (int w = 0; w < W; ++w) {
+    if (recent_pos[w] >= t_pos) {
+      a.thr[w] = L;  // at or after every window row
+    } else {
+      const unsigned long long gap = static_cast<unsigned long long>(t_pos) - static_cast<unsigned long long>(recent_pos[w]);
+      a.thr[w] = gap > static_cast<unsigned long long>(L) ? -1 : (L - 1) - static_cast<int>(gap);
+    }
+  }
+}
 // kmap / kmap32: K as [n_inst * cap][d] in 128-row and 32-row boxes of [64]
 // columns (128-byte swizzle); qmap: Qobs as [n_inst * n_obs_pad][d] in boxes
 // of n_obs_pad rows.
 cudaError_t launch_score(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32, const CUtensorMap& qmap,
                          const ScoreArgs& a, cudaStream_t st);
-// The mean form (a.mean), compiled in its own translation unit; launch_score forwards to it.
+// The mean form (a.mean) and the causal forms (a.causal), each compiled in its own translation
+// unit; launch_score forwards to them.
 cudaError_t launch_score_mean(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32,
                               const CUtensorMap& qmap, const ScoreArgs& a, cudaStream_t st);
+cudaError_t launch_score_causal(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32,
+                                const CUtensorMap& qmap, const ScoreArgs& a, cudaStream_t st);
+cudaError_t launch_score_causal_mean(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32,
+                                     const CUtensorMap& qmap, const ScoreArgs& a, cudaStream_t st);
 
 cudaError_t launch_select_gather(const Shape& s, const float* r, int L, int budget, __nv_bfloat16* K,
                                  __nv_bfloat16* V, int* kept, cudaStream_t st);

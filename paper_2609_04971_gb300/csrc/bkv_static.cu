@@ -116,7 +116,7 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
   if (cfg->n_beacons < 0 || cfg->n_beacons > bkv::kMaxBeacons) return bad("n_beacons must be in 0..32");
   if (cfg->window < 0 || cfg->window > bkv::kMaxWindow) return bad("window must be in 0..64");
   if (cfg->n_prefix < 0) return bad("n_prefix must be >= 0");
-  if (cfg->flags & ~BKV_F_MEAN_AGG) return bad("flags holds an unknown option");
+  if (cfg->flags & ~(BKV_F_MEAN_AGG | BKV_F_CAUSAL_WINDOW)) return bad("flags holds an unknown option");
   if (cfg->capacity < 1 || cfg->capacity > bkv::kMaxCapacity) return bad("capacity must be in 1..32768");
   if (!(cfg->rope_theta >= 0.0) || !std::isfinite(cfg->rope_theta)) return bad("rope_theta must be finite, >= 0");
   bkv::Shape s{};
@@ -221,6 +221,7 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
     sa.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(s.d)));
     sa.valid = valid;
     sa.mean = (cfg->flags & BKV_F_MEAN_AGG) != 0;
+    if (cfg->flags & BKV_F_CAUSAL_WINDOW) bkv::set_causal(sa, L, s.W, t_pos, recent_pos);
     sa.r_out = rscore;
     sa.scores_out = scores_out;
     sa.err = reinterpret_cast<int*>(dev_status);

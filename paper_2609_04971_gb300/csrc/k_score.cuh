@@ -51,8 +51,16 @@
 // barrier, so no CTA leaves while a peer may still write to its shared memory.
 // Outputs: r (log2 scores, for selection) and optionally 2^r.
 //
+// Causal form (CAUSAL): recent slot w must not see window rows after its own
+// position (row j >= L - W is masked for it when j > thr[w]); beacons and
+// older rows are never masked.  Only tiles that hold window rows take the
+// masked paths: pass 1 skips the masked (row, column) terms of the
+// statistics, pass 2 leaves them out of the maximum or the mean (a masked
+// weight is 0 and still counts in the mean's query count).
+//
 // This header holds the kernel template; k_score.cu instantiates the max
-// form and k_score_mean.cu the mean form, so that they compile in parallel.
+// form, k_score_mean.cu the mean form and k_score_causal*.cu their causal
+// forms, so that they compile in parallel.
 #pragma once
 #include "bkv_device.cuh"
 #include "bkv_internal.h"
@@ -242,7 +250,43 @@ __device__ __forceinline__ float tile_agg(uint32_t taddr, const float* lse2, flo
   }
 }
 
-template <int D, int NQ, bool MEAN>
+// tile_agg for a tile that holds window rows: column c is left out for key
+// `key` when key >= win0 and key > thr[c].
+template <int N, bool MEAN>
+__device__ __forceinline__ float tile_agg_causal(uint32_t taddr, const float* lse2, float sc, float inv_m, int key,
+                                                 int win0, const int* thr) {
+  const bool in_win = key >= win0;
+  float r = -INFINITY, sum = 0.f;
+#pragma unroll
+  for (int c0 = 0; c0 < N; c0 += 32) {
+    float v[32];
+    if (c0 + 32 <= N) {
+      tmem_ld32(taddr + c0, v);
+    } else {
+      tmem_ld16(taddr + c0, v);
+    }
+    tmem_wait_ld();
+#pragma unroll
+    for (int u = 0; u < 32; ++u) {
+      const int c = c0 + u;
+      if (c < N && !(in_win && key > thr[c])) {
+        const float x = fmaf(v[u], sc, -lse2[c]);
+        if constexpr (MEAN) {
+          sum += ex2_approx(x);
+        } else {
+          r = fmaxf(r, x);
+        }
+      }
+    }
+  }
+  if constexpr (MEAN) {
+    return lg2_approx(sum * inv_m);
+  } else {
+    return r;
+  }
+}
+
+template <int D, int NQ, bool MEAN, bool CAUSAL>
 __global__ void __launch_bounds__(kScThreads, 1)
     score_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap kmap32,
                  const __grid_constant__ CUtensorMap qmap, Shape s, ScoreArgs a, Plan plan, int n_stages) {
@@ -258,6 +302,7 @@ __global__ void __launch_bounds__(kScThreads, 1)
   __shared__ int abort_sh;
   __shared__ __align__(16) float lse2_sh[128];
   __shared__ int vcount_sh[4];  // valid queries per 32-column group of the instance (mean aggregation)
+  __shared__ int thr_sh[CAUSAL ? 128 : 1];  // causal form: last visible window row of each column
   __shared__ float wred_m[kEpiWarps][64], wred_s[kEpiWarps][64];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -301,6 +346,12 @@ __global__ void __launch_bounds__(kScThreads, 1)
     mbar_init(&recv_bar[1], 1);
     abort_sh = 0;
     fence_mbar_init();
+  }
+  if constexpr (CAUSAL) {
+    if (threadIdx.x < 128) {
+      const int c = threadIdx.x;  // recent slot c % W of head c / W, or a beacon / padding column
+      thr_sh[c] = c < s.G * s.W ? a.thr[c % s.W] : 0x7fffffff;
+    }
   }
   if (warp == 1) {
     tmem_alloc(&tmem_base_sh, kTmemCols);
@@ -493,8 +544,27 @@ __global__ void __launch_bounds__(kScThreads, 1)
         // Running sums relative to a reference m that moves only when a base-2
         // logit exceeds it by more than 64, so the terms stay below 2^64 and
         // the common step is one FFMA, one ex2 and one add per column.
-        if (have) {
-          const bool key_ok = k0 + j * kTile + key_row < k1;
+        const int tile0 = k0 + j * kTile;
+        if (have && CAUSAL && tile0 + kTile > a.win0) {
+          // a tile with window rows: the careful path, without the masked (row, column) terms
+          const int key = tile0 + key_row;
+          if (key < k1) {
+            const bool in_win = key >= a.win0;
+#pragma unroll
+            for (int c = 0; c < NQ; ++c) {
+              if (in_win && key > thr_sh[half * NQ + c]) continue;
+              const float t = fmaf(v[c], sc, -m[c]);
+              if (t > 64.f) {
+                const float y = v[c] * sc;
+                sm[c] = fmaf(sm[c], ex2_approx(m[c] - y), 1.f);
+                m[c] = y;
+              } else {
+                sm[c] += ex2_approx(t);
+              }
+            }
+          }
+        } else if (have) {
+          const bool key_ok = tile0 + key_row < k1;
           float t[NQ];
           bool rebase = !__all_sync(0xffffffffu, key_ok);  // a ragged tile takes the careful path
 #pragma unroll
@@ -574,11 +644,14 @@ __global__ void __launch_bounds__(kScThreads, 1)
       for (int j = half; j < R; j += 2) {
         const int slot = rs + j < ring ? rs + j : rs + j - ring;
         float r = -INFINITY;
-        if (resident_ok) r = tile_agg<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m);
+        const int key = k0 + j * kTile + key_row;
+        if (resident_ok)
+          r = (CAUSAL && k0 + j * kTile + kTile > a.win0)
+                  ? tile_agg_causal<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m, key, a.win0, thr_sh)
+                  : tile_agg<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_cnt(&slot_free[slot], 2);  // two arrivals: this warp stands for its pair
-        const int key = k0 + j * kTile + key_row;
         if (resident_ok && key < k1) {
           r_e[key] = r;
           if (s_e) s_e[key] = ex2_approx(r);
@@ -590,14 +663,16 @@ __global__ void __launch_bounds__(kScThreads, 1)
         bool have = !*abort_flag && mbar_wait(&slot_full[slot], u & 1, abort_flag, a.err, kDevTimeoutEpilogue);
         have = __all_sync(0xffffffffu, have);
         float r = -INFINITY;
+        const int key = k0 + j * kTile + key_row;
         if (have) {
           tc_fence_after();
-          r = tile_agg<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m);
+          r = (CAUSAL && k0 + j * kTile + kTile > a.win0)
+                  ? tile_agg_causal<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m, key, a.win0, thr_sh)
+                  : tile_agg<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m);
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_cnt(&slot_free[slot], 2);
-        const int key = k0 + j * kTile + key_row;
         if (have && key < k1) {
           r_e[key] = r;
           if (s_e) s_e[key] = ex2_approx(r);
@@ -640,14 +715,14 @@ Plan plan_score(int L, int n_obs_pad) {
   return Plan{cmax, cap - 4, 1};
 }
 
-template <int D, int NQ, bool MEAN>
+template <int D, int NQ, bool MEAN, bool CAUSAL>
 cudaError_t launch_score_dq(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32,
                             const CUtensorMap& qmap, const ScoreArgs& a, cudaStream_t st) {
   using C = ScoreCfg<D>;
   const Plan plan = plan_score(a.L, s.n_obs_pad);
   const size_t smem = C::smem_bytes(s.n_obs_pad, plan.csize);
   const int n_stages = C::stages(s.n_obs_pad, plan.csize);
-  cudaError_t err = cudaFuncSetAttribute(score_kernel<D, NQ, MEAN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t err = cudaFuncSetAttribute(score_kernel<D, NQ, MEAN, CAUSAL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
   if (err != cudaSuccess) return err;
   int dev = 0, sms = 0, max_clusters = 0;
@@ -666,37 +741,37 @@ cudaError_t launch_score_dq(const Shape& s, const CUtensorMap& kmap, const CUten
   cfg.numAttrs = 1;
   // one resident wave of clusters, each looping over its share of the instances
   cfg.gridDim = dim3(static_cast<unsigned>(plan.csize * sms));
-  if (cudaOccupancyMaxActiveClusters(&max_clusters, score_kernel<D, NQ, MEAN>, &cfg) != cudaSuccess || max_clusters < 1) {
+  if (cudaOccupancyMaxActiveClusters(&max_clusters, score_kernel<D, NQ, MEAN, CAUSAL>, &cfg) != cudaSuccess || max_clusters < 1) {
     cudaGetLastError();
     max_clusters = sms / plan.csize > 0 ? sms / plan.csize : 1;
   }
   const int n_clusters = max_clusters < s.n_inst ? max_clusters : s.n_inst;
   cfg.gridDim = dim3(static_cast<unsigned>(n_clusters * plan.csize));
-  return cudaLaunchKernelEx(&cfg, score_kernel<D, NQ, MEAN>, kmap, kmap32, qmap, s, a, plan, n_stages);
+  return cudaLaunchKernelEx(&cfg, score_kernel<D, NQ, MEAN, CAUSAL>, kmap, kmap32, qmap, s, a, plan, n_stages);
 }
 
-template <int D, bool MEAN>
+template <int D, bool MEAN, bool CAUSAL>
 cudaError_t launch_score_d(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32, const CUtensorMap& qmap,
                            const ScoreArgs& a, cudaStream_t st) {
   // query columns of each pass-1 warp: half of the padded query count
   switch (s.n_obs_pad) {
-    case 16: return launch_score_dq<D, 8, MEAN>(s, kmap, kmap32, qmap, a, st);
-    case 32: return launch_score_dq<D, 16, MEAN>(s, kmap, kmap32, qmap, a, st);
-    case 48: return launch_score_dq<D, 24, MEAN>(s, kmap, kmap32, qmap, a, st);
-    case 64: return launch_score_dq<D, 32, MEAN>(s, kmap, kmap32, qmap, a, st);
-    case 80: return launch_score_dq<D, 40, MEAN>(s, kmap, kmap32, qmap, a, st);
-    case 96: return launch_score_dq<D, 48, MEAN>(s, kmap, kmap32, qmap, a, st);
-    case 112: return launch_score_dq<D, 56, MEAN>(s, kmap, kmap32, qmap, a, st);
-    default: return launch_score_dq<D, 64, MEAN>(s, kmap, kmap32, qmap, a, st);
+    case 16: return launch_score_dq<D, 8, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
+    case 32: return launch_score_dq<D, 16, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
+    case 48: return launch_score_dq<D, 24, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
+    case 64: return launch_score_dq<D, 32, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
+    case 80: return launch_score_dq<D, 40, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
+    case 96: return launch_score_dq<D, 48, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
+    case 112: return launch_score_dq<D, 56, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
+    default: return launch_score_dq<D, 64, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
   }
 }
 
-// Dispatch on head_dim and the padded query count for one aggregation.
-template <bool MEAN>
+// Dispatch on head_dim and the padded query count for one aggregation and mask.
+template <bool MEAN, bool CAUSAL>
 cudaError_t launch_score_agg(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32,
                              const CUtensorMap& qmap, const ScoreArgs& a, cudaStream_t st) {
-  return s.d == 128 ? launch_score_d<128, MEAN>(s, kmap, kmap32, qmap, a, st)
-                    : launch_score_d<64, MEAN>(s, kmap, kmap32, qmap, a, st);
+  return s.d == 128 ? launch_score_d<128, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st)
+                    : launch_score_d<64, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
 }
 
 }  // namespace

@@ -5,7 +5,7 @@ namespace bkv {
 
 cudaError_t launch_score_mean(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32,
                               const CUtensorMap& qmap, const ScoreArgs& a, cudaStream_t st) {
-  return launch_score_agg<true>(s, kmap, kmap32, qmap, a, st);
+  return launch_score_agg<true, false>(s, kmap, kmap32, qmap, a, st);
 }
 
 }  // namespace bkv

@@ -51,6 +51,7 @@ class GpuRun:
     V_after: np.ndarray
     sample: np.ndarray     # instance ids copied to the host
     mean_agg: bool = False  # Eq. 6 mean form instead of the max
+    causal: bool = False    # causal mask inside the recent window
 
 
 def _inst_rows(t: torch.Tensor, wl: Workload) -> torch.Tensor:
@@ -60,7 +61,7 @@ def _inst_rows(t: torch.Tensor, wl: Workload) -> torch.Tensor:
 
 
 def run_gpu(wl: Workload, seed: int = 0, sample=None, with_scores: bool = True, inputs: dict | None = None,
-            L: int | None = None, budget: int | None = None, mean_agg: bool = False) -> GpuRun:
+            L: int | None = None, budget: int | None = None, mean_agg: bool = False, causal: bool = False) -> GpuRun:
     dev = torch.device("cuda")
     inp = inputs or synth.step_inputs(wl, seed, dev)
     L = wl.L if L is None else L
@@ -69,7 +70,7 @@ def run_gpu(wl: Workload, seed: int = 0, sample=None, with_scores: bool = True, 
     sample = np.arange(n_inst) if sample is None else np.asarray(sample)
     sidx = torch.as_tensor(sample, device=dev)
 
-    bk = BeaconKV.for_workload(wl, mean_agg=mean_agg)
+    bk = BeaconKV.for_workload(wl, mean_agg=mean_agg, causal_window=causal)
     try:
         bk.init_beacons(inp["q_init"])
         c0, s0, n0 = [x.cpu().numpy() for x in bk.state()]
@@ -95,7 +96,7 @@ def run_gpu(wl: Workload, seed: int = 0, sample=None, with_scores: bool = True, 
                   kept=kept.view(n_inst, -1).cpu().numpy(),
                   scores=None if scores is None else scores.view(n_inst, -1).cpu().numpy(),
                   K_before=K_before, V_before=V_before, K_after=K_after, V_after=V_after, sample=sample,
-                  mean_agg=mean_agg)
+                  mean_agg=mean_agg, causal=causal)
 
 
 @dataclasses.dataclass
@@ -161,7 +162,7 @@ def check_instance(run: GpuRun, k: int, L: int | None = None, budget: int | None
     rel, swaps = check_compress(wl, run.cent1[e], run.counts1[e], q_recent, inp["recent_pos"], inp["t_pos"],
                                 run.K_before[k], run.V_before[k], run.K_after[k], run.V_after[k], run.kept[e],
                                 None if run.scores is None else run.scores[e], L, budget, lib, tag=f"instance {e}",
-                                mean=run.mean_agg)
+                                mean=run.mean_agg, causal=run.causal)
     rep.max_score_rel = rel
     rep.boundary_swaps += swaps
     return rep
@@ -202,10 +203,12 @@ def check_update(q_new: np.ndarray, pre: dict, assign_g: np.ndarray, post: dict,
 
 def check_compress(wl: Workload, cent: np.ndarray, counts: np.ndarray, q_recent: np.ndarray, recent_pos, t_pos: int,
                    K0: np.ndarray, V0: np.ndarray, K1: np.ndarray, V1: np.ndarray, kept_g: np.ndarray,
-                   scores_g: np.ndarray | None, L: int, budget: int, lib, tag: str = "", mean: bool = False) -> tuple:
+                   scores_g: np.ndarray | None, L: int, budget: int, lib, tag: str = "", mean: bool = False,
+                   causal: bool = False) -> tuple:
     """One compress of one instance on the beacon state (cent, counts): scores within 1e-3, the kept set
     equal up to boundary ties, K / V rows byte-equal to the kept pre-compress rows.  K0 / V0 and K1 / V1
-    are the instance's uint16 rows before and after.  Returns (max score rel err, boundary swaps)."""
+    are the instance's uint16 rows before and after; `causal` applies the mask inside the recent window.
+    Returns (max score rel err, boundary swaps)."""
     W = wl.window
     if L <= budget:
         np.testing.assert_array_equal(kept_g[:L], np.arange(L))
@@ -213,7 +216,11 @@ def check_compress(wl: Workload, cent: np.ndarray, counts: np.ndarray, q_recent:
         np.testing.assert_array_equal(K1, K0)
         return 0.0, 0
     qobs, valid = O.build_qobs(cent, counts, q_recent, np.asarray(recent_pos, np.int64), t_pos, wl.rope_theta, lib)
-    s_o = O.score(qobs, valid, K0[:L], lib, mean=mean)
+    if causal and W > 0:
+        qpos, kpos = O.causal_positions(q_recent.shape[0], W, counts.shape[0], recent_pos, t_pos, L)
+        s_o = O.score(qobs, valid, K0[:L], lib, mean=mean, qpos=qpos, kpos=kpos)
+    else:
+        s_o = O.score(qobs, valid, K0[:L], lib, mean=mean)
     rel_max = 0.0
     if scores_g is not None:
         s_g = scores_g[:L].astype(np.float64)
@@ -242,7 +249,7 @@ def check_compress(wl: Workload, cent: np.ndarray, counts: np.ndarray, q_recent:
 
 def check_cfps_compress(wl: Workload, b_min: int, buf: np.ndarray, size: np.ndarray, q_rec: np.ndarray, recent_pos,
                         t_pos: int, K0, V0, K1, V1, kept_g, scores_g, L: int, budget: int, buf_after: np.ndarray,
-                        size_after: np.ndarray, lib, tag: str = "", mean: bool = False) -> tuple:
+                        size_after: np.ndarray, lib, tag: str = "", mean: bool = False, causal: bool = False) -> tuple:
     """One compress of one instance in the Continual FPS mode.  buf / size: the G buffers of the
     instance's query heads before the compress (uint16 [G, b_max, d], int [G]); q_rec: their window
     queries (uint16 [G, W, d]); buf_after / size_after: the GPU's buffers after it.  The beacons are
@@ -260,7 +267,7 @@ def check_cfps_compress(wl: Workload, b_min: int, buf: np.ndarray, size: np.ndar
         cent[g * b_min:g * b_min + len(picks)] = O.bf16_to_f64(rows)
         counts[g * b_min:g * b_min + len(picks)] = 1
     rel, swaps = check_compress(wl, cent, counts, q_rec, recent_pos, t_pos, K0, V0, K1, V1, kept_g, scores_g, L,
-                                budget, lib, tag=tag, mean=mean)
+                                budget, lib, tag=tag, mean=mean, causal=causal)
     for g in range(G):
         if L > budget:
             cand = np.vstack([beacons[g], q_rec[g]])

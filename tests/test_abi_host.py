@@ -53,7 +53,7 @@ def test_strerror_and_version(lib):
 
 @pytest.mark.parametrize("field,value", [
     ("n_kv_heads", 3), ("head_dim", 96), ("n_beacons", 33), ("window", -1), ("window", 65),
-    ("capacity", 0), ("capacity", 40000), ("rope_theta", -1.0), ("flags", 4), ("flags", 0x80000000), ("n_layers", 0),
+    ("capacity", 0), ("capacity", 40000), ("rope_theta", -1.0), ("flags", 8), ("flags", 0x80000000), ("n_layers", 0),
     ("n_prefix", -2)])
 def test_create_rejects_bad_config_before_touching_the_gpu(lib, field, value):
     cfg = bkv.BkvConfig(1, 1, 4, 2, 64, 4, 8, 0, 1088, 1e4, 0)

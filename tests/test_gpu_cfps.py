@@ -30,7 +30,7 @@ def _heads(t: torch.Tensor, d: int) -> np.ndarray:
     return _bits(t).reshape(-1, t.shape[-2], d)
 
 
-def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False):
+def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False, causal=False):
     dev = torch.device("cuda")
     inp = synth.step_inputs(wl, seed, dev)
     L = wl.L if L is None else L
@@ -41,7 +41,7 @@ def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False):
     q_new_t = inp["q_new"] if n_new is None else inp["q_new"][..., :n_new, :].contiguous()
     bk = BeaconKV(n_layers=wl.n_layers, batch=wl.batch, n_q_heads=wl.n_q_heads, n_kv_heads=wl.n_kv_heads, head_dim=d,
                   n_beacons=b_min, window=W, capacity=wl.capacity, rope_theta=wl.rope_theta, n_prefix=wl.n_prefix,
-                  continual_fps=True, mean_agg=mean_agg)
+                  continual_fps=True, mean_agg=mean_agg, causal_window=causal)
     try:
         bk.init_beacons(inp["q_init"])
         buf0, size0 = [x.cpu() for x in bk.cfps_state()]
@@ -90,7 +90,7 @@ def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False):
         hs = slice(e * G, (e + 1) * G)
         r, sw = P.check_cfps_compress(wl, b_min, buf1[hs], size1[hs], q_rec[hs], inp["recent_pos"], inp["t_pos"],
                                       Kb[e], Vb[e], K1[e], V1[e], kept_h[e], s_h[e], L, budget, buf2[hs], size2[hs],
-                                      lib, tag=f"instance {e}", mean=mean_agg)
+                                      lib, tag=f"instance {e}", mean=mean_agg, causal=causal)
         rel_max, swaps = max(rel_max, r), swaps + sw
     print(f"{wl.name}: {n_heads} heads, seed ties {fps_ties}, max score rel err {rel_max:.2e}, swaps {swaps}")
 
@@ -118,6 +118,11 @@ def test_continual_fps_ragged_cache():
 def test_continual_fps_with_mean_aggregation():
     wl = QWEN3_4B.scaled(name="cfps_mean_1L_b1", n_layers=1, batch=1, L=900, budget=500)
     _run_cfps(wl, 26, 8, mean_agg=True)
+
+
+def test_continual_fps_with_causal_window():
+    wl = QWEN3_4B.scaled(name="cfps_causal_1L_b1", n_layers=1, batch=1, L=900, budget=500)
+    _run_cfps(wl, 28, 8, causal=True)
 
 
 def test_continual_fps_state_round_trip():

@@ -8,6 +8,7 @@ import numpy as np
 import pytest
 import torch
 
+from paper_2609_04971_gb300 import synth
 from paper_2609_04971_gb300.workloads import LLAMA_8B, QWEN3_14B, QWEN3_4B, TINY
 
 pytestmark = pytest.mark.gpu
@@ -126,6 +127,40 @@ def test_deterministic_across_runs():
     np.testing.assert_array_equal(a.scores, b.scores)
     np.testing.assert_array_equal(a.cent1, b.cent1)
     np.testing.assert_array_equal(a.K_after, b.K_after)
+
+
+# ---------------------------------------------------------------- causal mask inside the window (BKV_F_CAUSAL_WINDOW)
+def _shift_positions(inp, W, t_pos, recent_pos):
+    inp = dict(inp)
+    inp["t_pos"] = int(t_pos)
+    inp["recent_pos"] = [int(p) for p in recent_pos][:W]
+    return inp
+
+
+@pytest.mark.parametrize("mean", [False, True], ids=["max", "mean"])
+@pytest.mark.parametrize("wl,seed", [
+    (TINY.scaled(name="causal_tiny"), 41),
+    (QWEN3_4B.scaled(name="causal_qwen3_4b_1L_b2", n_layers=1, batch=2), 42),
+    (QWEN3_4B.scaled(name="causal_ragged_L300_B40_w16", n_layers=1, batch=1, L=300, budget=40, window=16), 43),
+    (QWEN3_4B.scaled(name="causal_long_L20000", n_layers=1, batch=1, L=20000, budget=9000), 44),
+    (QWEN3_4B.scaled(name="causal_nb0", n_layers=1, batch=1, L=500, budget=260, n_beacons=0), 45),
+], ids=lambda x: getattr(x, "name", str(x)))
+def test_causal_window(wl, seed, mean):
+    _run(wl, seed=seed, mean_agg=mean, causal=True)
+
+
+@pytest.mark.parametrize("case", ["decode_after_evictions", "sparse_recent_positions"])
+def test_causal_window_positions(case):
+    """Positions that are not the last L rows: a decode step long after earlier evictions (t = 9000 with
+    640 cached rows), and recent queries at scattered earlier positions (some see no window row, one
+    sees them all)."""
+    wl = QWEN3_4B.scaled(name=f"causal_{case}", n_layers=1, batch=1, L=640, budget=300, window=8)
+    inp = synth.step_inputs(wl, 46, torch.device("cuda"))
+    if case == "decode_after_evictions":
+        inp = _shift_positions(inp, 8, 9000, range(8993, 9001))
+    else:
+        inp = _shift_positions(inp, 8, 9000, [100, 8990, 8994, 8995, 8996, 8998, 9000, 9000])
+    _run(wl, seed=46, inputs=inp, causal=True)
 
 
 # ---------------------------------------------------------------- Eq. 6 mean form (BKV_F_MEAN_AGG)

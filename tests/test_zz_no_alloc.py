@@ -18,11 +18,11 @@ from paper_2609_04971_gb300.workloads import QWEN3_4B, TINY
 pytestmark = pytest.mark.gpu
 
 
-def _compare_once(wl, seed):
+def _compare_once(wl, seed, causal=False):
     from paper_2609_04971_gb300 import bkv, synth
     dev = torch.device("cuda")
     inp = synth.step_inputs(wl, seed, dev)
-    bk = bkv.BeaconKV.for_workload(wl)
+    bk = bkv.BeaconKV.for_workload(wl, causal_window=causal)
     try:
         bk.init_beacons(inp["q_init"])
         bk.update(inp["q_new"])
@@ -56,6 +56,7 @@ def test_static_compress_matches_context_compress_on_consecutive_calls():
     _compare_once(ragged, seed=21)
     _compare_once(ragged, seed=22)        # same shape, new data over the previous scratch contents
     _compare_once(TINY, seed=23)          # another shape (head_dim 64) over the same scratch
+    _compare_once(ragged, seed=24, causal=True)   # the causal mask inside the window (cfg.flags)
 
 
 def test_static_compress_rejects_requests_beyond_its_scratch():
