@@ -47,7 +47,7 @@ def parse():
     ap.add_argument("--config", type=int, default=2, help="workload number (2 = Qwen3-4B shape)")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (small profiling captures)")
-    ap.add_argument("--e2e-steps", type=int, default=8, help="timed host-resident steps (pipelined)")
+    ap.add_argument("--e2e-steps", type=int, default=16, help="timed host-resident steps (pipelined)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
