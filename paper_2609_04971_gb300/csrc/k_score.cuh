@@ -520,74 +520,154 @@ __global__ void __launch_bounds__(kScThreads, 1)
         bool have = !*abort_flag && mbar_wait(&slot_full[slot], u & 1, abort_flag, a.err, kDevTimeoutEpilogue);
         have = __all_sync(0xffffffffu, have);
         if (j < R) resident_ok = resident_ok && have;
-        float v[NQ];
-        if (have) {
-          tc_fence_after();
-#pragma unroll
-          for (int c = 0; c < NQ; c += 8) {
-            uint32_t r[8];
-            asm volatile(
-                "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-                : "r"(tmem + slot * N + half * NQ + c + lane_addr));
-#pragma unroll
-            for (int q = 0; q < 8; ++q) v[c + q] = __uint_as_float(r[q]);
-          }
-          tmem_wait_ld();
-        }
-        if (j >= R) {  // a streaming slot is free once every warp has its columns
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&slot_free[slot]);
-          ++ks;
-        }
-        // Running sums relative to a reference m that moves only when a base-2
-        // logit exceeds it by more than 64, so the terms stay below 2^64 and
-        // the common step is one FFMA, one ex2 and one add per column.
-        const int tile0 = k0 + j * kTile;
-        if (have && CAUSAL && tile0 + kTile > a.win0) {
-          // a tile with window rows: the careful path, without the masked (row, column) terms
+        if constexpr (NQ > 32) {
+          // Many columns: the tile is read and summed in chunks of 32 columns, and each
+          // exponent argument is computed again where it is used, so that a thread holds its
+          // running (m, s) pairs and one chunk of logits; the values equal the one-chunk form.
+          constexpr int kCh = 32;
+          const int tile0 = k0 + j * kTile;
           const int key = tile0 + key_row;
-          if (key < k1) {
-            const bool in_win = key >= a.win0;
+          const bool key_ok = key < k1;
+          const bool ragged = !__all_sync(0xffffffffu, key_ok);
+          const bool masked_tile = CAUSAL && tile0 + kTile > a.win0;
+          const bool in_win = CAUSAL && key >= a.win0;
 #pragma unroll
-            for (int c = 0; c < NQ; ++c) {
-              if (in_win && key > thr_sh[half * NQ + c]) continue;
-              const float t = fmaf(v[c], sc, -m[c]);
-              if (t > 64.f) {
-                const float y = v[c] * sc;
-                sm[c] = fmaf(sm[c], ex2_approx(m[c] - y), 1.f);
-                m[c] = y;
+          for (int cc = 0; cc < NQ; cc += kCh) {
+            float v[kCh];
+            if (have) {
+              tc_fence_after();
+#pragma unroll
+              for (int c = 0; c < kCh; c += 8) {
+                if (cc + c < NQ) {
+                  uint32_t r[8];
+                  asm volatile(
+                      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                      : "r"(tmem + slot * N + half * NQ + cc + c + lane_addr));
+#pragma unroll
+                  for (int q = 0; q < 8; ++q) v[c + q] = __uint_as_float(r[q]);
+                }
+              }
+              tmem_wait_ld();
+              if (masked_tile) {
+                if (key_ok) {
+#pragma unroll
+                  for (int c = 0; c < kCh; ++c) {
+                    if (cc + c >= NQ || (in_win && key > thr_sh[half * NQ + cc + c])) continue;
+                    const float t = fmaf(v[c], sc, -m[cc + c]);
+                    if (t > 64.f) {
+                      const float y = v[c] * sc;
+                      sm[cc + c] = fmaf(sm[cc + c], ex2_approx(m[cc + c] - y), 1.f);
+                      m[cc + c] = y;
+                    } else {
+                      sm[cc + c] += ex2_approx(t);
+                    }
+                  }
+                }
               } else {
-                sm[c] += ex2_approx(t);
+                bool rebase = ragged;
+#pragma unroll
+                for (int c = 0; c < kCh; ++c)
+                  if (cc + c < NQ) rebase |= fmaf(v[c], sc, -m[cc + c]) > 64.f;
+                if (__any_sync(0xffffffffu, rebase)) {
+                  if (key_ok) {
+#pragma unroll
+                    for (int c = 0; c < kCh; ++c) {
+                      if (cc + c >= NQ) continue;
+                      const float t = fmaf(v[c], sc, -m[cc + c]);
+                      if (t > 64.f) {  // also the first key: m = -inf gives t = +inf
+                        const float y = v[c] * sc;
+                        sm[cc + c] = fmaf(sm[cc + c], ex2_approx(m[cc + c] - y), 1.f);
+                        m[cc + c] = y;
+                      } else {
+                        sm[cc + c] += ex2_approx(t);
+                      }
+                    }
+                  }
+                } else {
+#pragma unroll
+                  for (int c = 0; c < kCh; ++c)
+                    if (cc + c < NQ) sm[cc + c] += ex2_approx(fmaf(v[c], sc, -m[cc + c]));
+                }
               }
             }
           }
-        } else if (have) {
-          const bool key_ok = tile0 + key_row < k1;
-          float t[NQ];
-          bool rebase = !__all_sync(0xffffffffu, key_ok);  // a ragged tile takes the careful path
-#pragma unroll
-          for (int c = 0; c < NQ; ++c) {
-            t[c] = fmaf(v[c], sc, -m[c]);
-            rebase |= t[c] > 64.f;
+          if (j >= R) {  // a streaming slot is free once every warp has its columns
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&slot_free[slot]);
+            ++ks;
           }
-          if (__any_sync(0xffffffffu, rebase)) {
-            if (key_ok) {
+        } else {
+          float v[NQ];
+          if (have) {
+            tc_fence_after();
+#pragma unroll
+            for (int c = 0; c < NQ; c += 8) {
+              uint32_t r[8];
+              asm volatile(
+                  "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                  : "r"(tmem + slot * N + half * NQ + c + lane_addr));
+#pragma unroll
+              for (int q = 0; q < 8; ++q) v[c + q] = __uint_as_float(r[q]);
+            }
+            tmem_wait_ld();
+          }
+          if (j >= R) {  // a streaming slot is free once every warp has its columns
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&slot_free[slot]);
+            ++ks;
+          }
+          // Running sums relative to a reference m that moves only when a base-2
+          // logit exceeds it by more than 64, so the terms stay below 2^64 and
+          // the common step is one FFMA, one ex2 and one add per column.
+          const int tile0 = k0 + j * kTile;
+          if (have && CAUSAL && tile0 + kTile > a.win0) {
+            // a tile with window rows: the careful path, without the masked (row, column) terms
+            const int key = tile0 + key_row;
+            if (key < k1) {
+              const bool in_win = key >= a.win0;
 #pragma unroll
               for (int c = 0; c < NQ; ++c) {
-                if (t[c] > 64.f) {  // also the first key: m = -inf gives t = +inf
+                if (in_win && key > thr_sh[half * NQ + c]) continue;
+                const float t = fmaf(v[c], sc, -m[c]);
+                if (t > 64.f) {
                   const float y = v[c] * sc;
                   sm[c] = fmaf(sm[c], ex2_approx(m[c] - y), 1.f);
                   m[c] = y;
                 } else {
-                  sm[c] += ex2_approx(t[c]);
+                  sm[c] += ex2_approx(t);
                 }
               }
             }
-          } else {
+          } else if (have) {
+            const bool key_ok = tile0 + key_row < k1;
+            float t[NQ];
+            bool rebase = !__all_sync(0xffffffffu, key_ok);  // a ragged tile takes the careful path
 #pragma unroll
-            for (int c = 0; c < NQ; ++c) sm[c] += ex2_approx(t[c]);
+            for (int c = 0; c < NQ; ++c) {
+              t[c] = fmaf(v[c], sc, -m[c]);
+              rebase |= t[c] > 64.f;
+            }
+            if (__any_sync(0xffffffffu, rebase)) {
+              if (key_ok) {
+#pragma unroll
+                for (int c = 0; c < NQ; ++c) {
+                  if (t[c] > 64.f) {  // also the first key: m = -inf gives t = +inf
+                    const float y = v[c] * sc;
+                    sm[c] = fmaf(sm[c], ex2_approx(m[c] - y), 1.f);
+                    m[c] = y;
+                  } else {
+                    sm[c] += ex2_approx(t[c]);
+                  }
+                }
+              }
+            } else {
+#pragma unroll
+              for (int c = 0; c < NQ; ++c) sm[c] += ex2_approx(t[c]);
+            }
           }
         }
       }
