@@ -3,6 +3,7 @@
 // the rotary table, and kernel launches on the context's stream.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -449,13 +450,10 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
   }
   if (e != cudaSuccess) return cuda_fail(ctx, e, "qobs launch");
 
-  CUtensorMap kmap, kmap32, qmap;
+  CUtensorMap kmap, kmap32;
   int rc = encode_rows(ctx, &kmap, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 128);
   if (rc != BKV_OK) return rc;
   rc = encode_rows(ctx, &kmap32, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 32);
-  if (rc != BKV_OK) return rc;
-  rc = encode_rows(ctx, &qmap, ctx->qobs, static_cast<uint64_t>(s.n_inst) * s.n_obs_pad, s.d,
-                   static_cast<uint32_t>(s.n_obs_pad));
   if (rc != BKV_OK) return rc;
   bkv::ScoreArgs sa;
   sa.L = L;
@@ -464,13 +462,23 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
   sa.mean = (ctx->cfg.flags & BKV_F_MEAN_AGG) != 0;
   if (ctx->cfg.flags & BKV_F_CAUSAL_WINDOW) bkv::set_causal(sa, L, s.W, t_pos, recent_pos);
   sa.r_out = ctx->rscore;
-  sa.scores_out = scores_out;
   sa.err = ctx->err;
-  {
-    ProfScope ps(ctx, BKV_K_SCORE);
-    e = bkv::launch_score(s, kmap, kmap32, qmap, sa, ctx->stream);
+  // one launch per 64 scoring queries; later launches fold into the first's scores
+  for (int col0 = 0; col0 < s.n_obs_pad; col0 += bkv::kScoreMaxCols) {
+    CUtensorMap qmap;
+    sa.col0 = col0;
+    sa.n_cols = std::min(bkv::kScoreMaxCols, s.n_obs_pad - col0);
+    sa.combine = col0 > 0;
+    sa.scores_out = col0 + sa.n_cols == s.n_obs_pad ? scores_out : nullptr;
+    rc = encode_rows(ctx, &qmap, ctx->qobs, static_cast<uint64_t>(s.n_inst) * s.n_obs_pad, s.d,
+                     static_cast<uint32_t>(sa.n_cols));
+    if (rc != BKV_OK) return rc;
+    {
+      ProfScope ps(ctx, BKV_K_SCORE);
+      e = bkv::launch_score(s, kmap, kmap32, qmap, sa, ctx->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "score launch");
   }
-  if (e != cudaSuccess) return cuda_fail(ctx, e, "score launch");
   {
     ProfScope ps(ctx, BKV_K_SELECT_GATHER);
     e = bkv::launch_select_gather(s, ctx->rscore, L, budget, static_cast<__nv_bfloat16*>(K),

@@ -72,6 +72,9 @@ struct ScoreArgs {
   bool causal = false;             // causal mask inside the recent window (set_causal)
   int win0 = 0;                    // first window row, L - W
   int thr[kMaxWindow] = {};        // recent slot w sees window row j only if j <= thr[w]
+  int col0 = 0;                    // column split: first Q_obs row of this launch (a multiple of 64)
+  int n_cols = 0;                  // padded query rows of this launch: 16, 32, 48 or 64
+  bool combine = false;            // fold into r_out of the launch of the rows before col0
   float* r_out = nullptr;          // [n_inst][cap] log2-domain scores (log2 of the aggregated weight)
   float* scores_out = nullptr;     // [n_inst][cap] probabilities, or nullptr
   int* err = nullptr;              // device error word
@@ -91,9 +94,10 @@ inline void set_causal(ScoreArgs& a, int L, int W, long long t_pos, const int64_
     }
   }
 }
+constexpr int kScoreMaxCols = 64;  // scoring queries per score launch (column split beyond)
 // kmap / kmap32: K as [n_inst * cap][d] in 128-row and 32-row boxes of [64]
 // columns (128-byte swizzle); qmap: Qobs as [n_inst * n_obs_pad][d] in boxes
-// of n_obs_pad rows.
+// of n_cols rows (the launch's Q_obs rows start at row e * n_obs_pad + col0).
 cudaError_t launch_score(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32, const CUtensorMap& qmap,
                          const ScoreArgs& a, cudaStream_t st);
 // The mean form (a.mean) and the causal forms (a.causal), each compiled in its own translation

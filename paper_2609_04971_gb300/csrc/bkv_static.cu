@@ -22,6 +22,7 @@
 //   * the device address of the array is looked up with cudaGetSymbolAddress
 //     the first time this entry point runs on a device (with that device
 //     current), so that first call should come before any stream capture.
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -207,11 +208,9 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
   }
   e = bkv::launch_qobs(s, static_cast<const __nv_bfloat16*>(q_recent), centroids,
                        reinterpret_cast<const long long*>(counts), rope, rotate, qobs, valid, st);
-  CUtensorMap kmap, kmap32, qmap;
+  CUtensorMap kmap, kmap32;
   if (e == cudaSuccess && (!encode(&kmap, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 128) ||
-                           !encode(&kmap32, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 32) ||
-                           !encode(&qmap, qobs, static_cast<uint64_t>(s.n_inst) * s.n_obs_pad, s.d,
-                                   static_cast<uint32_t>(s.n_obs_pad)))) {
+                           !encode(&kmap32, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 32))) {
     message(err_msg, err_len, "cuTensorMapEncodeTiled failed");
     return BKV_ECUDA;
   }
@@ -223,9 +222,20 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
     sa.mean = (cfg->flags & BKV_F_MEAN_AGG) != 0;
     if (cfg->flags & BKV_F_CAUSAL_WINDOW) bkv::set_causal(sa, L, s.W, t_pos, recent_pos);
     sa.r_out = rscore;
-    sa.scores_out = scores_out;
     sa.err = reinterpret_cast<int*>(dev_status);
-    e = bkv::launch_score(s, kmap, kmap32, qmap, sa, st);
+    // one launch per 64 scoring queries; later launches fold into the first's scores
+    for (int col0 = 0; e == cudaSuccess && col0 < s.n_obs_pad; col0 += bkv::kScoreMaxCols) {
+      CUtensorMap qmap;
+      sa.col0 = col0;
+      sa.n_cols = std::min(bkv::kScoreMaxCols, s.n_obs_pad - col0);
+      sa.combine = col0 > 0;
+      sa.scores_out = col0 + sa.n_cols == s.n_obs_pad ? scores_out : nullptr;
+      if (!encode(&qmap, qobs, static_cast<uint64_t>(s.n_inst) * s.n_obs_pad, s.d, static_cast<uint32_t>(sa.n_cols))) {
+        message(err_msg, err_len, "cuTensorMapEncodeTiled failed");
+        return BKV_ECUDA;
+      }
+      e = bkv::launch_score(s, kmap, kmap32, qmap, sa, st);
+    }
   }
   if (e == cudaSuccess)
     e = bkv::launch_select_gather(s, rscore, L, budget, static_cast<__nv_bfloat16*>(K),

@@ -51,6 +51,14 @@
 // barrier, so no CTA leaves while a peer may still write to its shared memory.
 // Outputs: r (log2 scores, for selection) and optionally 2^r.
 //
+// Column split: a launch takes at most 64 scoring queries, Q_obs rows
+// [col0, col0 + N).  Each query's normaliser lse2_q depends on its own column
+// only, so with more queries the caller runs one launch per 64 rows and every
+// later launch folds its r into the previous one (max: the larger; mean: the
+// log2 of the sum of the two powers of 2, both scaled by the count of all
+// valid queries).  K is then read once per launch, and the tensor memory ring
+// keeps spare slots at every query count.
+//
 // Causal form (CAUSAL): recent slot w must not see window rows after its own
 // position (row j >= L - W is masked for it when j > thr[w]); beacons and
 // older rows are never masked.  Only tiles that hold window rows take the
@@ -81,20 +89,20 @@ template <int D>
 struct ScoreCfg {
   static constexpr int kBoxes = D / 64;                  // 64-column boxes per row
   static constexpr uint32_t kTileBytes = kTile * D * 2;  // one K tile
-  static size_t q_bytes(int n_obs_pad) { return 2 * static_cast<size_t>(kBoxes) * n_obs_pad * 128; }
-  // two receive buffers of csize x n_obs_pad (m, s) pairs
-  static size_t recv_bytes(int n_obs_pad, int csize) {
-    return csize > 1 ? 2 * static_cast<size_t>(csize) * n_obs_pad * 8 : 0;
+  static size_t q_bytes(int n_cols) { return 2 * static_cast<size_t>(kBoxes) * n_cols * 128; }
+  // two receive buffers of csize x n_cols (m, s) pairs
+  static size_t recv_bytes(int n_cols, int csize) {
+    return csize > 1 ? 2 * static_cast<size_t>(csize) * n_cols * 8 : 0;
   }
   // as many K stages as fit next to the query and receive buffers
-  static int stages(int n_obs_pad, int csize) {
-    const size_t room = kSmemBudget - 1024 - q_bytes(n_obs_pad) - recv_bytes(n_obs_pad, csize);
+  static int stages(int n_cols, int csize) {
+    const size_t room = kSmemBudget - 1024 - q_bytes(n_cols) - recv_bytes(n_cols, csize);
     const int n = static_cast<int>(room / (static_cast<size_t>(kBoxes) * kBoxBytes));
     return n < kMaxStages ? n : kMaxStages;
   }
-  static size_t smem_bytes(int n_obs_pad, int csize) {
-    return 1024 + q_bytes(n_obs_pad) + static_cast<size_t>(stages(n_obs_pad, csize)) * kBoxes * kBoxBytes +
-           recv_bytes(n_obs_pad, csize);
+  static size_t smem_bytes(int n_cols, int csize) {
+    return 1024 + q_bytes(n_cols) + static_cast<size_t>(stages(n_cols, csize)) * kBoxes * kBoxBytes +
+           recv_bytes(n_cols, csize);
   }
 };
 
@@ -250,6 +258,19 @@ __device__ __forceinline__ float tile_agg(uint32_t taddr, const float* lse2, flo
   }
 }
 
+// r of a key over the columns of two launches (column split): the max form
+// keeps the larger, the mean form adds the two powers of 2 (both launches
+// scale by the count of all valid queries).
+template <bool MEAN>
+__device__ __forceinline__ float fold_split(float r_prev, float r) {
+  if constexpr (MEAN) {
+    const float hi = fmaxf(r_prev, r), lo = fminf(r_prev, r);
+    return hi == -INFINITY ? hi : hi + lg2_approx(1.f + ex2_approx(lo - hi));
+  } else {
+    return fmaxf(r_prev, r);
+  }
+}
+
 // tile_agg for a tile that holds window rows: column c is left out for key
 // `key` when key >= win0 and key > thr[c].
 template <int N, bool MEAN>
@@ -286,13 +307,13 @@ __device__ __forceinline__ float tile_agg_causal(uint32_t taddr, const float* ls
   }
 }
 
-template <int D, int NQ, bool MEAN, bool CAUSAL>
+template <int D, int NQ, bool MEAN, bool CAUSAL, bool COMBINE>
 __global__ void __launch_bounds__(kScThreads, 1)
     score_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap kmap32,
                  const __grid_constant__ CUtensorMap qmap, Shape s, ScoreArgs a, Plan plan, int n_stages) {
   using C = ScoreCfg<D>;
   constexpr int N = 2 * NQ;  // padded query columns
-  static_assert(NQ % 8 == 0 && NQ <= 64, "query columns per pass-1 warp");
+  static_assert(NQ % 8 == 0 && NQ <= 32, "query columns per pass-1 warp");
   extern __shared__ unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kMaxStages], empty_bar[kMaxStages];
   __shared__ __align__(8) uint64_t slot_full[kMaxSlots], slot_free[kMaxSlots];
@@ -319,12 +340,13 @@ __global__ void __launch_bounds__(kScThreads, 1)
   const int n_str = T - R;                           // streaming tiles (plan.stream only)
   const int ring = plan.slots;                       // resident slots, used in cyclic order
   const int str_slot = ring;                         // pass-1 streaming slots; +2, +3: pass-2 slots
-  const uint32_t qbox = static_cast<uint32_t>(s.n_obs_pad) * 128;
+  const uint32_t qbox = static_cast<uint32_t>(a.n_cols) * 128;  // one 64-column box of this launch's queries (N rows)
+  const int col0 = COMBINE ? a.col0 : 0;  // only a later launch of a column split starts past row 0
 
   // 1024-byte aligned (the 128-byte swizzle pattern repeats every 1024 bytes);
   // offset from the __shared__ array itself so that accesses stay shared-space
   unsigned char* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-  unsigned char* q_smem = base;                         // [2 buffers][kBoxes][n_obs_pad rows x 128 B]
+  unsigned char* q_smem = base;                         // [2 buffers][kBoxes][N rows x 128 B]
   unsigned char* k_smem = base + 2 * C::kBoxes * qbox;  // [n_stages][kBoxes][128 rows x 128 B]
   float2* recv = reinterpret_cast<float2*>(k_smem + n_stages * C::kBoxes * kBoxBytes);  // [2][csize][N]
 
@@ -349,8 +371,8 @@ __global__ void __launch_bounds__(kScThreads, 1)
   }
   if constexpr (CAUSAL) {
     if (threadIdx.x < 128) {
-      const int c = threadIdx.x;  // recent slot c % W of head c / W, or a beacon / padding column
-      thr_sh[c] = c < s.G * s.W ? a.thr[c % s.W] : 0x7fffffff;
+      const int c = col0 + threadIdx.x;  // Q_obs row: recent slot c % W of head c / W, or a beacon / padding
+      thr_sh[threadIdx.x] = c < s.G * s.W ? a.thr[c % s.W] : 0x7fffffff;
     }
   }
   if (warp == 1) {
@@ -383,9 +405,10 @@ __global__ void __launch_bounds__(kScThreads, 1)
           ok = false;
           break;
         }
-        mbar_arrive_expect_tx(&qfull_bar[qb], static_cast<uint32_t>(s.n_obs_pad) * D * 2);
+        mbar_arrive_expect_tx(&qfull_bar[qb], static_cast<uint32_t>(a.n_cols) * D * 2);
         for (int b = 0; b < C::kBoxes; ++b)
-          tma_load_2d(q_smem + (qb * C::kBoxes + b) * qbox, &qmap, &qfull_bar[qb], b * 64, e * s.n_obs_pad, again);
+          tma_load_2d(q_smem + (qb * C::kBoxes + b) * qbox, &qmap, &qfull_bar[qb], b * 64,
+                      e * s.n_obs_pad + col0, again);
         q_issued = i + 1;
         for (int j = 0; j < T + n_str; ++j) {
           const int t = j < T ? j : R + (j - T);
@@ -490,12 +513,18 @@ __global__ void __launch_bounds__(kScThreads, 1)
     int ks = 0, kp2 = 0;  // uses of the pass-1 streaming slots / of this half's pass-2 slot
     int rs = 0, ru = 0;   // ring slot and use count of this instance's first tile
     // valid-row words are fetched one instance ahead: a global load queues
-    // behind the K stream for microseconds
-    uint32_t vnext = (te < 128 && n_my > 0) ? ld_nc_u32(&a.valid[cluster_id * 4 + (te >> 5)]) : 0u;
+    // behind the K stream for microseconds.  Thread te < N reads the word of
+    // its column (Q_obs row col0 + te); the four words that threads 0, 32, 64
+    // and 96 read are all of the instance's words in some order (their total
+    // is the valid count of the mean form).
+    uint32_t vnext = (te < 128 && n_my > 0)
+                         ? ld_nc_u32(&a.valid[cluster_id * 4 + (COMBINE ? ((col0 >> 5) + (te >> 5)) & 3 : te >> 5)])
+                         : 0u;
     for (int i = 0; i < n_my; ++i) {
       const int e = cluster_id + i * n_clusters;
       const uint32_t vword = vnext;
-      if (te < 128 && i + 1 < n_my) vnext = ld_nc_u32(&a.valid[(e + n_clusters) * 4 + (te >> 5)]);
+      if (te < 128 && i + 1 < n_my)
+        vnext = ld_nc_u32(&a.valid[(e + n_clusters) * 4 + (COMBINE ? ((col0 >> 5) + (te >> 5)) & 3 : te >> 5)]);
       float m[NQ], sm[NQ];
 #pragma unroll
       for (int c = 0; c < NQ; ++c) {
@@ -520,154 +549,74 @@ __global__ void __launch_bounds__(kScThreads, 1)
         bool have = !*abort_flag && mbar_wait(&slot_full[slot], u & 1, abort_flag, a.err, kDevTimeoutEpilogue);
         have = __all_sync(0xffffffffu, have);
         if (j < R) resident_ok = resident_ok && have;
-        if constexpr (NQ > 32) {
-          // Many columns: the tile is read and summed in chunks of 32 columns, and each
-          // exponent argument is computed again where it is used, so that a thread holds its
-          // running (m, s) pairs and one chunk of logits; the values equal the one-chunk form.
-          constexpr int kCh = 32;
-          const int tile0 = k0 + j * kTile;
+        float v[NQ];
+        if (have) {
+          tc_fence_after();
+#pragma unroll
+          for (int c = 0; c < NQ; c += 8) {
+            uint32_t r[8];
+            asm volatile(
+                "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                : "r"(tmem + slot * N + half * NQ + c + lane_addr));
+#pragma unroll
+            for (int q = 0; q < 8; ++q) v[c + q] = __uint_as_float(r[q]);
+          }
+          tmem_wait_ld();
+        }
+        if (j >= R) {  // a streaming slot is free once every warp has its columns
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&slot_free[slot]);
+          ++ks;
+        }
+        // Running sums relative to a reference m that moves only when a base-2
+        // logit exceeds it by more than 64, so the terms stay below 2^64 and
+        // the common step is one FFMA, one ex2 and one add per column.
+        const int tile0 = k0 + j * kTile;
+        if (have && CAUSAL && tile0 + kTile > a.win0) {
+          // a tile with window rows: the careful path, without the masked (row, column) terms
           const int key = tile0 + key_row;
-          const bool key_ok = key < k1;
-          const bool ragged = !__all_sync(0xffffffffu, key_ok);
-          const bool masked_tile = CAUSAL && tile0 + kTile > a.win0;
-          const bool in_win = CAUSAL && key >= a.win0;
+          if (key < k1) {
+            const bool in_win = key >= a.win0;
 #pragma unroll
-          for (int cc = 0; cc < NQ; cc += kCh) {
-            float v[kCh];
-            if (have) {
-              tc_fence_after();
-#pragma unroll
-              for (int c = 0; c < kCh; c += 8) {
-                if (cc + c < NQ) {
-                  uint32_t r[8];
-                  asm volatile(
-                      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-                      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-                      : "r"(tmem + slot * N + half * NQ + cc + c + lane_addr));
-#pragma unroll
-                  for (int q = 0; q < 8; ++q) v[c + q] = __uint_as_float(r[q]);
-                }
-              }
-              tmem_wait_ld();
-              if (masked_tile) {
-                if (key_ok) {
-#pragma unroll
-                  for (int c = 0; c < kCh; ++c) {
-                    if (cc + c >= NQ || (in_win && key > thr_sh[half * NQ + cc + c])) continue;
-                    const float t = fmaf(v[c], sc, -m[cc + c]);
-                    if (t > 64.f) {
-                      const float y = v[c] * sc;
-                      sm[cc + c] = fmaf(sm[cc + c], ex2_approx(m[cc + c] - y), 1.f);
-                      m[cc + c] = y;
-                    } else {
-                      sm[cc + c] += ex2_approx(t);
-                    }
-                  }
-                }
+            for (int c = 0; c < NQ; ++c) {
+              if (in_win && key > thr_sh[half * NQ + c]) continue;
+              const float t = fmaf(v[c], sc, -m[c]);
+              if (t > 64.f) {
+                const float y = v[c] * sc;
+                sm[c] = fmaf(sm[c], ex2_approx(m[c] - y), 1.f);
+                m[c] = y;
               } else {
-                bool rebase = ragged;
-#pragma unroll
-                for (int c = 0; c < kCh; ++c)
-                  if (cc + c < NQ) rebase |= fmaf(v[c], sc, -m[cc + c]) > 64.f;
-                if (__any_sync(0xffffffffu, rebase)) {
-                  if (key_ok) {
-#pragma unroll
-                    for (int c = 0; c < kCh; ++c) {
-                      if (cc + c >= NQ) continue;
-                      const float t = fmaf(v[c], sc, -m[cc + c]);
-                      if (t > 64.f) {  // also the first key: m = -inf gives t = +inf
-                        const float y = v[c] * sc;
-                        sm[cc + c] = fmaf(sm[cc + c], ex2_approx(m[cc + c] - y), 1.f);
-                        m[cc + c] = y;
-                      } else {
-                        sm[cc + c] += ex2_approx(t);
-                      }
-                    }
-                  }
-                } else {
-#pragma unroll
-                  for (int c = 0; c < kCh; ++c)
-                    if (cc + c < NQ) sm[cc + c] += ex2_approx(fmaf(v[c], sc, -m[cc + c]));
-                }
+                sm[c] += ex2_approx(t);
               }
             }
           }
-          if (j >= R) {  // a streaming slot is free once every warp has its columns
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&slot_free[slot]);
-            ++ks;
-          }
-        } else {
-          float v[NQ];
-          if (have) {
-            tc_fence_after();
+        } else if (have) {
+          const bool key_ok = tile0 + key_row < k1;
+          float t[NQ];
+          bool rebase = !__all_sync(0xffffffffu, key_ok);  // a ragged tile takes the careful path
 #pragma unroll
-            for (int c = 0; c < NQ; c += 8) {
-              uint32_t r[8];
-              asm volatile(
-                  "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-                  : "r"(tmem + slot * N + half * NQ + c + lane_addr));
-#pragma unroll
-              for (int q = 0; q < 8; ++q) v[c + q] = __uint_as_float(r[q]);
-            }
-            tmem_wait_ld();
+          for (int c = 0; c < NQ; ++c) {
+            t[c] = fmaf(v[c], sc, -m[c]);
+            rebase |= t[c] > 64.f;
           }
-          if (j >= R) {  // a streaming slot is free once every warp has its columns
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&slot_free[slot]);
-            ++ks;
-          }
-          // Running sums relative to a reference m that moves only when a base-2
-          // logit exceeds it by more than 64, so the terms stay below 2^64 and
-          // the common step is one FFMA, one ex2 and one add per column.
-          const int tile0 = k0 + j * kTile;
-          if (have && CAUSAL && tile0 + kTile > a.win0) {
-            // a tile with window rows: the careful path, without the masked (row, column) terms
-            const int key = tile0 + key_row;
-            if (key < k1) {
-              const bool in_win = key >= a.win0;
+          if (__any_sync(0xffffffffu, rebase)) {
+            if (key_ok) {
 #pragma unroll
               for (int c = 0; c < NQ; ++c) {
-                if (in_win && key > thr_sh[half * NQ + c]) continue;
-                const float t = fmaf(v[c], sc, -m[c]);
-                if (t > 64.f) {
+                if (t[c] > 64.f) {  // also the first key: m = -inf gives t = +inf
                   const float y = v[c] * sc;
                   sm[c] = fmaf(sm[c], ex2_approx(m[c] - y), 1.f);
                   m[c] = y;
                 } else {
-                  sm[c] += ex2_approx(t);
+                  sm[c] += ex2_approx(t[c]);
                 }
               }
             }
-          } else if (have) {
-            const bool key_ok = tile0 + key_row < k1;
-            float t[NQ];
-            bool rebase = !__all_sync(0xffffffffu, key_ok);  // a ragged tile takes the careful path
+          } else {
 #pragma unroll
-            for (int c = 0; c < NQ; ++c) {
-              t[c] = fmaf(v[c], sc, -m[c]);
-              rebase |= t[c] > 64.f;
-            }
-            if (__any_sync(0xffffffffu, rebase)) {
-              if (key_ok) {
-#pragma unroll
-                for (int c = 0; c < NQ; ++c) {
-                  if (t[c] > 64.f) {  // also the first key: m = -inf gives t = +inf
-                    const float y = v[c] * sc;
-                    sm[c] = fmaf(sm[c], ex2_approx(m[c] - y), 1.f);
-                    m[c] = y;
-                  } else {
-                    sm[c] += ex2_approx(t[c]);
-                  }
-                }
-              }
-            } else {
-#pragma unroll
-              for (int c = 0; c < NQ; ++c) sm[c] += ex2_approx(t[c]);
-            }
+            for (int c = 0; c < NQ; ++c) sm[c] += ex2_approx(t[c]);
           }
         }
       }
@@ -733,6 +682,7 @@ __global__ void __launch_bounds__(kScThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive_cnt(&slot_free[slot], 2);  // two arrivals: this warp stands for its pair
         if (resident_ok && key < k1) {
+          if constexpr (COMBINE) r = fold_split<MEAN>(r_e[key], r);
           r_e[key] = r;
           if (s_e) s_e[key] = ex2_approx(r);
         }
@@ -754,6 +704,7 @@ __global__ void __launch_bounds__(kScThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive_cnt(&slot_free[slot], 2);
         if (have && key < k1) {
+          if constexpr (COMBINE) r = fold_split<MEAN>(r_e[key], r);
           r_e[key] = r;
           if (s_e) s_e[key] = ex2_approx(r);
         }
@@ -779,12 +730,12 @@ __global__ void __launch_bounds__(kScThreads, 1)
 // whose tiles all fit the slot ring, with at least kSlack spare slots where
 // eight CTAs allow it; when not even eight CTAs hold an instance, eight CTAs
 // with streaming slots.  Slot barriers exist for kMaxSlots slots, and tensor
-// memory holds kTmemCols / n_obs_pad of them (at least 4, n_obs_pad <= 128).
+// memory holds kTmemCols / n_cols of them (at least 8: a launch has n_cols <= 64).
 constexpr int kSlack = 1;
 
-Plan plan_score(int L, int n_obs_pad) {
+Plan plan_score(int L, int n_cols) {
   const int U = (L + 31) / 32;
-  int cap = static_cast<int>(kTmemCols) / n_obs_pad;
+  int cap = static_cast<int>(kTmemCols) / n_cols;
   if (cap > kMaxSlots) cap = kMaxSlots;
   const int cmax = U < 8 ? U : 8;  // every CTA owns at least one 32-key unit
   for (int slack = kSlack; slack >= 0; --slack)
@@ -795,14 +746,14 @@ Plan plan_score(int L, int n_obs_pad) {
   return Plan{cmax, cap - 4, 1};
 }
 
-template <int D, int NQ, bool MEAN, bool CAUSAL>
+template <int D, int NQ, bool MEAN, bool CAUSAL, bool COMBINE>
 cudaError_t launch_score_dq(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32,
                             const CUtensorMap& qmap, const ScoreArgs& a, cudaStream_t st) {
   using C = ScoreCfg<D>;
-  const Plan plan = plan_score(a.L, s.n_obs_pad);
-  const size_t smem = C::smem_bytes(s.n_obs_pad, plan.csize);
-  const int n_stages = C::stages(s.n_obs_pad, plan.csize);
-  cudaError_t err = cudaFuncSetAttribute(score_kernel<D, NQ, MEAN, CAUSAL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  const Plan plan = plan_score(a.L, 2 * NQ);
+  const size_t smem = C::smem_bytes(2 * NQ, plan.csize);
+  const int n_stages = C::stages(2 * NQ, plan.csize);
+  cudaError_t err = cudaFuncSetAttribute(score_kernel<D, NQ, MEAN, CAUSAL, COMBINE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
   if (err != cudaSuccess) return err;
   int dev = 0, sms = 0, max_clusters = 0;
@@ -821,28 +772,35 @@ cudaError_t launch_score_dq(const Shape& s, const CUtensorMap& kmap, const CUten
   cfg.numAttrs = 1;
   // one resident wave of clusters, each looping over its share of the instances
   cfg.gridDim = dim3(static_cast<unsigned>(plan.csize * sms));
-  if (cudaOccupancyMaxActiveClusters(&max_clusters, score_kernel<D, NQ, MEAN, CAUSAL>, &cfg) != cudaSuccess || max_clusters < 1) {
+  if (cudaOccupancyMaxActiveClusters(&max_clusters, score_kernel<D, NQ, MEAN, CAUSAL, COMBINE>, &cfg) != cudaSuccess || max_clusters < 1) {
     cudaGetLastError();
     max_clusters = sms / plan.csize > 0 ? sms / plan.csize : 1;
   }
   const int n_clusters = max_clusters < s.n_inst ? max_clusters : s.n_inst;
   cfg.gridDim = dim3(static_cast<unsigned>(n_clusters * plan.csize));
-  return cudaLaunchKernelEx(&cfg, score_kernel<D, NQ, MEAN, CAUSAL>, kmap, kmap32, qmap, s, a, plan, n_stages);
+  return cudaLaunchKernelEx(&cfg, score_kernel<D, NQ, MEAN, CAUSAL, COMBINE>, kmap, kmap32, qmap, s, a, plan, n_stages);
 }
 
 template <int D, bool MEAN, bool CAUSAL>
 cudaError_t launch_score_d(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32, const CUtensorMap& qmap,
                            const ScoreArgs& a, cudaStream_t st) {
-  // query columns of each pass-1 warp: half of the padded query count
-  switch (s.n_obs_pad) {
-    case 16: return launch_score_dq<D, 8, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
-    case 32: return launch_score_dq<D, 16, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
-    case 48: return launch_score_dq<D, 24, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
-    case 64: return launch_score_dq<D, 32, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
-    case 80: return launch_score_dq<D, 40, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
-    case 96: return launch_score_dq<D, 48, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
-    case 112: return launch_score_dq<D, 56, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
-    default: return launch_score_dq<D, 64, MEAN, CAUSAL>(s, kmap, kmap32, qmap, a, st);
+  // query columns of each pass-1 warp: half of this launch's padded query count; a launch after
+  // the first of a column split folds into the scores before it
+  if (a.combine) {
+    switch (a.n_cols) {
+      case 16: return launch_score_dq<D, 8, MEAN, CAUSAL, true>(s, kmap, kmap32, qmap, a, st);
+      case 32: return launch_score_dq<D, 16, MEAN, CAUSAL, true>(s, kmap, kmap32, qmap, a, st);
+      case 48: return launch_score_dq<D, 24, MEAN, CAUSAL, true>(s, kmap, kmap32, qmap, a, st);
+      case 64: return launch_score_dq<D, 32, MEAN, CAUSAL, true>(s, kmap, kmap32, qmap, a, st);
+      default: return cudaErrorInvalidValue;
+    }
+  }
+  switch (a.n_cols) {
+    case 16: return launch_score_dq<D, 8, MEAN, CAUSAL, false>(s, kmap, kmap32, qmap, a, st);
+    case 32: return launch_score_dq<D, 16, MEAN, CAUSAL, false>(s, kmap, kmap32, qmap, a, st);
+    case 48: return launch_score_dq<D, 24, MEAN, CAUSAL, false>(s, kmap, kmap32, qmap, a, st);
+    case 64: return launch_score_dq<D, 32, MEAN, CAUSAL, false>(s, kmap, kmap32, qmap, a, st);
+    default: return cudaErrorInvalidValue;
   }
 }
 

@@ -81,9 +81,12 @@ def test_no_rotation_and_max_queries():
 
 
 @pytest.mark.parametrize("wl", [
-    # 128 scoring queries, 40 tiles: tensor memory holds none of them resident past eight CTAs
+    # 128 scoring queries, 40 tiles: two score launches of 64 queries, each resident in tensor memory
     QWEN3_4B.scaled(name="long_m128_L5000", n_layers=1, batch=1, n_q_heads=64, n_kv_heads=8, window=12,
                     n_beacons=32, L=5000, budget=3000, n_init=64, n_clusters=32),
+    # 128 scoring queries, 235 tiles: both launches stream tiles past the resident ones
+    QWEN3_4B.scaled(name="long_m128_L30000", n_layers=1, batch=1, n_q_heads=64, n_kv_heads=8, window=12,
+                    n_beacons=32, L=30000, budget=20000, n_init=64, n_clusters=32),
     # 48 scoring queries, 157 tiles: resident tiles plus streaming tiles in every CTA
     QWEN3_4B.scaled(name="long_L20000", n_layers=1, batch=1, L=20000, budget=12000),
 ], ids=lambda w: w.name)
@@ -144,6 +147,8 @@ def _shift_positions(inp, W, t_pos, recent_pos):
     (QWEN3_4B.scaled(name="causal_ragged_L300_B40_w16", n_layers=1, batch=1, L=300, budget=40, window=16), 43),
     (QWEN3_4B.scaled(name="causal_long_L20000", n_layers=1, batch=1, L=20000, budget=9000), 44),
     (QWEN3_4B.scaled(name="causal_nb0", n_layers=1, batch=1, L=500, budget=260, n_beacons=0), 45),
+    (QWEN3_4B.scaled(name="causal_m128", n_layers=1, batch=1, n_q_heads=64, n_kv_heads=8, window=12, n_beacons=32,
+                     L=900, budget=600, n_init=64, n_clusters=32), 47),
 ], ids=lambda x: getattr(x, "name", str(x)))
 def test_causal_window(wl, seed, mean):
     _run(wl, seed=seed, mean_agg=mean, causal=True)
@@ -170,6 +175,9 @@ def test_causal_window_positions(case):
     (QWEN3_4B.scaled(name="mean_ragged_L300_B17", n_layers=1, batch=1, L=300, budget=17), 13),
     (QWEN3_4B.scaled(name="mean_long_L20000", n_layers=1, batch=1, L=20000, budget=9000), 14),
     (LLAMA_8B.scaled(name="mean_w0", n_layers=1, batch=1, L=400, budget=200, window=0), 15),
+    (QWEN3_4B.scaled(name="mean_m128", n_layers=1, batch=1, n_q_heads=64, n_kv_heads=8, window=12, n_beacons=32,
+                     L=900, budget=600, n_init=64, n_clusters=32), 16),
+    (QWEN3_4B.scaled(name="mean_m80", n_layers=1, batch=1, window=16, L=700, budget=300), 17),
 ], ids=lambda x: getattr(x, "name", str(x)))
 def test_mean_aggregation(wl, seed):
     _run(wl, seed=seed, mean_agg=True)
