@@ -99,15 +99,12 @@ __global__ void __launch_bounds__(kQobsThreads) qobs_kernel(Shape s, const __nv_
     *reinterpret_cast<uint2*>(out + row * d + i) = *reinterpret_cast<const uint2*>(y1);
     *reinterpret_cast<uint2*>(out + row * d + i + h) = *reinterpret_cast<const uint2*>(y2);
   }
-  if (threadIdx.x < 4) {
-    uint32_t m = 0;
-    for (int bit = 0; bit < 32; ++bit) {
-      const int row = threadIdx.x * 32 + bit;
-      bool v = row < GW;
-      if (!v && row < s.n_obs) v = counts[static_cast<size_t>(e) * s.nb + (row - GW)] > 0;
-      if (v) m |= 1u << bit;
-    }
-    valid[e * 4 + threadIdx.x] = m;
+  if (threadIdx.x < 128) {  // warp w builds mask word w: one row per lane, loads in parallel
+    const int row = threadIdx.x;
+    bool v = row < GW;
+    if (!v && row < s.n_obs) v = counts[static_cast<size_t>(e) * s.nb + (row - GW)] > 0;
+    const uint32_t m = __ballot_sync(0xffffffffu, v);
+    if ((threadIdx.x & 31) == 0) valid[e * 4 + (threadIdx.x >> 5)] = m;
   }
 }
 
