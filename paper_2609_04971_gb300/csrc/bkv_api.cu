@@ -1,7 +1,6 @@
 // C ABI of the BeaconKV compression step (declared in include/bkv.h):
 // argument validation, context and scratch ownership, tensor-map encoding,
 // the rotary table, and kernel launches on the context's stream.
-#include <cudaTypedefs.h>
 
 #include <algorithm>
 #include <cmath>
@@ -114,31 +113,10 @@ void fold_profile(bkv_ctx* c) {
   c->pending.clear();
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q{};
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
-            cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  });
-  return fn;
-}
-
 // 2-D bf16 tensor [rows][d] viewed in boxes of [box_rows][64] with 128-byte swizzle.
 int encode_rows(bkv_ctx* c, CUtensorMap* map, const void* base, uint64_t rows, int d, uint32_t box_rows) {
-  auto enc = tensor_map_encoder();
-  if (!enc) return fail(c, BKV_ECUDA, "cuTensorMapEncodeTiled is unavailable");
-  cuuint64_t dims[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows)};
-  cuuint64_t strides[1] = {static_cast<cuuint64_t>(d) * 2};
-  cuuint32_t box[2] = {64, box_rows};
-  cuuint32_t estr[2] = {1, 1};
-  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  const CUresult r = bkv::encode_rows_bf16(map, base, rows, d, box_rows);
+  if (r == CUDA_ERROR_NOT_FOUND) return fail(c, BKV_ECUDA, "cuTensorMapEncodeTiled is unavailable");
   if (r != CUDA_SUCCESS) return fail(c, BKV_ECUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
   return BKV_OK;
 }

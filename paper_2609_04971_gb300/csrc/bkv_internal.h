@@ -94,6 +94,10 @@ inline void set_causal(ScoreArgs& a, int L, int W, long long t_pos, const int64_
     }
   }
 }
+// Tensor map of a bf16 matrix [rows][d] (row pitch d * 2 bytes) in boxes of [box_rows][64] with the
+// 128-byte swizzle; CUDA_ERROR_NOT_FOUND when the driver has no cuTensorMapEncodeTiled.
+CUresult encode_rows_bf16(CUtensorMap* map, const void* base, uint64_t rows, int d, uint32_t box_rows);
+
 constexpr int kScoreMaxCols = 64;  // scoring queries per score launch (column split beyond)
 // kmap / kmap32: K as [n_inst * cap][d] in 128-row and 32-row boxes of [64]
 // columns (128-byte swizzle); qmap: Qobs as [n_inst * n_obs_pad][d] in boxes
