@@ -14,7 +14,8 @@
 // (about twice the bound on their difference's error: 2^-17 |q| per dot from
 // the hi/lo split, 128 fp32 accumulation steps), the query is re-decided
 // exactly: the beacon maximising (q . c_b) / |c_b| in double-float arithmetic
-// (exact products, TwoSum accumulation, 1 / |c_b| rounded from fp64), which
+// (exact products, TwoSum accumulation, 1 / |c_b| from a double-float sum of
+// squares and one Newton step, to about 2^-44 relative), which
 // agrees with the cosine (q . c_b) / (|q| |c_b|) evaluated in fp64 except at
 // ties below ~1e-12 (the lowest beacon wins ties).  Zero queries and instances
 // without a valid beacon give -1.
@@ -99,12 +100,6 @@ __device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32
                : "memory");
 }
 
-__device__ __forceinline__ double warp_sum_f64(double v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-
 // round(x * 2^40) of the bf16 value whose bits sit in the upper half of
 // `hi16` (lower half zero): the scale is added to the fp32 exponent field
 // (exact for |x| < 2^88; a zero or subnormal x becomes a value below 2^-80,
@@ -166,6 +161,17 @@ __device__ __forceinline__ DF df_mul(DF a, DF b) {
 }
 
 __device__ __forceinline__ bool df_gt(DF a, DF b) { return a.hi > b.hi || (a.hi == b.hi && a.lo > b.lo); }
+
+// 1 / sqrt(a) for a double-float a > 0: the fp32 estimate y = rsqrtf(a.hi) (about 2^-22
+// relative) refined by one Newton-Raphson step for f(y) = 1 / y^2 - a,
+// y' = y + y (1 - a y^2) / 2, with the residual 1 - a y^2 formed in double-float
+// arithmetic; the result holds about 44 significant bits.  fp64 is slow on this part.
+__device__ __forceinline__ DF df_rsqrt(DF a) {
+  const float y = rsqrtf(a.hi);
+  const DF ay2 = df_mul(a, df_two_prod(y, y));
+  const float r = __fadd_rn(__fadd_rn(1.f, -ay2.hi), -ay2.lo);  // 1 - a y^2, about 2^-22: two roundings suffice
+  return df_add(DF{y, 0.f}, df_two_prod(y, 0.5f * r));
+}
 
 // Exact sums of bf16 values without a 64-bit conversion per element: x is
 // split into xh = x rounded to a multiple of 2^-3, xm = the rest rounded to a
@@ -627,13 +633,13 @@ __global__ void __launch_bounds__(kUThreads, 1)
       for (int b = wk; b < nbp; b += kKeepers) {
         float c[D / 32];
         float n2 = 0.f;
-        double n2d = 0.0;
+        DF n2d{0.f, 0.f};  // the exact products c^2 summed in double-float arithmetic
         int nz = 0;
 #pragma unroll
         for (int k = 0; k < D / 32; ++k) {
           c[k] = b < nb ? cs[b * D + lane + 32 * k] : 0.f;
           n2 = fmaf(c[k], c[k], n2);
-          n2d = fma(static_cast<double>(c[k]), static_cast<double>(c[k]), n2d);
+          n2d = df_add(n2d, df_two_prod(c[k], c[k]));
           nz |= (c[k] != 0.f);
         }
 #pragma unroll
@@ -641,7 +647,9 @@ __global__ void __launch_bounds__(kUThreads, 1)
           n2 += __shfl_xor_sync(0xffffffffu, n2, o);
           nz |= __shfl_xor_sync(0xffffffffu, nz, o);
         }
-        n2d = warp_sum_f64(n2d);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+          n2d = df_add(n2d, DF{__shfl_xor_sync(0xffffffffu, n2d.hi, o), __shfl_xor_sync(0xffffffffu, n2d.lo, o)});
         const bool ok = b < nb && cnt_old[pb][b] > 0 && nz;
         const float inv = ok ? rsqrtf(n2) : 0.f;
 #pragma unroll
@@ -655,10 +663,17 @@ __global__ void __launch_bounds__(kUThreads, 1)
         }
         if (lane == 0 && b < nb) {
           bvalid[pb][b] = ok;
-          const double inv = ok ? __drcp_rn(sqrt(n2d)) : 0.0;
-          const float inv_hi = __double2float_rn(inv);
-          cninv[pb][b] = DF{inv_hi, __double2float_rn(inv - static_cast<double>(inv_hi))};
-          if (ok && !(n2 > 1e-30f && n2 < 1e30f)) degenerate[pb] = 1;
+          const bool plain = n2 > 1e-30f && n2 < 1e30f;  // far from fp32 over- and underflow
+          DF inv_df{0.f, 0.f};
+          if (ok && plain) {
+            inv_df = df_rsqrt(n2d);
+          } else if (ok) {  // extreme norms (rare): the same quantity in fp64
+            const double inv = __drcp_rn(sqrt(static_cast<double>(n2d.hi) + static_cast<double>(n2d.lo)));
+            const float inv_hi = __double2float_rn(inv);
+            inv_df = DF{inv_hi, __double2float_rn(inv - static_cast<double>(inv_hi))};
+          }
+          cninv[pb][b] = inv_df;
+          if (ok && !plain) degenerate[pb] = 1;
         }
       }
       fence_proxy_async_smem();  // generic-proxy writes, read next by the tensor cores
