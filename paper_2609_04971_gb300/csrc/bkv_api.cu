@@ -347,6 +347,12 @@ int bkv_update_beacons(bkv_ctx* ctx, const void* q_new, int32_t n_new, int32_t* 
     cudaError_t e = bkv::launch_cfps(s.d, ca, ctx->stream);
     return e == cudaSuccess ? BKV_OK : cuda_fail(ctx, e, "continual FPS update launch");
   }
+  if (s.G * n_new <= bkv::kUpdateSmallMaxRows) {  // a decode step or a few: one warp per instance
+    ProfScope ps(ctx, BKV_K_UPDATE);
+    cudaError_t e = bkv::launch_update_small(s, static_cast<const __nv_bfloat16*>(q_new), n_new, ctx->cent, ctx->sums,
+                                             ctx->counts, assign_out, ctx->stream);
+    return e == cudaSuccess ? BKV_OK : cuda_fail(ctx, e, "update launch");
+  }
   // a tile is at most 128 queries of one instance: boxes no taller than that
   const uint64_t q_rows = static_cast<uint64_t>(s.n_inst) * s.G * n_new;
   uint64_t box_rows = (static_cast<uint64_t>(s.G) * n_new + 7) / 8 * 8;

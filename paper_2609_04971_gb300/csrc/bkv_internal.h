@@ -56,6 +56,11 @@ cudaError_t launch_fps_init(const Shape& s, const __nv_bfloat16* q_init, int n_i
 // error word.
 cudaError_t launch_update(const Shape& s, const CUtensorMap& qmap, int box_rows, int n_new, float* cent,
                           double* sums, long long* counts, int* assign_out, int* err, cudaStream_t st);
+// A few queries per instance (G * n_new <= kUpdateSmallMaxRows, e.g. one decode step): one warp
+// per instance, the same decisions and sums as launch_update (k_update_small.cu).
+constexpr int kUpdateSmallMaxRows = 32;
+cudaError_t launch_update_small(const Shape& s, const __nv_bfloat16* q_new, int n_new, float* cent, double* sums,
+                                long long* counts, int* assign_out, cudaStream_t st);
 
 // ---- compression (k_qobs.cu, k_score.cu, k_select_gather.cu)
 // rope: [W + 1][d / 2] fp64 (cos, sin) pairs, immediately followed by the same

@@ -40,6 +40,7 @@
 // (accumulators double-buffered by instance).  All waits are bounded.
 #include "bkv_device.cuh"
 #include "bkv_internal.h"
+#include "k_update_math.cuh"
 
 namespace bkv {
 namespace {
@@ -52,7 +53,6 @@ constexpr int kQTile = 128;                 // queries per tile (MMA M)
 constexpr uint32_t kQBox = 128 * 128;       // [128 rows][64 bf16] swizzled box slot
 constexpr int kUMaxStages = 8;
 constexpr size_t kUSmemBudget = 216 * 1024;
-constexpr float kMarginRel = 1e-4f;
 constexpr int kGroup = 4;  // rows an accumulator lane sums per step when they share a beacon
 
 struct UpdArgs {
@@ -128,67 +128,6 @@ __device__ __forceinline__ void add_fixed(long long (&s)[kCols], const unsigned 
     s[0] += bf16_fixed40(w << 16);
     s[1] += bf16_fixed40(w & 0xffff0000u);
   }
-}
-
-// Double-float arithmetic (an unevaluated sum hi + lo of two fp32 values,
-// about 48 significant bits) for the exact re-decisions: fp64 is slow on
-// this part.  TwoSum (Knuth) and the FMA-based exact product.
-struct DF {
-  float hi, lo;
-};
-
-__device__ __forceinline__ DF df_add(DF a, DF b) {
-  const float s = __fadd_rn(a.hi, b.hi);
-  const float bb = __fadd_rn(s, -a.hi);
-  const float err = __fadd_rn(__fadd_rn(a.hi, -__fadd_rn(s, -bb)), __fadd_rn(b.hi, -bb));
-  const float lo = __fadd_rn(__fadd_rn(a.lo, b.lo), err);
-  const float t = __fadd_rn(s, lo);
-  return DF{t, __fadd_rn(lo, -__fadd_rn(t, -s))};
-}
-
-__device__ __forceinline__ DF df_two_prod(float a, float b) {
-  const float p = __fmul_rn(a, b);
-  return DF{p, __fmaf_rn(a, b, -p)};
-}
-
-__device__ __forceinline__ DF df_mul(DF a, DF b) {
-  const float p = __fmul_rn(a.hi, b.hi);
-  float e = __fmaf_rn(a.hi, b.hi, -p);
-  e = __fmaf_rn(a.hi, b.lo, e);
-  e = __fmaf_rn(a.lo, b.hi, e);
-  const float t = __fadd_rn(p, e);
-  return DF{t, __fadd_rn(e, -__fadd_rn(t, -p))};
-}
-
-__device__ __forceinline__ bool df_gt(DF a, DF b) { return a.hi > b.hi || (a.hi == b.hi && a.lo > b.lo); }
-
-// 1 / sqrt(a) for a double-float a > 0: the fp32 estimate y = rsqrtf(a.hi) (about 2^-22
-// relative) refined by one Newton-Raphson step for f(y) = 1 / y^2 - a,
-// y' = y + y (1 - a y^2) / 2, with the residual 1 - a y^2 formed in double-float
-// arithmetic; the result holds about 44 significant bits.  fp64 is slow on this part.
-__device__ __forceinline__ DF df_rsqrt(DF a) {
-  const float y = rsqrtf(a.hi);
-  const DF ay2 = df_mul(a, df_two_prod(y, y));
-  const float r = __fadd_rn(__fadd_rn(1.f, -ay2.hi), -ay2.lo);  // 1 - a y^2, about 2^-22: two roundings suffice
-  return df_add(DF{y, 0.f}, df_two_prod(y, 0.5f * r));
-}
-
-// Exact sums of bf16 values without a 64-bit conversion per element: x is
-// split into xh = x rounded to a multiple of 2^-3, xm = the rest rounded to a
-// multiple of 2^-20 and xl = what remains (magic-number rounding, fp32 adds
-// only, two columns per paired-fp32 instruction); each part's fp32 running
-// sum is exact over up to 128 values with |x| < 2^14 (xl is exact for
-// |x| >= 2^-31).  `fixed40` turns the three sums into round(sum * 2^40) with
-// 32-bit conversions.
-struct Parts {
-  float h, m, l;
-};
-
-__device__ __forceinline__ long long fixed40(const Parts& p) {
-  const long long h = static_cast<long long>(__float2int_rn(p.h * 8.0f)) << 37;
-  const long long m = static_cast<long long>(__float2int_rn(p.m * 1048576.0f)) << 20;
-  const long long l = static_cast<long long>(__float2int_rn(p.l * 274877906944.0f)) << 2;
-  return h + m + l;
 }
 
 // The same split for two adjacent columns at once, on packed f32x2 values
@@ -489,29 +428,12 @@ __global__ void __launch_bounds__(kUThreads, 1)
         for (int k = ws; k < nr; k += kScreeners) {
           const int r = refine_t[ob][k];
           float x[D / 32];
-          int nz = 0;
 #pragma unroll
-          for (int j = 0; j < D / 32; ++j) {
+          for (int j = 0; j < D / 32; ++j)
             x[j] = __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(qs + sw128_offset(r, lane + 32 * j, kQBox)));
-            nz |= x[j] != 0.f;
-          }
-          DF b1{-INFINITY, 0.f};
-          int best_b = -1;
-          if (__any_sync(0xffffffffu, nz))  // a zero query stays unassigned
-            for (int b = 0; b < nb; ++b) {
-              if (!bvalid[pb][b]) continue;
-              DF dt{0.f, 0.f};
-#pragma unroll
-              for (int j = 0; j < D / 32; ++j) dt = df_add(dt, df_two_prod(x[j], cent_i[b * D + lane + 32 * j]));
-#pragma unroll
-              for (int o = 16; o > 0; o >>= 1)
-                dt = df_add(dt, DF{__shfl_xor_sync(0xffffffffu, dt.hi, o), __shfl_xor_sync(0xffffffffu, dt.lo, o)});
-              const DF cs = df_mul(dt, cninv[pb][b]);
-              if (best_b < 0 || df_gt(cs, b1)) {
-                b1 = cs;
-                best_b = b;
-              }
-            }
+          const int best_b = exact_decision<D>(
+              x, nb, [&](int b, int col) { return cent_i[b * D + col]; }, [&](int b) { return bvalid[pb][b] != 0; },
+              cninv[pb]);
           if (lane == 0) {
             if (assign_t) assign_t[r] = best_b;
             if (best_b >= 0) atomicAdd(&add_cnt[pb][best_b], 1);
@@ -663,17 +585,11 @@ __global__ void __launch_bounds__(kUThreads, 1)
         }
         if (lane == 0 && b < nb) {
           bvalid[pb][b] = ok;
-          const bool plain = n2 > 1e-30f && n2 < 1e30f;  // far from fp32 over- and underflow
+          bool plain = true;
           DF inv_df{0.f, 0.f};
-          if (ok && plain) {
-            inv_df = df_rsqrt(n2d);
-          } else if (ok) {  // extreme norms (rare): the same quantity in fp64
-            const double inv = __drcp_rn(sqrt(static_cast<double>(n2d.hi) + static_cast<double>(n2d.lo)));
-            const float inv_hi = __double2float_rn(inv);
-            inv_df = DF{inv_hi, __double2float_rn(inv - static_cast<double>(inv_hi))};
-          }
+          if (ok) inv_df = centroid_inv_norm(n2d, n2, plain);
           cninv[pb][b] = inv_df;
-          if (ok && !plain) degenerate[pb] = 1;
+          if (!plain) degenerate[pb] = 1;
         }
       }
       fence_proxy_async_smem();  // generic-proxy writes, read next by the tensor cores

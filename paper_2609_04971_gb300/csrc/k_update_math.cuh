@@ -1,0 +1,131 @@
+// Arithmetic shared by the beacon-update kernels (k_update.cu for many queries
+// per instance, k_update_small.cu for a few): double-float operations, the
+// exact per-column sums of bf16 values, the norm data of a centroid and the
+// exact re-decision of a close assignment.  Both kernels take their decisions
+// and sums with these same operations.
+#pragma once
+#include "bkv_device.cuh"
+
+namespace bkv {
+namespace {
+
+// A query is re-decided exactly when its best and second-best screened unit-centroid
+// dots differ by at most this fraction of |q| (about twice the screening error bound).
+constexpr float kMarginRel = 1e-4f;
+
+// Double-float arithmetic (an unevaluated sum hi + lo of two fp32 values,
+// about 48 significant bits) for the exact re-decisions: fp64 is slow on
+// this part.  TwoSum (Knuth) and the FMA-based exact product.
+struct DF {
+  float hi, lo;
+};
+
+__device__ __forceinline__ DF df_add(DF a, DF b) {
+  const float s = __fadd_rn(a.hi, b.hi);
+  const float bb = __fadd_rn(s, -a.hi);
+  const float err = __fadd_rn(__fadd_rn(a.hi, -__fadd_rn(s, -bb)), __fadd_rn(b.hi, -bb));
+  const float lo = __fadd_rn(__fadd_rn(a.lo, b.lo), err);
+  const float t = __fadd_rn(s, lo);
+  return DF{t, __fadd_rn(lo, -__fadd_rn(t, -s))};
+}
+
+__device__ __forceinline__ DF df_two_prod(float a, float b) {
+  const float p = __fmul_rn(a, b);
+  return DF{p, __fmaf_rn(a, b, -p)};
+}
+
+__device__ __forceinline__ DF df_mul(DF a, DF b) {
+  const float p = __fmul_rn(a.hi, b.hi);
+  float e = __fmaf_rn(a.hi, b.hi, -p);
+  e = __fmaf_rn(a.hi, b.lo, e);
+  e = __fmaf_rn(a.lo, b.hi, e);
+  const float t = __fadd_rn(p, e);
+  return DF{t, __fadd_rn(e, -__fadd_rn(t, -p))};
+}
+
+__device__ __forceinline__ bool df_gt(DF a, DF b) { return a.hi > b.hi || (a.hi == b.hi && a.lo > b.lo); }
+
+// 1 / sqrt(a) for a double-float a > 0: the fp32 estimate y = rsqrtf(a.hi) (about 2^-22
+// relative) refined by one Newton-Raphson step for f(y) = 1 / y^2 - a,
+// y' = y + y (1 - a y^2) / 2, with the residual 1 - a y^2 formed in double-float
+// arithmetic; the result holds about 44 significant bits.  fp64 is slow on this part.
+__device__ __forceinline__ DF df_rsqrt(DF a) {
+  const float y = rsqrtf(a.hi);
+  const DF ay2 = df_mul(a, df_two_prod(y, y));
+  const float r = __fadd_rn(__fadd_rn(1.f, -ay2.hi), -ay2.lo);  // 1 - a y^2, about 2^-22: two roundings suffice
+  return df_add(DF{y, 0.f}, df_two_prod(y, 0.5f * r));
+}
+
+// Exact sums of bf16 values without a 64-bit conversion per element: x is
+// split into xh = x rounded to a multiple of 2^-3, xm = the rest rounded to a
+// multiple of 2^-20 and xl = what remains (magic-number rounding, fp32 adds
+// only, two columns per paired-fp32 instruction); each part's fp32 running
+// sum is exact over up to 128 values with |x| < 2^14 (xl is exact for
+// |x| >= 2^-31).  `fixed40` turns the three sums into round(sum * 2^40) with
+// 32-bit conversions.
+struct Parts {
+  float h, m, l;
+};
+
+__device__ __forceinline__ long long fixed40(const Parts& p) {
+  const long long h = static_cast<long long>(__float2int_rn(p.h * 8.0f)) << 37;
+  const long long m = static_cast<long long>(__float2int_rn(p.m * 1048576.0f)) << 20;
+  const long long l = static_cast<long long>(__float2int_rn(p.l * 274877906944.0f)) << 2;
+  return h + m + l;
+}
+
+// Splits the bf16 value x (exact in fp32) into the three parts and adds them.
+__device__ __forceinline__ void parts_add(Parts& p, float x) {
+  const float xh = __fadd_rn(__fadd_rn(x, 1572864.f), -1572864.f);  // multiple of 2^-3 (1.5 * 2^20 magic)
+  const float r = __fadd_rn(x, -xh);
+  const float xm = __fadd_rn(__fadd_rn(r, 12.f), -12.f);  // multiple of 2^-20 (1.5 * 2^3 magic)
+  p.h = __fadd_rn(p.h, xh);
+  p.m = __fadd_rn(p.m, xm);
+  p.l = __fadd_rn(p.l, __fadd_rn(r, -xm));
+}
+
+// 1 / |c| of a centroid from its double-float sum of squares n2d (fp32 value n2),
+// and whether |c|^2 is far from fp32 over- and underflow (`plain`); outside that
+// range the same quantity is taken in fp64.
+__device__ __forceinline__ DF centroid_inv_norm(DF n2d, float n2, bool& plain) {
+  plain = n2 > 1e-30f && n2 < 1e30f;
+  if (plain) return df_rsqrt(n2d);
+  const double inv = __drcp_rn(sqrt(static_cast<double>(n2d.hi) + static_cast<double>(n2d.lo)));
+  const float inv_hi = __double2float_rn(inv);
+  return DF{inv_hi, __double2float_rn(inv - static_cast<double>(inv_hi))};
+}
+
+// Exact assignment of one query (warp-wide; x holds this lane's elements lane + 32 j):
+// the valid beacon maximising (q . c_b) * (1 / |c_b|) in double-float arithmetic (exact
+// products, TwoSum accumulation, then a butterfly over the lanes), ties to the lower
+// beacon; -1 for a zero query or when no beacon is valid.  cent_at(b, col) reads centroid
+// b; valid(b) is warp-uniform.
+template <int D, typename CentAt, typename Valid>
+__device__ __forceinline__ int exact_decision(const float (&x)[D / 32], int nb, CentAt cent_at, Valid valid,
+                                              const DF* cninv) {
+  const int lane = threadIdx.x & 31;
+  int nz = 0;
+#pragma unroll
+  for (int j = 0; j < D / 32; ++j) nz |= x[j] != 0.f;
+  DF b1{-INFINITY, 0.f};
+  int best_b = -1;
+  if (__any_sync(0xffffffffu, nz))
+    for (int b = 0; b < nb; ++b) {
+      if (!valid(b)) continue;
+      DF dt{0.f, 0.f};
+#pragma unroll
+      for (int j = 0; j < D / 32; ++j) dt = df_add(dt, df_two_prod(x[j], cent_at(b, lane + 32 * j)));
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1)
+        dt = df_add(dt, DF{__shfl_xor_sync(0xffffffffu, dt.hi, o), __shfl_xor_sync(0xffffffffu, dt.lo, o)});
+      const DF cs = df_mul(dt, cninv[b]);
+      if (best_b < 0 || df_gt(cs, b1)) {
+        b1 = cs;
+        best_b = b;
+      }
+    }
+  return best_b;
+}
+
+}  // namespace
+}  // namespace bkv

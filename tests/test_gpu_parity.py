@@ -122,6 +122,35 @@ def test_full_size_sampled(wl):
     assert run.counts1.sum(axis=1).min() == wl.group * (wl.n_init * 0 + wl.n_new) + wl.n_beacons
 
 
+# ---------------------------------------------------------------- a few queries per instance (decode steps)
+@pytest.mark.parametrize("wl", [
+    QWEN3_4B.scaled(name="few_n1", n_layers=1, batch=2, n_new=1),   # 4 rows per instance: one decode step
+    QWEN3_4B.scaled(name="few_n3", n_layers=1, batch=2, n_new=3),   # 12 rows
+    QWEN3_4B.scaled(name="few_n8", n_layers=1, batch=2, n_new=8),   # 32 rows: the largest few-query call
+    QWEN3_4B.scaled(name="few_n9", n_layers=1, batch=2, n_new=9),   # 36 rows: the batched kernel
+    TINY.scaled(name="few_d64_n4", n_new=4),                        # head_dim 64, 8 rows
+    QWEN3_4B.scaled(name="few_g8_nb32_n4", n_layers=1, batch=1, n_q_heads=64, n_kv_heads=8, window=12, n_beacons=32,
+                    L=700, budget=500, n_init=64, n_clusters=32, n_new=4),   # 32 rows, 32 beacons
+    QWEN3_4B.scaled(name="qwen3_4b_decode_step", n_new=1),          # all 4608 instances, sampled
+], ids=lambda w: w.name)
+def test_few_queries_per_instance(wl):
+    sample = None
+    if wl.n_inst > 64:
+        rng = np.random.default_rng(1)
+        sample = np.unique(np.concatenate([[0, wl.n_inst - 1], rng.choice(wl.n_inst, 6, replace=False)]))
+    _run(wl, seed=wl.n_new + 30, sample=sample)
+
+
+def test_few_queries_with_zero_queries():
+    """Zero queries stay unassigned (-1) and add nothing, in the few-query kernel."""
+    wl = QWEN3_4B.scaled(name="few_zero", n_layers=1, batch=1, n_new=2)
+    from paper_2609_04971_gb300 import synth
+    inp = synth.step_inputs(wl, 33, torch.device("cuda"))
+    inp["q_new"][:, :, ::3, 1, :] = 0
+    run, _ = _run(wl, inputs=inp)
+    assert (run.assign == -1).sum() > 0
+
+
 def test_deterministic_across_runs():
     wl = QWEN3_4B.scaled(name="det", n_layers=1, batch=2, L=900, budget=500)
     a = P.run_gpu(wl, seed=12)
