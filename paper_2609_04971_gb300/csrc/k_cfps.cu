@@ -24,7 +24,8 @@
 // latency is hidden.
 //
 // The same warp routine serves three calls:
-//   update   append the call's queries in order; whenever the buffer holds
+//   update   append the call's queries in order (a call that does not fill the
+//            buffer only copies them behind its rows); whenever the buffer holds
 //            b_max = b_min + window rows, replace it by the FPS selection of
 //            b_min of them, in pick order;
 //   beacons  the beacons of a compress: the FPS selection of min(b_min, size)
@@ -289,6 +290,15 @@ __global__ void __launch_bounds__(32 * kHeadsPerCta, R == 16 ? 2 : 1) cfps_kerne
   // the rows to add, in order: update: the buffer's own rows (their cosines are rebuilt), then
   // the new queries; beacons: the buffer's rows; merge: this compress's beacons, then the window
   const int n_old = min(max(a.size[h], 0), a.b_max);
+  if (MODE == kCfpsUpdate && n_old + a.n_q < a.b_max) {
+    // the buffer does not fill: the new queries are appended in order and nothing is compressed
+    const int words = a.n_q * D / 2;  // 32-bit words of the new rows
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(qh);
+    uint32_t* dst = reinterpret_cast<uint32_t*>(buf + static_cast<size_t>(n_old) * D);
+    for (int i = lane; i < words; i += 32) dst[i] = src[i];
+    if (lane == 0) a.size[h] = n_old + a.n_q;
+    return;
+  }
   int nbc = 0;
   if (MODE == kCfpsMerge)
     for (int t = 0; t < a.b_min; ++t) nbc += bcnt[t] != 0;
