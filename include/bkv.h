@@ -35,7 +35,9 @@
  * Streams.  All work is enqueued on the CUDA stream given to bkv_create (or
  * bkv_set_stream); calls return before it completes.  Outputs are valid once
  * that stream has been synchronised (bkv_sync does so and reports device-side
- * errors).  One context must not be used from two host threads at once.
+ * errors).  bkv_compress stages its rotary table in one of four pinned host
+ * buffers and waits only when the stream is more than four compress calls
+ * behind.  One context must not be used from two host threads at once.
  *
  * Errors.  Every call returns BKV_OK (0) or a negative code; nothing throws.
  * Argument errors are detected on the host before any work is enqueued and

@@ -38,7 +38,13 @@ struct bkv_ctx {
   float* rscore = nullptr;        // [n_inst][cap]
   double2* rope = nullptr;        // [W + 1][d / 2] fp64 (cos, sin), then the same table in fp32
   int* err = nullptr;             // device error word
-  std::vector<double2> rope_host;  // fp64 entries followed by fp32 entries (packed two per double2)
+  // pinned host staging of the rotary table, a ring of kRopeSlots: a compress fills the next slot
+  // and uploads it asynchronously; the slot is refilled only after its upload's event completed
+  static constexpr int kRopeSlots = 4;
+  double2* rope_pinned[kRopeSlots] = {};
+  cudaEvent_t rope_ev[kRopeSlots] = {};
+  bool rope_used[kRopeSlots] = {};
+  int rope_next = 0;
   std::string last_error;
   // per-kernel timing
   struct Rec {
@@ -178,6 +184,10 @@ void free_all(bkv_ctx* c) {
   cudaFree(c->rscore);
   cudaFree(c->rope);
   cudaFree(c->err);
+  for (int i = 0; i < bkv_ctx::kRopeSlots; ++i) {
+    if (c->rope_pinned[i]) cudaFreeHost(c->rope_pinned[i]);
+    if (c->rope_ev[i]) cudaEventDestroy(c->rope_ev[i]);
+  }
 }
 
 }  // namespace
@@ -253,7 +263,17 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
     delete c;
     return BKV_ECUDA;
   }
-  c->rope_host.resize(static_cast<size_t>(s.W + 1) * (s.d / 2) * 3 / 2 + 1);
+  const size_t rope_bytes = sizeof(double2) * (static_cast<size_t>(s.W + 1) * (s.d / 2) * 3 / 2 + 1);
+  for (int i = 0; i < bkv_ctx::kRopeSlots; ++i) {
+    if ((e = cudaMallocHost(reinterpret_cast<void**>(&c->rope_pinned[i]), rope_bytes)) != cudaSuccess ||
+        (e = cudaEventCreateWithFlags(&c->rope_ev[i], cudaEventDisableTiming)) != cudaSuccess) {
+      const int code = (e == cudaErrorMemoryAllocation) ? BKV_ENOMEM : BKV_ECUDA;
+      cudaGetLastError();
+      free_all(c);
+      delete c;
+      return code;
+    }
+  }
   *out = c;
   return BKV_OK;
 }
@@ -398,19 +418,27 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
   const int rotate = theta != 0.0;
   if (rotate) {
     const size_t n = static_cast<size_t>(s.W + 1) * h;
-    float2* tab32 = reinterpret_cast<float2*>(ctx->rope_host.data() + n);
+    const int rs = ctx->rope_next;
+    ctx->rope_next = (rs + 1) % bkv_ctx::kRopeSlots;
+    if (ctx->rope_used[rs] && (e = cudaEventSynchronize(ctx->rope_ev[rs])) != cudaSuccess)
+      return cuda_fail(ctx, e, "rope staging wait");
+    double2* tab = ctx->rope_pinned[rs];
+    float2* tab32 = reinterpret_cast<float2*>(tab + n);
     for (int slot = 0; slot <= s.W; ++slot) {
       const double pos = static_cast<double>(slot < s.W ? recent_pos[slot] : t_pos);
       for (int i = 0; i < h; ++i) {
         const double inv_freq = std::pow(theta, -static_cast<double>(2 * i) / static_cast<double>(s.d));
         const double ang = pos * inv_freq;
         const double c = std::cos(ang), sn = std::sin(ang);
-        ctx->rope_host[static_cast<size_t>(slot) * h + i] = make_double2(c, sn);
+        tab[static_cast<size_t>(slot) * h + i] = make_double2(c, sn);
         tab32[static_cast<size_t>(slot) * h + i] = make_float2(static_cast<float>(c), static_cast<float>(sn));
       }
     }
-    e = cudaMemcpyAsync(ctx->rope, ctx->rope_host.data(), sizeof(double2) * n + sizeof(float2) * n,
-                        cudaMemcpyHostToDevice, ctx->stream);
+    // pinned source: the copy is asynchronous, and the slot is not refilled before its event
+    e = cudaMemcpyAsync(ctx->rope, tab, sizeof(double2) * n + sizeof(float2) * n, cudaMemcpyHostToDevice,
+                        ctx->stream);
+    if (e == cudaSuccess) e = cudaEventRecord(ctx->rope_ev[rs], ctx->stream);
+    ctx->rope_used[rs] = true;
     if (e != cudaSuccess) return cuda_fail(ctx, e, "rope table upload");
   }
   bkv::CfpsArgs ca{};
