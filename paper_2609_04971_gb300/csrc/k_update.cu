@@ -27,8 +27,9 @@
 // exact for 2^-31 <= |x| < 2^14, the conversion to fixed point per beacon
 // change rather than per element); re-decided rows are converted directly.
 // The per-call sum is exact and independent of the order.  It is then
-// added once to the fp64 running sum, and c = fp32(sum * (1 / count)) in
-// fp64, within one fp32 ulp of fp32(sum / count).
+// added once to the fp64 running sum (the only fp64 operation per element
+// besides the int64 conversion), and c = fp32(sum / count) to within one fp32
+// ulp from double-float arithmetic on the sum's bits.
 //
 // Warp roles (26 warps): warp 0 TMA producer; warp 1 TMEM allocation and MMA
 // issue; warps 2..5 screeners (one per TMEM lane quarter: decisions, the
@@ -187,7 +188,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
   __shared__ int bvalid[2][kMaxBeacons];
   __shared__ DF cninv[2][kMaxBeacons];  // 1 / |c_b| as a double-float
   __shared__ long long cnt_old[2][kMaxBeacons];
-  __shared__ double rcp_sh[kMaxBeacons];
+  __shared__ DF rcp_sh[kMaxBeacons];  // 1 / count after this call, as a double-float
   __shared__ int degenerate[2];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -602,16 +603,16 @@ __global__ void __launch_bounds__(kUThreads, 1)
       long long* acc_i = acc + pb * cells;
       mbar_wait(&accdone[pb], (idx >> 1) & 1, abort_flag, a.err, kDevTimeoutEpilogue);
       mbar_wait(&sbar, idx & 1, abort_flag, a.err, kDevTimeoutEpilogue);
-      if (tk < nb) rcp_sh[tk] = __drcp_rn(static_cast<double>(cnt_old[pb][tk] + add_cnt[pb][tk]));
+      if (tk < nb) rcp_sh[tk] = count_reciprocal(cnt_old[pb][tk] + add_cnt[pb][tk]);
       named_barrier(3, 32 * kKeepers);
       for (int c = tk; c < cells; c += 32 * kKeepers) {
         const int b = c / D, col = c - b * D;
         const int ai = b * D + (col % kCols) * 32 + col / kCols;  // the accumulator cell of (b, col)
         if (add_cnt[pb][b] > 0) {
           const size_t gi = static_cast<size_t>(e) * cells + c;
-          const double s_new = __dadd_rn(sums_sm[c], static_cast<double>(acc_i[ai]) * 0x1p-40);
+          const double s_new = __dadd_rn(sums_sm[c], fixed40_to_double(acc_i[ai]));
           a.sums[gi] = s_new;
-          a.cent[gi] = __double2float_rn(__dmul_rn(s_new, rcp_sh[b]));
+          a.cent[gi] = centroid_value(s_new, rcp_sh[b]);
         }
         acc_i[ai] = 0;  // the cell this thread read: no other thread touches it
       }

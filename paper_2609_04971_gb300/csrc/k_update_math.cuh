@@ -95,6 +95,57 @@ __device__ __forceinline__ DF centroid_inv_norm(DF n2d, float n2, bool& plain) {
   return DF{inv_hi, __double2float_rn(inv - static_cast<double>(inv_hi))};
 }
 
+// The fold of a call's exact sum into the running state.  acc * 2^-40 as a double: one
+// round-to-nearest conversion of the int64 (exact below 2^53), the power of two applied to
+// the exponent field (|acc| >= 1 keeps the result normal).
+__device__ __forceinline__ double fixed40_to_double(long long acc) {
+  if (acc == 0) return 0.0;
+  return __longlong_as_double(__double_as_longlong(__ll2double_rn(acc)) - (40LL << 52));
+}
+
+// 1 / n for a count n >= 1 as a double-float: the correctly rounded fp32 reciprocal of n
+// refined by one Newton-Raphson step r' = r + r (1 - n r), the residual formed exactly.
+__device__ __forceinline__ DF count_reciprocal(long long n) {
+  const float nf = static_cast<float>(n);                      // n rounded (exact below 2^24)
+  const float nl = static_cast<float>(n - static_cast<long long>(nf));
+  const float r = __frcp_rn(nf);
+  const float p = __fmul_rn(nf, r);
+  const float pe = __fmaf_rn(nl, r, __fmaf_rn(nf, r, -p));     // n r - p
+  const float e = __fadd_rn(__fadd_rn(1.f, -p), -pe);          // 1 - n r (1 - p is exact: p is near 1)
+  const float d = __fmul_rn(r, e);
+  const float hi = __fadd_rn(r, d);
+  return DF{hi, __fadd_rn(d, -__fadd_rn(hi, -r))};
+}
+
+// 2^k as a float, for -126 <= k <= 127.
+__device__ __forceinline__ float pow2f(int k) { return __uint_as_float(static_cast<uint32_t>(k + 127) << 23); }
+
+// fp32(s * (1 / n)) from the running sum s (fp64) and rcp = count_reciprocal(n), without fp64
+// arithmetic: s is split into hi (its significand rounded to 24 bits) and lo (the remainder,
+// rounded to fp32) by integer operations on its bits, multiplied by rcp as double-floats and
+// rounded once to fp32; within one fp32 ulp of fp32(s / n).  |s| outside [2^-70, 2^100]
+// (and zero) takes the fp64 route.
+__device__ __forceinline__ float centroid_value(double s, DF rcp) {
+  const unsigned long long bits = static_cast<unsigned long long>(__double_as_longlong(s));
+  const int e = static_cast<int>((bits >> 52) & 0x7ff);
+  if (e < 1023 - 70 || e > 1023 + 100)
+    return __double2float_rn(__dmul_rn(s, __dadd_rn(static_cast<double>(rcp.hi), static_cast<double>(rcp.lo))));
+  const unsigned long long m = (bits & ((1ull << 52) - 1)) | (1ull << 52);  // 53-bit significand
+  const unsigned long long m_hi = (m + (1ull << 28) - 1 + ((m >> 29) & 1)) >> 29;  // m / 2^29, nearest even
+  const long long rem = static_cast<long long>(m) - static_cast<long long>(m_hi << 29);  // |rem| <= 2^28
+  float hi = __fmul_rn(static_cast<float>(m_hi), pow2f(e - 1046));  // exact: m_hi <= 2^24
+  float lo = __fmul_rn(static_cast<float>(rem), pow2f(e - 1075));
+  if (bits >> 63) {
+    hi = -hi;
+    lo = -lo;
+  }
+  const float p = __fmul_rn(hi, rcp.hi);
+  float err = __fmaf_rn(hi, rcp.hi, -p);
+  err = __fmaf_rn(hi, rcp.lo, err);
+  err = __fmaf_rn(lo, rcp.hi, err);
+  return __fadd_rn(p, err);
+}
+
 // Exact assignment of one query (warp-wide; x holds this lane's elements lane + 32 j):
 // the valid beacon maximising (q . c_b) * (1 / |c_b|) in double-float arithmetic (exact
 // products, TwoSum accumulation, then a butterfly over the lanes), ties to the lower

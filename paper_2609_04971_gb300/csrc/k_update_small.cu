@@ -16,8 +16,8 @@
 //     batched kernel, so both kernels take the same decisions;
 //   sums: per beacon, the rows assigned to it are added as the same three
 //     exact fp32 parts, turned into round(sum * 2^40), added once to the fp64
-//     running sum, and c = fp32(sum * (1 / count)) in fp64, as in the batched
-//     kernel's fold.
+//     running sum, and c = fp32(sum / count) to within one ulp from double-float
+//     arithmetic, as in the batched kernel's fold.
 // All queries of the call see the centroids as they were at call start.
 #include "bkv_device.cuh"
 #include "bkv_internal.h"
@@ -54,6 +54,8 @@ __global__ void __launch_bounds__(32 * kSmallWarps) update_small_kernel(SmallArg
   const int nb = a.nb, nq = a.nq;
   float* cs = small_cent + static_cast<size_t>(w) * nb * D;
   const size_t cbase = static_cast<size_t>(e) * nb * D;
+  const __nv_bfloat16* qe = a.q + static_cast<size_t>(e) * nq * D;
+  const long long cnt_lane = lane < nb ? a.counts[static_cast<size_t>(e) * nb + lane] : 0;  // lane b: beacon b's count
   for (int i = lane; i < nb * D / 4; i += 32)
     reinterpret_cast<float4*>(cs)[i] = reinterpret_cast<const float4*>(a.cent + cbase)[i];
   __syncwarp();
@@ -80,7 +82,7 @@ __global__ void __launch_bounds__(32 * kSmallWarps) update_small_kernel(SmallArg
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1)
       n2d = df_add(n2d, DF{__shfl_xor_sync(0xffffffffu, n2d.hi, o), __shfl_xor_sync(0xffffffffu, n2d.lo, o)});
-    const bool ok = a.counts[static_cast<size_t>(e) * nb + b] > 0 && nz;
+    const bool ok = __shfl_sync(0xffffffffu, cnt_lane, b) > 0 && nz;
     bool plain = true;
     DF inv_df{0.f, 0.f};
     if (ok) inv_df = centroid_inv_norm(n2d, n2, plain);
@@ -94,7 +96,6 @@ __global__ void __launch_bounds__(32 * kSmallWarps) update_small_kernel(SmallArg
   __syncwarp();
 
   // ---- decisions, against the centroids at call start; lane r keeps query r's beacon
-  const __nv_bfloat16* qe = a.q + static_cast<size_t>(e) * nq * D;
   int my_b = -1;
   for (int r = 0; r < nq; ++r) {
     float x[D / 32];
@@ -143,16 +144,15 @@ __global__ void __launch_bounds__(32 * kSmallWarps) update_small_kernel(SmallArg
       for (int j = 0; j < D / 32; ++j) parts_add(p[j], __bfloat162float(qe[static_cast<size_t>(r) * D + lane + 32 * j]));
     }
     const size_t ci = static_cast<size_t>(e) * nb + b;
-    const long long cnt = a.counts[ci] + __popc(rows);
-    const double rcp = __drcp_rn(static_cast<double>(cnt));
+    const long long cnt = __shfl_sync(0xffffffffu, cnt_lane, b) + __popc(rows);
+    const DF rcp = count_reciprocal(cnt);
 #pragma unroll
     for (int j = 0; j < D / 32; ++j) {
       const size_t gi = cbase + static_cast<size_t>(b) * D + lane + 32 * j;
-      const double s_new = __dadd_rn(a.sums[gi], static_cast<double>(fixed40(p[j])) * 0x1p-40);
+      const double s_new = __dadd_rn(a.sums[gi], fixed40_to_double(fixed40(p[j])));
       a.sums[gi] = s_new;
-      a.cent[gi] = __double2float_rn(__dmul_rn(s_new, rcp));
+      a.cent[gi] = centroid_value(s_new, rcp);
     }
-    __syncwarp();  // every lane has read the old count
     if (lane == 0) a.counts[ci] = cnt;
   }
 }
