@@ -125,6 +125,13 @@ def test_continual_fps_with_causal_window():
     _run_cfps(wl, 28, 8, causal=True)
 
 
+def test_continual_fps_all_options_at_128_queries():
+    """16 beacons + 16 window queries per head (the paper's buffer sizes): 128 scoring queries per group, so
+    two score launches folded into one score, with the mean form and the causal mask."""
+    wl = QWEN3_4B.scaled(name="cfps_nb16_w16_mean_causal", n_layers=1, batch=1, window=16, L=1200, budget=700)
+    _run_cfps(wl, 29, 16, mean_agg=True, causal=True)
+
+
 def test_continual_fps_state_round_trip():
     """bkv_set_cfps_state restores buffers that bkv_get_cfps_state saved: an update from the restored
     state gives the same buffers as from the original."""

@@ -18,11 +18,11 @@ from paper_2609_04971_gb300.workloads import QWEN3_4B, TINY
 pytestmark = pytest.mark.gpu
 
 
-def _compare_once(wl, seed, causal=False):
+def _compare_once(wl, seed, causal=False, mean=False):
     from paper_2609_04971_gb300 import bkv, synth
     dev = torch.device("cuda")
     inp = synth.step_inputs(wl, seed, dev)
-    bk = bkv.BeaconKV.for_workload(wl, causal_window=causal)
+    bk = bkv.BeaconKV.for_workload(wl, causal_window=causal, mean_agg=mean)
     try:
         bk.init_beacons(inp["q_init"])
         bk.update(inp["q_new"])
@@ -57,6 +57,12 @@ def test_static_compress_matches_context_compress_on_consecutive_calls():
     _compare_once(ragged, seed=22)        # same shape, new data over the previous scratch contents
     _compare_once(TINY, seed=23)          # another shape (head_dim 64) over the same scratch
     _compare_once(ragged, seed=24, causal=True)   # the causal mask inside the window (cfg.flags)
+    _compare_once(ragged, seed=25, causal=True, mean=True)
+    # 128 scoring queries: two score launches folded into one score
+    m128 = QWEN3_4B.scaled(name="static_m128", n_layers=1, batch=1, n_q_heads=64, n_kv_heads=8, window=12,
+                           n_beacons=32, L=900, budget=600, n_init=64, n_clusters=32)
+    _compare_once(m128, seed=26)
+    _compare_once(m128, seed=27, causal=True, mean=True)
 
 
 def test_static_compress_rejects_requests_beyond_its_scratch():
