@@ -33,8 +33,9 @@ __device__ __forceinline__ __nv_bfloat16 rot_exact(double xa, double xb, double 
   return __float2bfloat16_rn(__double2float_rn(y));
 }
 
-// bf16 of (xa*c +- xb*s) through the fp32 fast path when provably equal to the definition.
-__device__ __forceinline__ __nv_bfloat16 rot_fast(float xa, float xb, float c32, float s32, double c, double s,
+// bf16 of (xa*c +- xb*s) through the fp32 fast path when provably equal to the definition; the
+// fp64 (cos, sin) pair `cs` is read only on the exact path.
+__device__ __forceinline__ __nv_bfloat16 rot_fast(float xa, float xb, float c32, float s32, const double2* cs,
                                                    bool plus) {
   const float p = xb * s32;
   const float v = fmaf(xa, c32, plus ? p : -p);
@@ -46,7 +47,8 @@ __device__ __forceinline__ __nv_bfloat16 rot_fast(float xa, float xb, float c32,
     const int dist = abs(static_cast<int>(t & 0xffffu) - 0x8000);
     if (static_cast<float>(dist - 1) * ulp > delta) return __float2bfloat16_rn(v);
   }
-  return rot_exact(xa, xb, c, s, plus);
+  const double2 c = *cs;
+  return rot_exact(xa, xb, c.x, c.y, plus);
 }
 
 __global__ void __launch_bounds__(kQobsThreads) qobs_kernel(Shape s, const __nv_bfloat16* __restrict__ q_recent,
@@ -87,10 +89,10 @@ __global__ void __launch_bounds__(kQobsThreads) qobs_kernel(Shape s, const __nv_
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       if (row < s.n_obs && rotate) {
-        const double2 cs = rope[slot * h + i + k];
         const float2 cs32 = rope32[slot * h + i + k];
-        y1[k] = rot_fast(xa[k], xb[k], cs32.x, cs32.y, cs.x, cs.y, false);
-        y2[k] = rot_fast(xb[k], xa[k], cs32.x, cs32.y, cs.x, cs.y, true);
+        const double2* cs64 = rope + slot * h + i + k;
+        y1[k] = rot_fast(xa[k], xb[k], cs32.x, cs32.y, cs64, false);
+        y2[k] = rot_fast(xb[k], xa[k], cs32.x, cs32.y, cs64, true);
       } else {
         y1[k] = __float2bfloat16_rn(xa[k]);
         y2[k] = __float2bfloat16_rn(xb[k]);
