@@ -161,7 +161,7 @@ int bkv_init_beacons(bkv_ctx* ctx, const void* q_init, int32_t n_init);
  * non-zero centroid, using the centroids as they were when the call started
  * (ties go to the lowest b; a zero query is skipped).  Then for each beacon
  * sums_b += sum of its assigned queries, counts_b += their number and
- * c_b = fp32(sums_b / counts_b).  Query elements must be finite with
+ * c_b = fp32(sums_b / counts_b) to within one fp32 ulp.  Query elements must be finite with
  * |x| < 2^14, and one call's sum for a beacon must stay below 2^23 in every
  * element (int64 fixed point with 40 fractional bits); that sum is then
  * exact, except that elements below 2^-31 in magnitude are rounded to
@@ -183,7 +183,8 @@ int bkv_update_beacons(bkv_ctx* ctx, const void* q_new, int32_t n_new, int32_t* 
  * beacons with count > 0 rotated to t_pos; each is rounded to bf16 after the
  * rotation.  Score[j] = max over those queries of the softmax weight of key
  * j over all L cached keys (Eq. 4, Eq. 6 max form; logits q.k / sqrt(d)), or
- * their mean under BKV_F_MEAN_AGG.
+ * their mean under BKV_F_MEAN_AGG; under BKV_F_CAUSAL_WINDOW a recent query
+ * leaves out the window rows after its own position.
  * Kept rows = [0, n_prefix) U [L - window, L) U the (budget - n_prefix -
  * window) other rows with the largest Score (ties to the lower index), in
  * ascending order (Eq. 7, Algorithm 2).  Row i of K and V then holds what row
