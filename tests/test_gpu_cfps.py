@@ -30,7 +30,9 @@ def _heads(t: torch.Tensor, d: int) -> np.ndarray:
     return _bits(t).reshape(-1, t.shape[-2], d)
 
 
-def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False, causal=False):
+def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False, causal=False, sample=None):
+    """One init + update + compress; every instance is checked, or only the instances in `sample` (the
+    others still on their sizes and kept sets)."""
     dev = torch.device("cuda")
     inp = synth.step_inputs(wl, seed, dev)
     L = wl.L if L is None else L
@@ -49,15 +51,19 @@ def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False, 
         buf1, size1 = [x.cpu() for x in bk.cfps_state()]
         K, V = inp["K"], inp["V"]
         n_inst = wl.n_inst
-        Kb = _bits(K).reshape(n_inst, wl.capacity, d)
-        Vb = _bits(V).reshape(n_inst, wl.capacity, d)
+        insts = np.arange(n_inst) if sample is None else np.asarray(sample)
+        sel = torch.as_tensor(insts, device=dev)
+
+        def rows(t):  # the checked instances' cache rows, [len(insts), capacity, d] uint16
+            return _bits(t.view(n_inst, wl.capacity, d).index_select(0, sel))
+
+        Kb, Vb = rows(K), rows(V)
         scores = torch.full((wl.n_layers, wl.batch, wl.n_kv_heads, wl.capacity), -1.0, device=dev)
         kept = bk.compress(K, V, L=L, budget=budget, t_pos=inp["t_pos"], q_recent=inp["q_recent"],
                            recent_pos=inp["recent_pos"], scores_out=scores)
         buf2, size2 = [x.cpu() for x in bk.cfps_state()]
         bk.sync()
-        K1 = _bits(K).reshape(n_inst, wl.capacity, d)
-        V1 = _bits(V).reshape(n_inst, wl.capacity, d)
+        K1, V1 = rows(K), rows(V)
     finally:
         bk.close()
 
@@ -68,9 +74,9 @@ def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False, 
     buf1 = buf1.view(torch.int16).numpy().view(np.uint16).reshape(-1, b_max, d)
     buf2 = buf2.view(torch.int16).numpy().view(np.uint16).reshape(-1, b_max, d)
     size0, size1, size2 = (x.numpy().reshape(-1) for x in (size0, size1, size2))
-    n_heads = q_init.shape[0]
+    heads = (insts[:, None] * G + np.arange(G)[None, :]).reshape(-1)
     fps_ties = 0
-    for h in range(n_heads):
+    for h in heads:
         # ---- seeding: fp64 FPS of the head's prompt queries
         picks, gaps = O.fps(q_init[h], b_min, lib)
         assert size0[h] == b_min
@@ -83,16 +89,24 @@ def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False, 
         assert size1[h] == wsize, f"head {h}: size {size1[h]} vs {wsize}"
         np.testing.assert_array_equal(buf1[h, :wsize], want[:wsize], err_msg=f"head {h}: buffer after update")
 
+    # every head: the sizes of a head depend only on the call's lengths
+    assert np.all(size0 == b_min)
+    assert np.all(size1 == size1[heads[0]]) and np.all(size2 == size2[heads[0]])
+
     rel_max, swaps = 0.0, 0
     kept_h = kept.view(n_inst, budget).cpu().numpy()
     s_h = scores.view(n_inst, wl.capacity).cpu().numpy()
-    for e in range(n_inst):
+    if L > budget:  # every instance: ascending, the recent window kept
+        assert np.all(np.diff(kept_h, axis=1) > 0)
+        assert np.all(kept_h[:, budget - W:] == np.arange(L - W, L))
+    for i, e in enumerate(insts):
         hs = slice(e * G, (e + 1) * G)
         r, sw = P.check_cfps_compress(wl, b_min, buf1[hs], size1[hs], q_rec[hs], inp["recent_pos"], inp["t_pos"],
-                                      Kb[e], Vb[e], K1[e], V1[e], kept_h[e], s_h[e], L, budget, buf2[hs], size2[hs],
+                                      Kb[i], Vb[i], K1[i], V1[i], kept_h[e], s_h[e], L, budget, buf2[hs], size2[hs],
                                       lib, tag=f"instance {e}", mean=mean_agg, causal=causal)
         rel_max, swaps = max(rel_max, r), swaps + sw
-    print(f"{wl.name}: {n_heads} heads, seed ties {fps_ties}, max score rel err {rel_max:.2e}, swaps {swaps}")
+    print(f"{wl.name}: {len(heads)} heads checked, seed ties {fps_ties}, max score rel err {rel_max:.2e}, "
+          f"swaps {swaps}")
 
 
 @pytest.mark.parametrize("wl,b_min,seed", [
@@ -102,6 +116,15 @@ def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False, 
 ], ids=lambda x: getattr(x, "name", str(x)))
 def test_continual_fps_step(wl, b_min, seed):
     _run_cfps(wl, seed, b_min)
+
+
+def test_continual_fps_full_size_sampled():
+    """The Qwen3-4B step that the benchmark times in this mode (36 layers, batch 16, 8 beacons + 8 window
+    queries per query head, 128 new queries per head): eight sampled instances checked in full."""
+    wl = QWEN3_4B.scaled(n_beacons=8, name="qwen3_4b_cfps8")
+    rng = np.random.default_rng(1)
+    sample = np.unique(np.concatenate([[0, wl.n_inst - 1], rng.choice(wl.n_inst, 6, replace=False)]))
+    _run_cfps(wl, 30, 8, sample=sample)
 
 
 def test_continual_fps_short_call_and_no_eviction():
