@@ -375,7 +375,10 @@ def main():
             bl = b * args.steps / n  # more than 64 scoring queries: two score launches per step read K twice
             kernels[name] = {"ms_per_launch": per, "launches": n, "alg_bytes_per_launch": bl,
                              "achieved_gbs": bl / (per * 1e-3) / 1e9, "frac_of_hbm": bl / (per * 1e-3) / 1e9 / hbm_gbs}
-    dom = max((k for k in kernels if "ms_per_launch" in kernels[k]),
+    ms, n = prof.get("rope_stage", (0.0, 0))
+    if n:  # the rotary table of a compress, 24 (W + 1) d / 2 bytes copied from pinned host memory
+        kernels["rope_stage"] = {"ms_per_launch": ms / n, "launches": n}
+    dom = max((k for k in kernels if "alg_bytes_per_launch" in kernels[k]),
               key=lambda k: kernels[k]["ms_per_launch"] * kernels[k]["launches"])
     kd = kernels[dom]
     traffic = traffic_from_profiles(dom, wl.n_inst)

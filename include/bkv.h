@@ -36,7 +36,9 @@
  * bkv_set_stream); calls return before it completes.  Outputs are valid once
  * that stream has been synchronised (bkv_sync does so and reports device-side
  * errors).  bkv_compress stages its rotary table in one of four pinned host
- * buffers and waits only when the stream is more than four compress calls
+ * buffers, which a kernel on the stream copies to the device (no copy-engine
+ * transfer, so the stream does not queue behind other streams' bulk host
+ * copies), and waits only when the stream is more than four compress calls
  * behind.  One context must not be used from two host threads at once.
  *
  * Errors.  Every call returns BKV_OK (0) or a negative code; nothing throws.
@@ -264,7 +266,8 @@ int bkv_selftest_wait_timeout(bkv_ctx* ctx, int64_t limit_ns);
 #define BKV_K_SELECT_GATHER 4
 #define BKV_K_KEEP_ALL 5
 #define BKV_K_CFPS 6 /* Continual FPS buffer update, beacon selection and merge */
-#define BKV_NUM_KERNELS 7
+#define BKV_K_ROPE 7 /* rotary table of a compress, copied from pinned host memory */
+#define BKV_NUM_KERNELS 8
 int bkv_profile_enable(bkv_ctx* ctx, int on);
 int bkv_profile_read(bkv_ctx* ctx, double* ms, int64_t* launches, int32_t n_kernels);
 

@@ -23,7 +23,7 @@ BKV_ECUDA = -3
 BKV_ETIMEOUT = -4
 BKV_ESTATE = -5
 
-KERNEL_NAMES = ("fps_init", "update", "qobs", "score", "select_gather", "keep_all", "cfps")
+KERNEL_NAMES = ("fps_init", "update", "qobs", "score", "select_gather", "keep_all", "cfps", "rope_stage")
 
 
 # bkv_config.flags options (include/bkv.h)

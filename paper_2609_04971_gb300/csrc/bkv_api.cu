@@ -38,10 +38,12 @@ struct bkv_ctx {
   float* rscore = nullptr;        // [n_inst][cap]
   double2* rope = nullptr;        // [W + 1][d / 2] fp64 (cos, sin), then the same table in fp32
   int* err = nullptr;             // device error word
-  // pinned host staging of the rotary table, a ring of kRopeSlots: a compress fills the next slot
-  // and uploads it asynchronously; the slot is refilled only after its upload's event completed
+  // pinned host staging of the rotary table, a ring of kRopeSlots: a compress fills the next slot,
+  // a kernel on the stream copies it to `rope` through the slot's device mapping, and the slot is
+  // refilled only after that copy's event completed
   static constexpr int kRopeSlots = 4;
   double2* rope_pinned[kRopeSlots] = {};
+  void* rope_mapped[kRopeSlots] = {};  // device address of rope_pinned[i]
   cudaEvent_t rope_ev[kRopeSlots] = {};
   bool rope_used[kRopeSlots] = {};
   int rope_next = 0;
@@ -266,6 +268,7 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
   const size_t rope_bytes = sizeof(double2) * (static_cast<size_t>(s.W + 1) * (s.d / 2) * 3 / 2 + 1);
   for (int i = 0; i < bkv_ctx::kRopeSlots; ++i) {
     if ((e = cudaMallocHost(reinterpret_cast<void**>(&c->rope_pinned[i]), rope_bytes)) != cudaSuccess ||
+        (e = cudaHostGetDevicePointer(&c->rope_mapped[i], c->rope_pinned[i], 0)) != cudaSuccess ||
         (e = cudaEventCreateWithFlags(&c->rope_ev[i], cudaEventDisableTiming)) != cudaSuccess) {
       const int code = (e == cudaErrorMemoryAllocation) ? BKV_ENOMEM : BKV_ECUDA;
       cudaGetLastError();
@@ -434,9 +437,11 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
         tab32[static_cast<size_t>(slot) * h + i] = make_float2(static_cast<float>(c), static_cast<float>(sn));
       }
     }
-    // pinned source: the copy is asynchronous, and the slot is not refilled before its event
-    e = cudaMemcpyAsync(ctx->rope, tab, sizeof(double2) * n + sizeof(float2) * n, cudaMemcpyHostToDevice,
-                        ctx->stream);
+    {  // the slot is not refilled before this copy's event
+      ProfScope ps(ctx, BKV_K_ROPE);
+      e = bkv::launch_rope_stage(ctx->rope_mapped[rs], ctx->rope, sizeof(double2) * n + sizeof(float2) * n,
+                                 ctx->stream);
+    }
     if (e == cudaSuccess) e = cudaEventRecord(ctx->rope_ev[rs], ctx->stream);
     ctx->rope_used[rs] = true;
     if (e != cudaSuccess) return cuda_fail(ctx, e, "rope table upload");

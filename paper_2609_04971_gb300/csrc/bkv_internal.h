@@ -66,6 +66,9 @@ cudaError_t launch_update_small(const Shape& s, const __nv_bfloat16* q_new, int 
 // rope: [W + 1][d / 2] fp64 (cos, sin) pairs, immediately followed by the same
 // [W + 1][d / 2] table as fp32 pairs; entry w < W is recent slot w, entry W
 // is the beacon position.  rotate == 0 leaves vectors unrotated.
+// Device copy of `bytes` (a multiple of 16, both ends 16-byte aligned) from a
+// device-mapped pinned host buffer, by a kernel on `st`.
+cudaError_t launch_rope_stage(const void* src, void* dst, size_t bytes, cudaStream_t st);
 cudaError_t launch_qobs(const Shape& s, const __nv_bfloat16* q_recent, const float* cent, const long long* counts,
                         const double2* rope, int rotate, __nv_bfloat16* qobs, uint32_t* valid, cudaStream_t st);
 

@@ -110,7 +110,26 @@ __global__ void __launch_bounds__(kQobsThreads) qobs_kernel(Shape s, const __nv_
   }
 }
 
+// Copies one compress's rotary table from pinned host memory, read through its
+// device mapping, into device memory.  The copy is made by the SMs rather than
+// a copy engine, so the stream's kernels never wait in a copy-engine queue
+// behind bulk host transfers that other streams have issued.
+__global__ void __launch_bounds__(256) rope_stage_kernel(const uint4* __restrict__ src, uint4* __restrict__ dst,
+                                                         int n16) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n16) dst[i] = src[i];
+}
+
 }  // namespace
+
+cudaError_t launch_rope_stage(const void* src, void* dst, size_t bytes, cudaStream_t st) {
+  if (bytes == 0) return cudaSuccess;
+  if (bytes % 16 != 0 || (reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) % 16 != 0)
+    return cudaErrorInvalidValue;
+  const int n16 = static_cast<int>(bytes / 16);
+  rope_stage_kernel<<<(n16 + 255) / 256, 256, 0, st>>>(static_cast<const uint4*>(src), static_cast<uint4*>(dst), n16);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_qobs(const Shape& s, const __nv_bfloat16* q_recent, const float* cent, const long long* counts,
                         const double2* rope, int rotate, __nv_bfloat16* qobs, uint32_t* valid, cudaStream_t st) {
