@@ -26,3 +26,57 @@ def test_expired_wait_reports_timeout_then_context_recovers():
     # the device and the library still compute correct results afterwards
     run = P.run_gpu(TINY)
     P.check_run(run)
+
+
+def test_rejected_arguments_leave_everything_untouched():
+    """Argument errors of bkv_update_beacons and bkv_compress are caught on the host before any work is
+    enqueued: each call raises with its documented code, and K, V, the kept-index output and the beacon
+    state are unchanged afterwards; an update of zero queries is a no-op."""
+    from paper_2609_04971_gb300 import synth
+    wl = TINY
+    dev = torch.device("cuda")
+    inp = synth.step_inputs(wl, 3, dev)
+    K, V = inp["K"], inp["V"]
+    kept = torch.full((wl.n_layers, wl.batch, wl.n_kv_heads, wl.budget), -7, dtype=torch.int32, device=dev)
+    pos = dict(t_pos=inp["t_pos"], recent_pos=inp["recent_pos"])
+
+    def code_of(fn):
+        with pytest.raises(bkv.BkvError) as ei:
+            fn()
+        return ei.value.code
+
+    bk = bkv.BeaconKV.for_workload(wl)
+    try:
+        # before bkv_init_beacons: no beacon state yet
+        assert code_of(lambda: bkv.bkv_update_beacons(bk.ctx, inp["q_new"], wl.n_new)) == bkv.BKV_ESTATE
+        assert code_of(lambda: bkv.bkv_compress(bk.ctx, K, V, wl.L, wl.budget, q_recent=inp["q_recent"],
+                                                kept_idx_out=kept, **pos)) == bkv.BKV_ESTATE
+        bk.init_beacons(inp["q_init"])
+        state0 = [t.clone() for t in bk.state()]
+        K0, V0 = K.clone(), V.clone()
+        q_odd = inp["q_new"].view(-1)[1:]  # 2 bytes past a 16-byte boundary
+        K_odd = K.view(-1)[1:]
+        assert code_of(lambda: bkv.bkv_update_beacons(bk.ctx, inp["q_new"], -1)) == bkv.BKV_EINVAL
+        assert code_of(lambda: bkv.bkv_update_beacons(bk.ctx, q_odd, wl.n_new)) == bkv.BKV_EINVAL
+        bkv.bkv_update_beacons(bk.ctx, inp["q_new"], 0)  # no queries: nothing to do
+        for L, budget, k, q in [(0, wl.budget, K, inp["q_recent"]),                 # empty cache
+                                (wl.capacity + 1, wl.budget, K, inp["q_recent"]),   # past the capacity
+                                (wl.L, wl.window - 1, K, inp["q_recent"]),          # budget below the window
+                                (wl.L, wl.budget, K_odd, inp["q_recent"]),          # misaligned K
+                                (wl.L, wl.budget, K, None)]:                        # window queries missing
+            assert code_of(lambda: bkv.bkv_compress(bk.ctx, k, V, L, budget, q_recent=q, kept_idx_out=kept,
+                                                    **pos)) == bkv.BKV_EINVAL, (L, budget)
+        bk.sync()
+        assert torch.equal(K, K0) and torch.equal(V, V0)
+        assert bool((kept == -7).all())
+        for a, b in zip(bk.state(), state0):
+            assert torch.equal(a, b)
+        # the context still works: a valid step keeps the budget with the window
+        bk.update(inp["q_new"])
+        bk.compress(K, V, L=wl.L, budget=wl.budget, q_recent=inp["q_recent"], kept_out=kept, **pos)
+        bk.sync()
+        k_h = kept.view(-1, wl.budget).cpu()
+        assert bool((k_h[:, 1:] > k_h[:, :-1]).all())
+        assert bool((k_h[:, -wl.window:] == torch.arange(wl.L - wl.window, wl.L, dtype=torch.int32)).all())
+    finally:
+        bk.close()
