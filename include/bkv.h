@@ -143,7 +143,11 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out);
 /* Frees everything the context owns (after synchronising its stream). NULL is ignored. */
 void bkv_destroy(bkv_ctx* ctx);
 
-/* Changes the stream used by later calls. */
+/* Changes the stream used by later calls.  The new stream is made to wait
+ * (cudaStreamWaitEvent) for the work already enqueued on the old one, so a
+ * switch never lets two calls of one context run concurrently.  Returns
+ * BKV_ECUDA if the event record or the wait fails (the stream is then
+ * unchanged). */
 int bkv_set_stream(bkv_ctx* ctx, void* stream);
 
 /*

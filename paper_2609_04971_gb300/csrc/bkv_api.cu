@@ -47,6 +47,7 @@ struct bkv_ctx {
   cudaEvent_t rope_ev[kRopeSlots] = {};
   bool rope_used[kRopeSlots] = {};
   int rope_next = 0;
+  cudaEvent_t switch_ev = nullptr;  // orders a new stream after the previous one (bkv_set_stream)
   std::string last_error;
   // per-kernel timing
   struct Rec {
@@ -190,6 +191,7 @@ void free_all(bkv_ctx* c) {
     if (c->rope_pinned[i]) cudaFreeHost(c->rope_pinned[i]);
     if (c->rope_ev[i]) cudaEventDestroy(c->rope_ev[i]);
   }
+  if (c->switch_ev) cudaEventDestroy(c->switch_ev);
 }
 
 }  // namespace
@@ -277,6 +279,12 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
       return code;
     }
   }
+  if ((e = cudaEventCreateWithFlags(&c->switch_ev, cudaEventDisableTiming)) != cudaSuccess) {
+    cudaGetLastError();
+    free_all(c);
+    delete c;
+    return BKV_ECUDA;
+  }
   *out = c;
   return BKV_OK;
 }
@@ -290,7 +298,15 @@ void bkv_destroy(bkv_ctx* ctx) {
 
 int bkv_set_stream(bkv_ctx* ctx, void* stream) {
   if (!ctx) return BKV_EINVAL;
-  ctx->stream = static_cast<cudaStream_t>(stream);
+  const cudaStream_t next = static_cast<cudaStream_t>(stream);
+  if (next != ctx->stream) {
+    // the context's scratch and state are reused by the next call: its work on the new stream
+    // starts after everything already enqueued on the old one
+    cudaError_t e = cudaEventRecord(ctx->switch_ev, ctx->stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(next, ctx->switch_ev, 0);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "stream switch");
+  }
+  ctx->stream = next;
   return BKV_OK;
 }
 

@@ -161,6 +161,38 @@ def test_deterministic_across_runs():
     np.testing.assert_array_equal(a.K_after, b.K_after)
 
 
+def test_stream_switch_matches_one_stream():
+    """Calls split across two streams by bkv_set_stream give the results of one stream: the switch orders
+    the new stream after the work already enqueued on the old one."""
+    from paper_2609_04971_gb300 import bkv
+    wl = QWEN3_4B.scaled(name="switch", n_layers=2, batch=2)
+    dev = torch.device("cuda")
+    inp = synth.step_inputs(wl, 31, dev)
+    outs = []
+    for switch in (False, True):
+        K, V = inp["K"].clone(), inp["V"].clone()
+        s1, s2 = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        torch.cuda.synchronize()
+        bk = bkv.BeaconKV.for_workload(wl, stream=s1)
+        try:
+            with torch.cuda.stream(s1):
+                bk.init_beacons(inp["q_init"])
+                bk.update(inp["q_new"])
+            if switch:
+                bkv.bkv_set_stream(bk.ctx, s2)
+            with torch.cuda.stream(s2 if switch else s1):
+                kept = bk.compress(K, V, L=wl.L, budget=wl.budget, t_pos=inp["t_pos"], q_recent=inp["q_recent"],
+                                   recent_pos=inp["recent_pos"])
+                state = bk.state()
+            bk.sync()
+            torch.cuda.synchronize()
+            outs.append([kept.cpu(), K.cpu(), V.cpu()] + [t.cpu() for t in state])
+        finally:
+            bk.close()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+
+
 # ---------------------------------------------------------------- causal mask inside the window (BKV_F_CAUSAL_WINDOW)
 def _shift_positions(inp, W, t_pos, recent_pos):
     inp = dict(inp)
