@@ -13,6 +13,11 @@ Every step is bracketed by CUDA events on the stream the library launches on.
 
     python bench.py [--gpus N --steps K --warmup W] [--impl reference]
 
+--config 3 / 4 time the same step on the Llama-8B and Qwen3-14B shapes.
+--config 5 (or --trace-steps N) runs the long decode trace instead: one beacon
+update per decode step and a compress whenever the cache reaches L rows, timed
+as the total device time of the library calls over the trace (trace_main).
+
 Prints one JSON line (rank 0).  --impl reference times the CPU oracle (the
 plain fp64 restatement of the method) on the host cores instead.
 """
@@ -54,6 +59,8 @@ def parse():
                     help="beacon maintenance: running-mean centroids, or the paper's Continual FPS buffers")
     ap.add_argument("--cfps-beacons", type=int, default=8,
                     help="Continual FPS: beacons per query head (the buffer holds this + window queries)")
+    ap.add_argument("--trace-steps", type=int, default=0,
+                    help="decode steps of the long-trace mode (0: the workload's own; config 5 runs a trace)")
     return ap.parse_args()
 
 
@@ -284,6 +291,9 @@ def main():
     if args.impl == "reference":
         reference_arm(args, wl, rank)
         return
+    if args.trace_steps or wl.trace_steps:
+        trace_main(args, wl, rank, world, local_rank, cfps)
+        return
 
     import torch
     import torch.distributed as dist
@@ -415,6 +425,196 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds, args.seed)
     bk.close()
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+# ------------------------------------------------------------------ long decode trace
+TRACE_POOL = 256  # decode steps of pre-generated queries and K / V rows that the trace cycles through
+
+
+def trace_schedule(prefill: int, budget: int, grow: int, steps: int) -> list[int]:
+    """0-based decode steps after whose token the cache holds budget + grow rows and is compressed
+    back to budget (one token is appended per step, starting from a prompt of `prefill` rows)."""
+    sched, L = [], prefill
+    for s in range(steps):
+        L += 1
+        if L >= budget + grow:
+            sched.append(s)
+            L = budget
+    return sched
+
+
+def trace_main(args, wl, rank: int, world: int, local_rank: int, cfps: bool) -> None:
+    """Long decode trace.  After a prompt of wl.prefill tokens (FPS-seeded beacons), every decode step
+    adds one pre-RoPE query per query head (one beacon update with n_new = 1) and one K / V row; when
+    the cache reaches wl.L rows it is compressed to wl.budget.  The timed quantity is the compression
+    overhead of the whole trace: the device time of every bkv_update_beacons and bkv_compress call, each
+    bracketed by CUDA events on the library's stream.  The model's own work between them (appending the
+    K / V row, building the recent-query block) runs outside the events.  Queries and K / V rows cycle
+    through TRACE_POOL pre-generated decode steps (drifting clusters within the pool), so that host-side
+    input generation does not pace the trace."""
+    import collections
+
+    import torch
+    import torch.distributed as dist
+    from paper_2609_04971_gb300 import bkv, synth
+
+    steps = args.trace_steps or wl.trace_steps
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    hbm_gbs, bf16_tflops, peak_src = peaks()
+    nl, B, Hkv, d, W = wl.n_layers, wl.batch, wl.n_kv_heads, wl.head_dim, wl.window
+    cap, budget = wl.L, wl.budget
+    sched = trace_schedule(wl.prefill, budget, cap - budget, steps)
+    if sched and sched[0] + 1 < W:
+        raise SystemExit("trace: the first compress comes before the recent window has filled")
+    seed = rank_seed(args.seed, rank)
+    gen = synth.TraceGen(wl, seed, dev)
+    q_init, k0, v0 = gen.prefill()
+    pool = max(W, 1, min(TRACE_POOL, steps))   # the warm-up compress takes its W recent queries from the pool
+    # step-major pools: q_pool[j] is one decode step's contiguous [nl, B, Hq, 1, d] query block
+    q_pool = torch.stack([gen.step_queries() for _ in range(pool)])
+    k_pool, v_pool = (x.permute(3, 0, 1, 2, 4).contiguous() for x in gen.kv_rows(pool))  # [P, nl, B, Hkv, d]
+    K = torch.empty(nl, B, Hkv, cap, d, dtype=torch.bfloat16, device=dev)
+    V = torch.empty_like(K)
+    kept = torch.empty(nl, B, Hkv, budget, dtype=torch.int32, device=dev)
+
+    # warm-up on a throw-away context: updates and one compress of a full cache of random rows
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed + 1)
+    K.normal_(generator=g)
+    V.normal_(generator=g)
+    wb = bkv.BeaconKV.for_workload(wl, continual_fps=cfps)
+    wb.init_beacons(q_init)
+    for i in range(max(args.warmup, W)):
+        wb.update(q_pool[i % pool])
+    t = cap - 1
+    wb.compress(K, V, L=cap, budget=budget, t_pos=t,
+                q_recent=q_pool[:W, :, :, :, 0].permute(1, 2, 3, 0, 4).contiguous(),
+                recent_pos=list(range(t - W + 1, t + 1)), kept_out=kept)
+    wb.sync()
+    wb.close()
+
+    K[:, :, :, :wl.prefill].copy_(k0)
+    V[:, :, :, :wl.prefill].copy_(v0)
+    del k0, v0
+    bk = bkv.BeaconKV.for_workload(wl, continual_fps=cfps)
+    bk.init_beacons(q_init)
+    bk.sync()
+    bkv.bkv_profile_read(bk.ctx)
+    bkv.bkv_profile_enable(bk.ctx, True)
+
+    drain = 256  # events are read back (host-side, outside the timed brackets) every `drain` steps
+    ev_u = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(drain)]
+    ev_c = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in range(len(sched))]
+    upd_ms = 0.0
+    hist = collections.deque(maxlen=W)   # (query [nl, B, Hq, d], absolute position) of the latest steps
+    L, pos, c = wl.prefill, wl.prefill, 0
+    compress_at = set(sched)
+
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    gpu_index = int(vis.split(",")[local_rank]) if vis and vis.split(",")[0].isdigit() else local_rank
+    sampler = ClockSampler(gpu_index)
+    sampler.start()
+    barrier()
+    torch.cuda.synchronize()
+    wall0 = time.perf_counter()
+    for s in range(steps):
+        j = s % pool
+        e0, e1 = ev_u[s % drain]
+        e0.record()
+        bk.update(q_pool[j])
+        e1.record()
+        K[:, :, :, L].copy_(k_pool[j])
+        V[:, :, :, L].copy_(v_pool[j])
+        hist.append((q_pool[j, :, :, :, 0], pos))
+        L += 1
+        pos += 1
+        if s in compress_at:
+            q_recent = torch.stack([h[0] for h in hist], dim=3)
+            a, b = ev_c[c]
+            a.record()
+            bk.compress(K, V, L=L, budget=budget, t_pos=pos - 1, q_recent=q_recent,
+                        recent_pos=[h[1] for h in hist], kept_out=kept)
+            b.record()
+            c += 1
+            L = budget
+        if s % drain == drain - 1 or s == steps - 1:
+            ev_u[s % drain][1].synchronize()
+            upd_ms += sum(x.elapsed_time(y) for x, y in ev_u[:s % drain + 1])
+    torch.cuda.synchronize()
+    wall_s = time.perf_counter() - wall0
+    barrier()
+    clocks = sampler.stop()
+    bk.sync()
+    prof = bkv.bkv_profile_read(bk.ctx)
+    bkv.bkv_profile_enable(bk.ctx, False)
+    bk.close()
+    cmp_ms = [x.elapsed_time(y) for x, y in ev_c]
+    total_ms = max_over_ranks(upd_ms + sum(cmp_ms), world, dev)
+
+    tokens = len(sched) * wl.n_inst * cap * world
+    if cfps:  # lower bound: read each new query and write it into its head's buffer
+        upd_bytes = 2 * wl.n_layers * wl.batch * wl.n_q_heads * d * 2
+    else:
+        upd_bytes = wl.update_bytes(1)
+    trace_bytes = len(sched) * wl.compress_bytes() + steps * upd_bytes
+    trace_flops = len(sched) * wl.compress_flops() + (0 if cfps else steps * wl.update_flops(1))
+    roof_ms = 1e3 * max(trace_bytes / (hbm_gbs * 1e9), trace_flops / (bf16_tflops * 1e12))
+    per_launch_bytes = {"qobs": wl.n_inst * wl.group * W * d * 2, "score": wl.n_inst * cap * d * 2,
+                        "select_gather": wl.n_inst * (budget * d * 2 * 4 + budget * 4)}
+    if not cfps:
+        per_launch_bytes["update"] = upd_bytes
+    kernels = {}
+    for name, (ms, n) in prof.items():
+        if not n:
+            continue
+        k = {"ms_per_launch": ms / n, "launches": n, "ms_total": ms}
+        if name in per_launch_bytes:
+            bl = per_launch_bytes[name] * (len(sched) if name != "update" else steps) / n
+            k.update(alg_bytes_per_launch=bl, achieved_gbs=bl / (ms / n * 1e-3) / 1e9,
+                     frac_of_hbm=bl / (ms / n * 1e-3) / 1e9 / hbm_gbs)
+        kernels[name] = k
+    cands = [k for k in kernels if "achieved_gbs" in kernels[k]]
+    dom = max(cands, key=lambda k: kernels[k]["ms_total"]) if cands else None
+    roofline = None
+    if dom is not None:
+        kd = kernels[dom]
+        # the recorded ncu traffic of the update kernel is the batched form's; decode steps run the few-query form
+        traffic = None if dom == "update" else traffic_from_profiles(dom, wl.n_inst)
+        roofline = {"bound": "hbm", "kernel": dom, "achieved": kd["achieved_gbs"], "peak": hbm_gbs, "unit": "GB/s",
+                    "frac": kd["achieved_gbs"] / hbm_gbs, "traffic": traffic, "peak_source": f"{peak_src} hbm_gbs"}
+    out = {
+        "metric": METRIC, "value": tokens / (total_ms / 1e3), "unit": UNIT, "n_gpus": world, "steps": steps,
+        "warmup": args.warmup, "ms_per_step": total_ms / steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": dict(config_block(wl, world), beacon_mode=args.beacons, decode_steps=steps,
+                       compresses=len(sched), query_pool_steps=pool,
+                       l2="K/V working set 10 GB > L2; no flush between decode steps"),
+        "roofline": roofline,
+        "step_roofline": {"alg_bytes": trace_bytes, "alg_flops": trace_flops, "roofline_ms": roof_ms,
+                          "frac": roof_ms / total_ms,
+                          "note": "whole trace: every compress plus one update per decode step"
+                                  + ("; Continual FPS updates counted as query read + buffer append only"
+                                     if cfps else "")},
+        "trace": {"overhead_s": total_ms / 1e3, "overhead_us_per_decode_step": 1e3 * total_ms / steps,
+                  "update_us_per_step": 1e3 * upd_ms / steps,
+                  "compress_ms_mean": statistics.mean(cmp_ms) if cmp_ms else 0.0,
+                  "wall_s": wall_s},
+        "kernels": kernels, "gpu_launches": sum(n for _, n in prof.values()), "clocks": clocks,
+        "e2e": None, "e2e_note": "trace mode: device-resident inputs only",
+    }
     if rank == 0:
         print(json.dumps(out), flush=True)
     if world > 1:

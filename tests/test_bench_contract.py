@@ -6,6 +6,8 @@ import subprocess
 import sys
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
 
 
 def test_reference_arm_json_line():
@@ -23,3 +25,15 @@ def test_reference_arm_json_line():
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1 and cb["sample"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
+def test_trace_schedule_of_the_long_trace():
+    """The long-trace mode compresses whenever the cache reaches L rows: after a 128-token prompt and
+    32768 decode steps that is once at step 4095 (128 + 4096 = 4224 rows) and then every 128 steps,
+    225 compresses in all."""
+    import bench
+    from paper_2609_04971_gb300.workloads import QWEN3_8B_TRACE as T
+    sched = bench.trace_schedule(T.prefill, T.budget, T.L - T.budget, T.trace_steps)
+    assert len(sched) == 225 and sched[0] == T.L - T.prefill - 1
+    assert all(b - a == T.L - T.budget for a, b in zip(sched, sched[1:]))
+    assert bench.trace_schedule(10, 8, 4, 1) == [] and bench.trace_schedule(10, 8, 4, 6) == [1, 5]
