@@ -279,14 +279,42 @@ class BeaconKV:
         except Exception:  # noqa: BLE001 - interpreter shutdown
             pass
 
+    # The C ABI receives bare pointers and trusts the sizes that the context's shape implies; these
+    # checks turn a tensor of the wrong size into a ValueError here instead of an out-of-bounds access
+    # on the device.
+    @staticmethod
+    def _expect(t: torch.Tensor | None, n: int, name: str) -> None:
+        if t is not None and t.numel() != n:
+            raise ValueError(f"{name} has {t.numel()} elements; this context's shape needs {n}")
+
+    def _rows(self, q: torch.Tensor, name: str) -> int:
+        """Queries per query head of a [n_layers, batch, n_q_heads, n, head_dim] block."""
+        c = self.cfg
+        if q.dim() < 2 or q.shape[-1] != c.head_dim:
+            raise ValueError(f"{name} must end in [n, head_dim = {c.head_dim}], got {tuple(q.shape)}")
+        n = q.shape[-2]
+        self._expect(q, c.n_layers * c.batch * c.n_q_heads * n * c.head_dim, name)
+        return n
+
     def init_beacons(self, q_init: torch.Tensor):
-        bkv_init_beacons(self.ctx, q_init, q_init.shape[-2])
+        bkv_init_beacons(self.ctx, q_init, self._rows(q_init, "q_init"))
 
     def update(self, q_new: torch.Tensor, assign_out: torch.Tensor | None = None):
-        bkv_update_beacons(self.ctx, q_new, q_new.shape[-2], assign_out)
+        n_new = self._rows(q_new, "q_new")
+        c = self.cfg
+        self._expect(assign_out, c.n_layers * c.batch * c.n_q_heads * n_new, "assign_out")
+        bkv_update_beacons(self.ctx, q_new, n_new, assign_out)
 
     def compress(self, K, V, *, L, budget, t_pos, q_recent, recent_pos, kept_out=None, scores_out=None):
         c = self.cfg
+        per_head = c.n_layers * c.batch * c.n_kv_heads
+        self._expect(K, per_head * c.capacity * c.head_dim, "K")
+        self._expect(V, per_head * c.capacity * c.head_dim, "V")
+        self._expect(q_recent, c.n_layers * c.batch * c.n_q_heads * c.window * c.head_dim, "q_recent")
+        if len(recent_pos) != c.window:
+            raise ValueError(f"recent_pos has {len(recent_pos)} positions; the window is {c.window}")
+        self._expect(kept_out, per_head * budget, "kept_out")
+        self._expect(scores_out, per_head * c.capacity, "scores_out")
         if kept_out is None:
             kept_out = torch.empty(c.n_layers, c.batch, c.n_kv_heads, budget, dtype=torch.int32, device=K.device)
         bkv_compress(self.ctx, K, V, L, budget, t_pos, q_recent, recent_pos, kept_out, scores_out)
@@ -302,6 +330,10 @@ class BeaconKV:
         return cent, sums, counts
 
     def set_state(self, cent, sums, counts):
+        c = self.cfg
+        self._expect(cent, self.n_inst * c.n_beacons * c.head_dim, "centroids")
+        self._expect(sums, self.n_inst * c.n_beacons * c.head_dim, "sums")
+        self._expect(counts, self.n_inst * c.n_beacons, "counts")
         bkv_set_state(self.ctx, cent, sums, counts)
 
     def cfps_state(self):
@@ -315,6 +347,10 @@ class BeaconKV:
         return buf, sizes
 
     def set_cfps_state(self, buf, sizes):
+        c = self.cfg
+        heads = c.n_layers * c.batch * c.n_q_heads
+        self._expect(buf, heads * (c.n_beacons + c.window) * c.head_dim, "buffers")
+        self._expect(sizes, heads, "sizes")
         bkv_set_cfps_state(self.ctx, buf, sizes)
 
     def sync(self):

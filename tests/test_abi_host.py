@@ -99,3 +99,44 @@ def test_byte_accounting_matches_closed_form():
 
 def test_selftest_rejects_null_context(lib):
     assert lib.bkv_selftest_wait_timeout(None, 1_000_000) == bkv.BKV_EINVAL
+
+
+def test_binding_rejects_tensors_of_the_wrong_size(lib):
+    """The C ABI takes bare pointers and trusts the sizes the context's shape implies, so the Python
+    binding checks every tensor's element count first: a wrong size is a ValueError before any call
+    reaches the library (checked here on a context object with no device context behind it); a right
+    size gets as far as the device-pointer check, which rejects these CPU tensors."""
+    import torch
+    wl = TINY
+    bk = bkv.BeaconKV.__new__(bkv.BeaconKV)
+    bk.cfg = bkv.BkvConfig(wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.n_beacons,
+                           wl.window, 0, wl.capacity, wl.rope_theta, 0)
+    bk.ctx = None
+    bk.n_inst = wl.n_inst
+    nl, B, Hq, Hkv, d, W, cap = wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.window, wl.capacity
+    bf = dict(dtype=torch.bfloat16)
+    q = torch.zeros(nl, B, Hq, 3, d, **bf)
+    K = torch.zeros(nl, B, Hkv, cap, d, **bf)
+    qr = torch.zeros(nl, B, Hq, W, d, **bf)
+    kept = torch.zeros(nl, B, Hkv, wl.budget, dtype=torch.int32)
+    pos = dict(L=wl.L, budget=wl.budget, t_pos=wl.L - 1, recent_pos=list(range(wl.L - W, wl.L)))
+    bad = [
+        lambda: bk.update(torch.zeros(nl, B, Hq - 1, 3, d, **bf)),                       # a head short
+        lambda: bk.update(torch.zeros(nl, B, Hq, 3, d // 2, **bf)),                      # wrong head_dim
+        lambda: bk.update(q, torch.zeros(nl, B, Hq, 2, dtype=torch.int32)),              # assign_out too small
+        lambda: bk.init_beacons(torch.zeros(nl, B, Hq * 3 * d, **bf)),                   # no row axis
+        lambda: bk.compress(K[..., :-1, :], K, q_recent=qr, kept_out=kept, **pos),       # K short of capacity
+        lambda: bk.compress(K, K, q_recent=qr[..., :-1, :], kept_out=kept, **pos),      # window short
+        lambda: bk.compress(K, K, q_recent=qr, kept_out=kept[..., :-1], **pos),          # kept_out too small
+        lambda: bk.compress(K, K, q_recent=qr, kept_out=kept, scores_out=torch.zeros(nl, B, Hkv, cap - 1), **pos),
+        lambda: bk.compress(K, K, q_recent=qr, kept_out=kept, **dict(pos, recent_pos=[0])),
+        lambda: bk.set_state(torch.zeros(wl.n_inst, wl.n_beacons, d), torch.zeros(wl.n_inst, wl.n_beacons, d - 1),
+                             torch.zeros(wl.n_inst, wl.n_beacons, dtype=torch.int64)),
+    ]
+    for i, call in enumerate(bad):
+        with pytest.raises(ValueError):
+            call()
+    for call in (lambda: bk.update(q), lambda: bk.init_beacons(q),
+                 lambda: bk.compress(K, K, q_recent=qr, kept_out=kept, **pos)):
+        with pytest.raises(TypeError, match="CUDA tensor"):
+            call()
