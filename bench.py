@@ -522,6 +522,7 @@ def trace_main(args, wl, rank: int, world: int, local_rank: int, cfps: bool) -> 
     hist = collections.deque(maxlen=W)   # (query [nl, B, Hq, d], absolute position) of the latest steps
     L, pos, c = wl.prefill, wl.prefill, 0
     compress_at = set(sched)
+    prof = {name: (0.0, 0) for name in bkv.KERNEL_NAMES}
 
     vis = os.environ.get("CUDA_VISIBLE_DEVICES")
     gpu_index = int(vis.split(",")[local_rank]) if vis and vis.split(",")[0].isdigit() else local_rank
@@ -553,12 +554,13 @@ def trace_main(args, wl, rank: int, world: int, local_rank: int, cfps: bool) -> 
         if s % drain == drain - 1 or s == steps - 1:
             ev_u[s % drain][1].synchronize()
             upd_ms += sum(x.elapsed_time(y) for x, y in ev_u[:s % drain + 1])
+            for name, (ms, n) in bkv.bkv_profile_read(bk.ctx).items():  # recycles the library's events
+                prof[name] = (prof[name][0] + ms, prof[name][1] + n)
     torch.cuda.synchronize()
     wall_s = time.perf_counter() - wall0
     barrier()
     clocks = sampler.stop()
     bk.sync()
-    prof = bkv.bkv_profile_read(bk.ctx)
     bkv.bkv_profile_enable(bk.ctx, False)
     bk.close()
     cmp_ms = [x.elapsed_time(y) for x, y in ev_c]
