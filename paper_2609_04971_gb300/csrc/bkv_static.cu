@@ -131,6 +131,12 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
     return bad(buf);
   }
 
+  // the scoring inputs matter only when rows are evicted; checked before anything is enqueued
+  if (L > budget && s.W > 0 && (!q_recent || !aligned(q_recent, 16) || !recent_pos))
+    return bad("q_recent (16-byte aligned) and recent_pos are required when window > 0");
+  if (L > budget && s.nb > 0 && (!centroids || !counts || !aligned(centroids, 4) || !aligned(counts, 8)))
+    return bad("centroids and counts are required when n_beacons > 0");
+
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaError_t e;
   if (dev_status && (e = cudaMemsetAsync(dev_status, 0, sizeof(int32_t), st)) != cudaSuccess) {
@@ -142,10 +148,6 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
     if (e != cudaSuccess) message(err_msg, err_len, cudaGetErrorString(e));
     return e == cudaSuccess ? BKV_OK : BKV_ECUDA;
   }
-  if (s.W > 0 && (!q_recent || !aligned(q_recent, 16) || !recent_pos))
-    return bad("q_recent (16-byte aligned) and recent_pos are required when window > 0");
-  if (s.nb > 0 && (!centroids || !counts || !aligned(centroids, 4) || !aligned(counts, 8)))
-    return bad("centroids and counts are required when n_beacons > 0");
 
   void* base = nullptr;
   if ((e = scratch_address(&base)) != cudaSuccess) {

@@ -140,3 +140,50 @@ def test_binding_rejects_tensors_of_the_wrong_size(lib):
                  lambda: bk.compress(K, K, q_recent=qr, kept_out=kept, **pos)):
         with pytest.raises(TypeError, match="CUDA tensor"):
             call()
+
+
+def test_static_compress_rejects_bad_arguments_before_any_cuda_call(lib):
+    """bkv_compress_static validates its configuration, pointers, sizes and scratch budget on the host
+    and returns BKV_EINVAL with a reason before it enqueues anything.  The pointers below are never
+    dereferenced: every case fails validation first."""
+    raw = ctypes.CDLL(_build.LIB_PATH)
+    fn = raw.bkv_compress_static
+    fn.restype = ctypes.c_int
+    wl = TINY
+    P = ctypes.c_void_p
+    dev_a, dev_b, dev_c = P(0x10000), P(0x20000), P(0x30000)   # 16-byte aligned stand-ins, never touched
+
+    def cfg(**kw):
+        base = dict(n_layers=wl.n_layers, batch=wl.batch, n_q_heads=wl.n_q_heads, n_kv_heads=wl.n_kv_heads,
+                    head_dim=wl.head_dim, n_beacons=wl.n_beacons, window=wl.window, n_prefix=0,
+                    capacity=wl.capacity, rope_theta=wl.rope_theta, flags=0)
+        base.update(kw)
+        return bkv.BkvConfig(*base.values())
+
+    pos = (ctypes.c_int64 * wl.window)(*range(wl.L - wl.window, wl.L))
+
+    def call(c, K=dev_a, V=dev_b, kept=dev_c, L=wl.L, budget=wl.budget, q_recent=dev_a, recent=pos,
+             centroids=dev_b, counts=dev_c):
+        msg = ctypes.create_string_buffer(200)
+        rc = fn(None if c is None else ctypes.byref(c), centroids, counts, K, V, ctypes.c_int32(L),
+                ctypes.c_int32(budget), ctypes.c_int64(wl.L - 1), q_recent, recent, kept, None, None, None, msg,
+                ctypes.c_size_t(ctypes.sizeof(msg)))
+        return rc, msg.value.decode()
+
+    cases = [
+        (dict(c=None), "cfg is NULL"),
+        (dict(c=cfg(head_dim=96)), "head_dim"),
+        (dict(c=cfg(flags=bkv.BKV_F_CONTINUAL_FPS)), "flags"),
+        (dict(c=cfg(n_q_heads=3)), "head"),
+        (dict(c=cfg(), K=None), "non-NULL"),
+        (dict(c=cfg(), V=P(0x20008)), "aligned"),
+        (dict(c=cfg(), L=wl.capacity + 1), "L must be"),
+        (dict(c=cfg(), budget=wl.window - 1), "budget"),
+        (dict(c=cfg(n_layers=64, capacity=32768), L=32768), "scratch"),
+        (dict(c=cfg(), q_recent=None), "q_recent"),
+        (dict(c=cfg(), recent=None), "recent_pos"),
+        (dict(c=cfg(), centroids=None), "centroids"),
+    ]
+    for kw, why in cases:
+        rc, msg = call(**kw)
+        assert rc == bkv.BKV_EINVAL and why in msg, (kw, rc, msg)
