@@ -129,6 +129,7 @@ def test_full_size_sampled(wl):
     QWEN3_4B.scaled(name="few_n8", n_layers=1, batch=2, n_new=8),   # 32 rows: the largest few-query call
     QWEN3_4B.scaled(name="few_n9", n_layers=1, batch=2, n_new=9),   # 36 rows: the batched kernel
     TINY.scaled(name="few_d64_n4", n_new=4),                        # head_dim 64, 8 rows
+    QWEN3_14B.scaled(name="few_g5_n1", n_layers=1, batch=2, n_new=1),  # GQA group 5: 5 rows, 16 beacons
     QWEN3_4B.scaled(name="few_g8_nb32_n4", n_layers=1, batch=1, n_q_heads=64, n_kv_heads=8, window=12, n_beacons=32,
                     L=700, budget=500, n_init=64, n_clusters=32, n_new=4),   # 32 rows, 32 beacons
     QWEN3_4B.scaled(name="qwen3_4b_decode_step", n_new=1),          # all 4608 instances, sampled
