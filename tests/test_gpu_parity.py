@@ -9,7 +9,7 @@ import pytest
 import torch
 
 from paper_2609_04971_gb300 import synth
-from paper_2609_04971_gb300.workloads import LLAMA_8B, QWEN3_14B, QWEN3_4B, TINY
+from paper_2609_04971_gb300.workloads import LLAMA_8B, QWEN3_14B, QWEN3_4B, QWEN3_8B_TRACE, TINY
 
 pytestmark = pytest.mark.gpu
 
@@ -133,6 +133,7 @@ def test_full_size_sampled(wl):
     QWEN3_4B.scaled(name="few_g8_nb32_n4", n_layers=1, batch=1, n_q_heads=64, n_kv_heads=8, window=12, n_beacons=32,
                     L=700, budget=500, n_init=64, n_clusters=32, n_new=4),   # 32 rows, 32 beacons
     QWEN3_4B.scaled(name="qwen3_4b_decode_step", n_new=1),          # all 4608 instances, sampled
+    QWEN3_8B_TRACE.scaled(name="qwen3_8b_trace_decode_step"),       # the long trace's step: 16 beacons, 4608
 ], ids=lambda w: w.name)
 def test_few_queries_per_instance(wl):
     sample = None
