@@ -2,22 +2,28 @@
 // the decode-step pattern, where each call brings the queries of one or a few
 // generated tokens (Algorithm 2's decode branch), G * n_new <= 32 per instance.
 //
-// One warp per instance, kSmallWarps instances per CTA, no tensor cores: at a
-// handful of rows an instance is too small for the batched kernel's pipeline
-// (TMA ring, MMA screening, accumulator and bookkeeping warps), whose
-// per-instance handoffs then bound the call.  The warp copies the instance's
-// centroids to shared memory, takes each centroid's norm data, and walks the
-// queries in order:
-//   screening: fp32 dots of q with the unit centroids c / |c| (rsqrtf), summed
-//     over the lanes by a butterfly; error far below 1e-4 |q|;
-//   decision: the best valid beacon, ties to the lower one; when best and
-//     second best differ by at most 1e-4 |q| (or a norm is extreme) the query
-//     is re-decided exactly, with the same double-float arithmetic as the
-//     batched kernel, so both kernels take the same decisions;
-//   sums: per beacon, the rows assigned to it are added as the same three
-//     exact fp32 parts, turned into round(sum * 2^40), added once to the fp64
-//     running sum, and c = fp32(sum / count) to within one ulp from double-float
-//     arithmetic, as in the batched kernel's fold.
+// One warp per instance, no tensor cores: at a handful of rows an instance is
+// too small for the batched kernel's pipeline (TMA ring, MMA screening,
+// accumulator and bookkeeping warps), whose per-instance handoffs then bound
+// the call.  The warp stages the call's queries in shared memory as fp32 and
+// gives each lane one beacon:
+//   screening: lane b streams centroid b's row from HBM once and forms, in
+//     column order, its squared norm and its dot with every query; the
+//     screened value of (query r, beacon b) is dot * rsqrtf(|c_b|^2), whose
+//     error is far below 1e-4 |q|.  No cross-lane reduction is needed, and the
+//     centroids are never held in shared memory, so every instance of a
+//     decode step fits in one wave;
+//   decision: lane r scans the screened values of query r in beacon order for
+//     the best valid beacon, ties to the lower one; when best and second best
+//     differ by at most 1e-4 |q| (or a norm is extreme) the query is re-decided
+//     exactly, with the same double-float arithmetic and the same centroid
+//     norm data as the batched kernel (built only when a call needs it), so
+//     both kernels take the same decisions;
+//   sums: per touched beacon, the rows assigned to it are added as the same
+//     three exact fp32 parts, turned into round(sum * 2^40), added once to the
+//     fp64 running sum, and c = fp32(sum / count) to within one ulp from
+//     double-float arithmetic, as in the batched kernel's fold.  The running
+//     sums of every touched beacon are prefetched into L2 at once.
 // All queries of the call see the centroids as they were at call start.
 #include "bkv_device.cuh"
 #include "bkv_internal.h"
@@ -25,8 +31,6 @@
 
 namespace bkv {
 namespace {
-
-constexpr int kSmallWarps = 8;
 
 struct SmallArgs {
   int n_inst, nq, nb;
@@ -37,134 +41,225 @@ struct SmallArgs {
   int* assign_out;         // [n_inst * nq] or nullptr
 };
 
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
+// Per-warp shared memory (floats), for at most NQ queries of head_dim D:
+//   qs    [NQ][D + 4]   the queries as fp32; the 4-float pad makes the row-per-lane
+//                       16-byte reads of the norm pass conflict-free
+//   sc    [NQ][33]      screened value of (query r, beacon b) at r * 33 + b
+//   cninv [kMaxBeacons] double-float 1 / |c_b| (exact re-decisions only)
+template <int D, int NQ>
+struct SmallLayout {
+  static constexpr int kPitch = D + 4;
+  static constexpr int kScPitch = 33;
+  static constexpr int kQs = 0;
+  static constexpr int kSc = NQ * kPitch;
+  static constexpr int kCninv = kSc + NQ * kScPitch;             // even: DF-aligned
+  static constexpr int kPerWarp = kCninv + 2 * kMaxBeacons;      // a multiple of 4: float4-aligned warps
+  static constexpr int kWarps = NQ <= 8 ? 8 : 4;
+  static_assert(kSc % 4 == 0 && kCninv % 2 == 0 && kPerWarp % 4 == 0, "shared-memory alignment");
+};
 
-template <int D>
-__global__ void __launch_bounds__(32 * kSmallWarps) update_small_kernel(SmallArgs a) {
-  extern __shared__ __align__(16) float small_cent[];  // [kSmallWarps][nb][D]
-  __shared__ DF cninv_sh[kSmallWarps][kMaxBeacons];
-  __shared__ float inv_sh[kSmallWarps][kMaxBeacons];
+// Up to this many touched beacons have their running sums loaded at once (all of them are
+// prefetched into L2 first).
+constexpr int kFoldChunk = 2;
+
+template <int D, int NQ>
+__global__ void __launch_bounds__(32 * SmallLayout<D, NQ>::kWarps, NQ <= 8 ? 4 : 2)
+    update_small_kernel(SmallArgs a) {
+  using Lay = SmallLayout<D, NQ>;
+  constexpr int P = Lay::kPitch, SP = Lay::kScPitch;
+  extern __shared__ __align__(16) float small_sh[];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int e = blockIdx.x * kSmallWarps + w;
+  const int e = blockIdx.x * Lay::kWarps + w;
   if (e >= a.n_inst) return;  // whole warp
   const int nb = a.nb, nq = a.nq;
-  float* cs = small_cent + static_cast<size_t>(w) * nb * D;
+  float* qs = small_sh + static_cast<size_t>(w) * Lay::kPerWarp + Lay::kQs;
+  float* sc = small_sh + static_cast<size_t>(w) * Lay::kPerWarp + Lay::kSc;
+  DF* cninv = reinterpret_cast<DF*>(small_sh + static_cast<size_t>(w) * Lay::kPerWarp + Lay::kCninv);
   const size_t cbase = static_cast<size_t>(e) * nb * D;
   const __nv_bfloat16* qe = a.q + static_cast<size_t>(e) * nq * D;
   const long long cnt_lane = lane < nb ? a.counts[static_cast<size_t>(e) * nb + lane] : 0;  // lane b: beacon b's count
-  for (int i = lane; i < nb * D / 4; i += 32)
-    reinterpret_cast<float4*>(cs)[i] = reinterpret_cast<const float4*>(a.cent + cbase)[i];
-  __syncwarp();
 
-  // ---- norm data of every centroid (the operations of the batched kernel's operand build)
-  uint32_t vmask = 0;  // valid beacons: count > 0 and a nonzero centroid
-  bool degenerate = false;
-  for (int b = 0; b < nb; ++b) {
-    float n2 = 0.f;
-    DF n2d{0.f, 0.f};
-    int nz = 0;
-#pragma unroll
-    for (int k = 0; k < D / 32; ++k) {
-      const float c = cs[b * D + lane + 32 * k];
-      n2 = fmaf(c, c, n2);
-      n2d = df_add(n2d, df_two_prod(c, c));
-      nz |= (c != 0.f);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      n2 += __shfl_xor_sync(0xffffffffu, n2, o);
-      nz |= __shfl_xor_sync(0xffffffffu, nz, o);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1)
-      n2d = df_add(n2d, DF{__shfl_xor_sync(0xffffffffu, n2d.hi, o), __shfl_xor_sync(0xffffffffu, n2d.lo, o)});
-    const bool ok = __shfl_sync(0xffffffffu, cnt_lane, b) > 0 && nz;
-    bool plain = true;
-    DF inv_df{0.f, 0.f};
-    if (ok) inv_df = centroid_inv_norm(n2d, n2, plain);
-    if (lane == 0) {
-      cninv_sh[w][b] = inv_df;
-      inv_sh[w][b] = ok ? rsqrtf(n2) : 0.f;
-    }
-    if (ok) vmask |= 1u << b;
-    if (!plain) degenerate = true;
+  // ---- the call's queries, bf16 -> fp32 (exact), 8 values per 16-byte load; rows nq..NQ-1 are zero
+  for (int i = lane; i < NQ * D / 8; i += 32) {
+    const int r = i / (D / 8), c = (i % (D / 8)) * 8;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (r < nq) v = reinterpret_cast<const uint4*>(qe)[i];
+    float4* dst = reinterpret_cast<float4*>(qs + r * P + c);
+    dst[0] = make_float4(__uint_as_float(v.x << 16), __uint_as_float(v.x & 0xffff0000u), __uint_as_float(v.y << 16),
+                         __uint_as_float(v.y & 0xffff0000u));
+    dst[1] = make_float4(__uint_as_float(v.z << 16), __uint_as_float(v.z & 0xffff0000u), __uint_as_float(v.w << 16),
+                         __uint_as_float(v.w & 0xffff0000u));
   }
   __syncwarp();
 
-  // ---- decisions, against the centroids at call start; lane r keeps query r's beacon
-  int my_b = -1;
-  for (int r = 0; r < nq; ++r) {
-    float x[D / 32];
+  // ---- lane b: centroid b's squared norm and its dot with every query, in column order
+  const bool has_row = lane < nb;
+  const float4* crow = reinterpret_cast<const float4*>(a.cent + cbase + static_cast<size_t>(has_row ? lane : 0) * D);
+  float acc[NQ];
 #pragma unroll
-    for (int j = 0; j < D / 32; ++j) x[j] = __bfloat162float(qe[static_cast<size_t>(r) * D + lane + 32 * j]);
+  for (int r = 0; r < NQ; ++r) acc[r] = 0.f;
+  float n2 = 0.f;
+  int nz = 0;
+#pragma unroll(NQ <= 4 ? 4 : 2)
+  for (int k = 0; k < D / 4; ++k) {
+    const float4 c = has_row ? crow[k] : make_float4(0.f, 0.f, 0.f, 0.f);
+    n2 = fmaf(c.x, c.x, n2);
+    n2 = fmaf(c.y, c.y, n2);
+    n2 = fmaf(c.z, c.z, n2);
+    n2 = fmaf(c.w, c.w, n2);
+    nz |= (c.x != 0.f) | (c.y != 0.f) | (c.z != 0.f) | (c.w != 0.f);
+#pragma unroll
+    for (int r = 0; r < NQ; ++r) {
+      const float4 x = *reinterpret_cast<const float4*>(qs + r * P + 4 * k);  // same address in every lane
+      acc[r] = fmaf(x.x, c.x, acc[r]);
+      acc[r] = fmaf(x.y, c.y, acc[r]);
+      acc[r] = fmaf(x.z, c.z, acc[r]);
+      acc[r] = fmaf(x.w, c.w, acc[r]);
+    }
+  }
+  const bool valid = has_row && cnt_lane > 0 && nz;  // count > 0 and a nonzero centroid
+  const uint32_t vmask = __ballot_sync(0xffffffffu, valid);
+  const bool degenerate = __any_sync(0xffffffffu, valid && !(n2 > 1e-30f && n2 < 1e30f));
+  const float inv = valid ? rsqrtf(n2) : 0.f;
+#pragma unroll
+  for (int r = 0; r < NQ; ++r)
+    if (r < nq) sc[r * SP + lane] = valid ? acc[r] * inv : -INFINITY;
+  __syncwarp();
+
+  // ---- lane r: decision for query r against the centroids at call start
+  int dec = -1;
+  bool need_exact = false;
+  if (lane < nq) {
+    const float* qr = qs + lane * P;
     float qn2 = 0.f;
-#pragma unroll
-    for (int j = 0; j < D / 32; ++j) qn2 = fmaf(x[j], x[j], qn2);
-    qn2 = warp_sum(qn2);
+#pragma unroll 8
+    for (int k = 0; k < D / 4; ++k) {
+      const float4 x = *reinterpret_cast<const float4*>(qr + 4 * k);
+      qn2 = fmaf(x.x, x.x, qn2);
+      qn2 = fmaf(x.y, x.y, qn2);
+      qn2 = fmaf(x.z, x.z, qn2);
+      qn2 = fmaf(x.w, x.w, qn2);
+    }
     float best = -INFINITY, second = -INFINITY;
-    int bi = -1;
     for (int b = 0; b < nb; ++b) {
       if (!((vmask >> b) & 1u)) continue;
-      const float inv = inv_sh[w][b];
-      float p = 0.f;
-#pragma unroll
-      for (int j = 0; j < D / 32; ++j) p = fmaf(x[j], cs[b * D + lane + 32 * j] * inv, p);
-      p = warp_sum(p);
+      const float p = sc[lane * SP + b];
       if (p > best) {
         second = best;
         best = p;
-        bi = b;
+        dec = b;
       } else if (p > second) {
         second = p;
       }
     }
-    int dec = bi;
-    if (bi >= 0 && (degenerate || !(qn2 > 1e-30f && qn2 < 1e30f) || !(best - second > kMarginRel * sqrtf(qn2))))
-      dec = exact_decision<D>(
-          x, nb, [&](int b, int col) { return cs[b * D + col]; }, [&](int b) { return ((vmask >> b) & 1u) != 0; },
-          cninv_sh[w]);
-    if (a.assign_out && lane == 0) a.assign_out[static_cast<size_t>(e) * nq + r] = dec;
-    if (lane == r) my_b = dec;
+    need_exact =
+        dec >= 0 && (degenerate || !(qn2 > 1e-30f && qn2 < 1e30f) || !(best - second > kMarginRel * sqrtf(qn2)));
   }
 
-  // ---- per beacon: exact sum of its rows, added once to the running sum
-  for (int b = 0; b < nb; ++b) {
-    const uint32_t rows = __ballot_sync(0xffffffffu, lane < nq && my_b == b);
-    if (!rows) continue;
-    Parts p[D / 32];
+  // ---- close calls: exact re-decisions, with the batched kernel's centroid norm data
+  const uint32_t need = __ballot_sync(0xffffffffu, need_exact);
+  if (need) {
+    for (int b = 0; b < nb; ++b) {
+      if (!((vmask >> b) & 1u)) continue;  // warp-uniform
+      float n2b = 0.f;
+      DF n2d{0.f, 0.f};
 #pragma unroll
-    for (int j = 0; j < D / 32; ++j) p[j] = Parts{0.f, 0.f, 0.f};
-    for (uint32_t m = rows; m; m &= m - 1) {
+      for (int k = 0; k < D / 32; ++k) {
+        const float c = a.cent[cbase + static_cast<size_t>(b) * D + lane + 32 * k];
+        n2b = fmaf(c, c, n2b);
+        n2d = df_add(n2d, df_two_prod(c, c));
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) n2b += __shfl_xor_sync(0xffffffffu, n2b, o);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1)
+        n2d = df_add(n2d, DF{__shfl_xor_sync(0xffffffffu, n2d.hi, o), __shfl_xor_sync(0xffffffffu, n2d.lo, o)});
+      bool plain = true;
+      const DF inv_df = centroid_inv_norm(n2d, n2b, plain);
+      if (lane == 0) cninv[b] = inv_df;
+    }
+    __syncwarp();
+    for (uint32_t m = need; m; m &= m - 1) {
       const int r = __ffs(m) - 1;
+      float x[D / 32];
 #pragma unroll
-      for (int j = 0; j < D / 32; ++j) parts_add(p[j], __bfloat162float(qe[static_cast<size_t>(r) * D + lane + 32 * j]));
+      for (int j = 0; j < D / 32; ++j) x[j] = qs[r * P + lane + 32 * j];
+      const int d = exact_decision<D>(
+          x, nb, [&](int b, int col) { return a.cent[cbase + static_cast<size_t>(b) * D + col]; },
+          [&](int b) { return ((vmask >> b) & 1u) != 0; }, cninv);
+      if (lane == r) dec = d;
     }
-    const size_t ci = static_cast<size_t>(e) * nb + b;
-    const long long cnt = __shfl_sync(0xffffffffu, cnt_lane, b) + __popc(rows);
-    const DF rcp = count_reciprocal(cnt);
-#pragma unroll
-    for (int j = 0; j < D / 32; ++j) {
-      const size_t gi = cbase + static_cast<size_t>(b) * D + lane + 32 * j;
-      const double s_new = __dadd_rn(a.sums[gi], fixed40_to_double(fixed40(p[j])));
-      a.sums[gi] = s_new;
-      a.cent[gi] = centroid_value(s_new, rcp);
-    }
-    if (lane == 0) a.counts[ci] = cnt;
   }
+  if (a.assign_out && lane < nq) a.assign_out[static_cast<size_t>(e) * nq + lane] = dec;
+
+  // ---- per touched beacon: exact sum of its rows, added once to the running sum
+  uint32_t touched = __reduce_or_sync(0xffffffffu, dec >= 0 ? (1u << dec) : 0u);
+  for (uint32_t m = touched; m; m &= m - 1) {
+    const double* srow = a.sums + cbase + static_cast<size_t>(__ffs(m) - 1) * D + lane;
+#pragma unroll
+    for (int j = 0; j < D / 32; ++j) asm volatile("prefetch.global.L2 [%0];" ::"l"(srow + 32 * j));
+  }
+  while (touched) {
+    int bs[kFoldChunk];
+    int nbk = 0;
+#pragma unroll
+    for (int i = 0; i < kFoldChunk; ++i) {
+      bs[i] = touched ? __ffs(touched) - 1 : 0;
+      if (touched) {
+        touched &= touched - 1;
+        nbk = i + 1;
+      }
+    }
+    double s_old[kFoldChunk][D / 32];
+#pragma unroll
+    for (int i = 0; i < kFoldChunk; ++i)
+#pragma unroll
+      for (int j = 0; j < D / 32; ++j)
+        s_old[i][j] = i < nbk ? a.sums[cbase + static_cast<size_t>(bs[i]) * D + lane + 32 * j] : 0.0;
+#pragma unroll
+    for (int i = 0; i < kFoldChunk; ++i) {
+      if (i >= nbk) break;  // warp-uniform
+      const int b = bs[i];
+      const uint32_t rows = __ballot_sync(0xffffffffu, lane < nq && dec == b);
+      Parts p[D / 32];
+#pragma unroll
+      for (int j = 0; j < D / 32; ++j) p[j] = Parts{0.f, 0.f, 0.f};
+      for (uint32_t m = rows; m; m &= m - 1) {
+        const int r = __ffs(m) - 1;
+#pragma unroll
+        for (int j = 0; j < D / 32; ++j) parts_add(p[j], qs[r * P + lane + 32 * j]);
+      }
+      const long long cnt = __shfl_sync(0xffffffffu, cnt_lane, b) + __popc(rows);
+      const DF rcp = count_reciprocal(cnt);
+#pragma unroll
+      for (int j = 0; j < D / 32; ++j) {
+        const size_t gi = cbase + static_cast<size_t>(b) * D + lane + 32 * j;
+        const double s_new = __dadd_rn(s_old[i][j], fixed40_to_double(fixed40(p[j])));
+        a.sums[gi] = s_new;
+        a.cent[gi] = centroid_value(s_new, rcp);
+      }
+      if (lane == 0) a.counts[static_cast<size_t>(e) * nb + b] = cnt;
+    }
+  }
+}
+
+template <int D, int NQ>
+cudaError_t launch_small_dq(const SmallArgs& a, cudaStream_t st) {
+  using Lay = SmallLayout<D, NQ>;
+  const size_t smem = sizeof(float) * Lay::kWarps * Lay::kPerWarp;
+  cudaError_t e = cudaFuncSetAttribute(update_small_kernel<D, NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  update_small_kernel<D, NQ><<<(a.n_inst + Lay::kWarps - 1) / Lay::kWarps, 32 * Lay::kWarps, smem, st>>>(a);
+  return cudaGetLastError();
 }
 
 template <int D>
 cudaError_t launch_small_d(const SmallArgs& a, cudaStream_t st) {
-  const size_t smem = sizeof(float) * kSmallWarps * a.nb * D;
-  cudaError_t e = cudaFuncSetAttribute(update_small_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
-  update_small_kernel<D><<<(a.n_inst + kSmallWarps - 1) / kSmallWarps, 32 * kSmallWarps, smem, st>>>(a);
-  return cudaGetLastError();
+  if (a.nq <= 4) return launch_small_dq<D, 4>(a, st);
+  if (a.nq <= 8) return launch_small_dq<D, 8>(a, st);
+  if (a.nq <= 16) return launch_small_dq<D, 16>(a, st);
+  return launch_small_dq<D, 32>(a, st);
 }
 
 }  // namespace
