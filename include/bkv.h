@@ -298,11 +298,15 @@ int bkv_profile_read(bkv_ctx* ctx, double* ms, int64_t* launches, int32_t n_kern
  *   dev_status  device int32 or NULL: cleared by the call, set non-zero if a
  *               kernel's bounded wait expires (outputs are then invalid).
  *   err_msg     host buffer of err_len bytes or NULL: reason of a failure.
+ * The rotary table (rope_theta != 0) reaches the device inside the
+ * parameters of small kernels on `stream`, 16 KB per launch: no copy from
+ * host memory, and the call does not wait for earlier work on the stream.
  * All calls share the scratch array and it keeps the previous call's
  * contents; calls that overlap on the GPU (other streams, other threads
  * without ordering) race on it.  The array's device address is looked up
- * with cudaGetSymbolAddress during the first call on each device (with that
- * device current), so make that first call before any stream capture.
+ * with cudaGetSymbolAddress during the first call on each device (any call
+ * that passes argument validation, with that device current), so make that
+ * first call before any stream capture.
  */
 int bkv_compress_static(const bkv_config* cfg, const float* centroids, const int64_t* counts, void* K, void* V,
                         int32_t L, int32_t budget, int64_t t_pos, const void* q_recent, const int64_t* recent_pos,

@@ -120,6 +120,13 @@ def _stream(stream) -> ctypes.c_void_p:
     return ctypes.c_void_p(handle)
 
 
+def _expect(t: torch.Tensor | None, n: int, name: str) -> None:
+    """The C ABI receives bare pointers and trusts the sizes that the shape implies: a tensor of the
+    wrong element count is a ValueError here instead of an out-of-bounds access on the device."""
+    if t is not None and t.numel() != n:
+        raise ValueError(f"{name} has {t.numel()} elements; the configured shape needs {n}")
+
+
 def _check(rc: int, where: str, ctx=None) -> None:
     if rc != BKV_OK:
         detail = _l().bkv_last_error(ctx).decode() if ctx is not None else ""
@@ -226,7 +233,26 @@ def bkv_compress_static(cfg: BkvConfig, centroids, counts, K, V, L: int, budget:
 
     For callers that cannot allocate on the device, e.g. an engine whose KV
     page allocator owns all of HBM.  Scratch lives in a fixed 16 MiB array
-    inside the library; concurrent calls on different streams race on it."""
+    inside the library; concurrent calls on different streams race on it.
+    Every tensor's element count is checked against the sizes cfg implies
+    before any pointer reaches the library."""
+    c = cfg
+    n_inst = c.n_layers * c.batch * c.n_kv_heads
+    if n_inst < 1 or c.head_dim < 1 or c.capacity < 1 or budget < 1 or c.window < 0 or c.n_beacons < 0:
+        raise ValueError("cfg must describe at least one instance of head_dim, capacity and budget >= 1")
+    _expect(K, n_inst * c.capacity * c.head_dim, "K")
+    _expect(V, n_inst * c.capacity * c.head_dim, "V")
+    _expect(kept_idx_out, n_inst * int(budget), "kept_idx_out")
+    _expect(scores_out, n_inst * c.capacity, "scores_out")
+    _expect(q_recent, c.n_layers * c.batch * c.n_q_heads * c.window * c.head_dim, "q_recent")
+    _expect(centroids, n_inst * c.n_beacons * c.head_dim, "centroids")
+    _expect(counts, n_inst * c.n_beacons, "counts")
+    if dev_status is not None and dev_status.numel() < 1:
+        raise ValueError("dev_status must hold one int32")
+    if recent_pos is None:
+        recent_pos = []
+    if c.window > 0 and len(recent_pos) != c.window:
+        raise ValueError(f"recent_pos has {len(recent_pos)} positions; the window is {c.window}")
     pos = (ctypes.c_int64 * max(1, len(recent_pos)))(*[int(p) for p in recent_pos])
     msg = ctypes.create_string_buffer(256)
     rc = _l().bkv_compress_static(
@@ -279,13 +305,8 @@ class BeaconKV:
         except Exception:  # noqa: BLE001 - interpreter shutdown
             pass
 
-    # The C ABI receives bare pointers and trusts the sizes that the context's shape implies; these
-    # checks turn a tensor of the wrong size into a ValueError here instead of an out-of-bounds access
-    # on the device.
-    @staticmethod
-    def _expect(t: torch.Tensor | None, n: int, name: str) -> None:
-        if t is not None and t.numel() != n:
-            raise ValueError(f"{name} has {t.numel()} elements; this context's shape needs {n}")
+    # The C ABI receives bare pointers and trusts the sizes that the context's shape implies (_expect).
+    _expect = staticmethod(_expect)
 
     def _rows(self, q: torch.Tensor, name: str) -> int:
         """Queries per query head of a [n_layers, batch, n_q_heads, n, head_dim] block."""

@@ -22,6 +22,11 @@
 //   * the device address of the array is looked up with cudaGetSymbolAddress
 //     the first time this entry point runs on a device (with that device
 //     current), so that first call should come before any stream capture.
+//
+// The rotary table of a call (at most 65 positions x 64 frequency pairs, in
+// fp64 and fp32) reaches the device as by-value kernel parameters, in chunks
+// of 16 KB that a small kernel writes into the array: no copy from pageable
+// host memory, so the call never waits for the stream.
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
@@ -73,6 +78,53 @@ bool encode(CUtensorMap* map, const void* base, uint64_t rows, int d, uint32_t b
 }
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+// One chunk of the rotary table, passed by value: 16-byte units [first, first + count).
+constexpr int kRopeChunkUnits = 1024;
+struct RopeChunk {
+  uint32_t first, count;
+  uint4 unit[kRopeChunkUnits];
+};
+
+__global__ void __launch_bounds__(256) rope_param_kernel(const __grid_constant__ RopeChunk c, uint4* table) {
+  for (uint32_t i = threadIdx.x; i < c.count; i += blockDim.x) table[c.first + i] = c.unit[i];
+}
+
+// 16-byte unit u of the table laid out as bkv_compress lays it out: units [0, n) are the fp64
+// (cos, sin) entries, units [n, 3n/2) two fp32 (cos, sin) entries each (n is even: d/2 is 32 or 64).
+// Entry k is slot k / h (recent slot w < W at recent_pos[w], slot W at t_pos), frequency k % h.
+struct RopeTable {
+  double theta;
+  int d, h, W;
+  int64_t t_pos;
+  const int64_t* recent_pos;
+  size_t n;
+  void entry(size_t k, double& c, double& s) const {
+    const int slot = static_cast<int>(k / h), i = static_cast<int>(k % h);
+    const double pos = static_cast<double>(slot < W ? recent_pos[slot] : t_pos);
+    const double inv_freq = std::pow(theta, -static_cast<double>(2 * i) / static_cast<double>(d));
+    const double ang = pos * inv_freq;
+    c = std::cos(ang);
+    s = std::sin(ang);
+  }
+  uint4 unit(size_t u) const {
+    uint4 out;
+    double c, s;
+    if (u < n) {
+      entry(u, c, s);
+      const double2 v = make_double2(c, s);
+      std::memcpy(&out, &v, sizeof out);
+    } else {
+      float2 v[2];
+      for (int j = 0; j < 2; ++j) {
+        entry(2 * (u - n) + j, c, s);
+        v[j] = make_float2(static_cast<float>(c), static_cast<float>(s));
+      }
+      std::memcpy(&out, v, sizeof out);
+    }
+    return out;
+  }
+};
 
 }  // namespace
 
@@ -139,6 +191,12 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
 
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaError_t e;
+  // the set-up of this device (the array's address) happens on its first call, whatever that call keeps
+  void* base = nullptr;
+  if ((e = scratch_address(&base)) != cudaSuccess) {
+    message(err_msg, err_len, cudaGetErrorString(e));
+    return BKV_ECUDA;
+  }
   if (dev_status && (e = cudaMemsetAsync(dev_status, 0, sizeof(int32_t), st)) != cudaSuccess) {
     message(err_msg, err_len, cudaGetErrorString(e));
     return BKV_ECUDA;
@@ -149,11 +207,6 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
     return e == cudaSuccess ? BKV_OK : BKV_ECUDA;
   }
 
-  void* base = nullptr;
-  if ((e = scratch_address(&base)) != cudaSuccess) {
-    message(err_msg, err_len, cudaGetErrorString(e));
-    return BKV_ECUDA;
-  }
   unsigned char* b = static_cast<unsigned char*>(base);
   auto* qobs = reinterpret_cast<__nv_bfloat16*>(b + off_qobs);
   auto* valid = reinterpret_cast<uint32_t*>(b + off_valid);
@@ -164,25 +217,19 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
   const double theta = cfg->rope_theta;
   const int rotate = theta != 0.0;
   if (rotate) {
-    // fp64 (cos, sin) entries followed by the same entries in fp32
-    double2 tab[(bkv::kMaxWindow + 1) * 64 * 3 / 2];
-    const size_t n = static_cast<size_t>(s.W + 1) * h;
-    float2* tab32 = reinterpret_cast<float2*>(tab + n);
-    for (int slot = 0; slot <= s.W; ++slot) {
-      const double pos = static_cast<double>(slot < s.W ? recent_pos[slot] : t_pos);
-      for (int i = 0; i < h; ++i) {
-        const double inv_freq = std::pow(theta, -static_cast<double>(2 * i) / static_cast<double>(s.d));
-        const double ang = pos * inv_freq;
-        const double c = std::cos(ang), sn = std::sin(ang);
-        tab[slot * h + i] = make_double2(c, sn);
-        tab32[slot * h + i] = make_float2(static_cast<float>(c), static_cast<float>(sn));
+    // fp64 (cos, sin) entries followed by the same entries in fp32, as kernel parameters
+    const RopeTable tab{theta, s.d, h, s.W, t_pos, recent_pos, static_cast<size_t>(s.W + 1) * h};
+    const size_t units = tab.n + tab.n / 2;
+    RopeChunk chunk;
+    for (size_t u0 = 0; u0 < units; u0 += kRopeChunkUnits) {
+      chunk.first = static_cast<uint32_t>(u0);
+      chunk.count = static_cast<uint32_t>(std::min<size_t>(kRopeChunkUnits, units - u0));
+      for (uint32_t i = 0; i < chunk.count; ++i) chunk.unit[i] = tab.unit(u0 + i);
+      rope_param_kernel<<<1, 256, 0, st>>>(chunk, reinterpret_cast<uint4*>(rope));
+      if ((e = cudaGetLastError()) != cudaSuccess) {
+        message(err_msg, err_len, cudaGetErrorString(e));
+        return BKV_ECUDA;
       }
-    }
-    // pageable source: the copy has consumed `tab` when the call returns
-    if ((e = cudaMemcpyAsync(rope, tab, (sizeof(double2) + sizeof(float2)) * n, cudaMemcpyHostToDevice, st)) !=
-        cudaSuccess) {
-      message(err_msg, err_len, cudaGetErrorString(e));
-      return BKV_ECUDA;
     }
   }
   e = bkv::launch_qobs(s, static_cast<const __nv_bfloat16*>(q_recent), centroids,

@@ -187,3 +187,40 @@ def test_static_compress_rejects_bad_arguments_before_any_cuda_call(lib):
     for kw, why in cases:
         rc, msg = call(**kw)
         assert rc == bkv.BKV_EINVAL and why in msg, (kw, rc, msg)
+
+
+def test_static_binding_rejects_tensors_of_the_wrong_size():
+    """bkv_compress_static has no context, so its binding checks every tensor against the sizes cfg
+    implies (and the length of recent_pos against the window) before a pointer reaches the library:
+    a wrong size is a ValueError; right sizes reach the device-pointer check, which rejects these CPU
+    tensors."""
+    import torch
+    wl = TINY
+    nl, B, Hq, Hkv, d, W, cap, nb = (wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.window,
+                                     wl.capacity, wl.n_beacons)
+    cfg = bkv.BkvConfig(nl, B, Hq, Hkv, d, nb, W, 0, cap, wl.rope_theta, 0)
+    bf = dict(dtype=torch.bfloat16)
+    K = torch.zeros(nl, B, Hkv, cap, d, **bf)
+    qr = torch.zeros(nl, B, Hq, W, d, **bf)
+    kept = torch.zeros(nl, B, Hkv, wl.budget, dtype=torch.int32)
+    sc = torch.zeros(nl, B, Hkv, cap)
+    cent = torch.zeros(wl.n_inst, nb, d)
+    cnt = torch.zeros(wl.n_inst, nb, dtype=torch.int64)
+    pos = list(range(wl.L - W, wl.L))
+    good = dict(centroids=cent, counts=cnt, K=K, V=K, q_recent=qr, recent_pos=pos, kept_idx_out=kept,
+                scores_out=sc)
+
+    def call(**over):
+        a = dict(good, **over)
+        bkv.bkv_compress_static(cfg, a["centroids"], a["counts"], a["K"], a["V"], wl.L, wl.budget, wl.L - 1,
+                                a["q_recent"], a["recent_pos"], a["kept_idx_out"], a["scores_out"])
+
+    bad = [dict(K=K[..., :-1, :].contiguous()), dict(V=torch.zeros(nl, B, Hkv, cap, d // 2, **bf)),
+           dict(q_recent=qr[..., :-1, :].contiguous()), dict(kept_idx_out=kept[..., :-1].contiguous()),
+           dict(scores_out=sc[..., :-1].contiguous()), dict(centroids=cent[:-1]), dict(counts=cnt[:, :-1]),
+           dict(recent_pos=pos[:-1]), dict(recent_pos=None)]
+    for over in bad:
+        with pytest.raises(ValueError):
+            call(**over)
+    with pytest.raises(TypeError, match="CUDA tensor"):
+        call()
