@@ -23,7 +23,7 @@
  *   - beacons are kept per KV head and fed by all G query heads of its group;
  *     they are maintained as running-mean centroids seeded by FPS; in the
  *     Continual FPS mode they are instead each query head's fill-and-compress
- *     buffer (Eq. 9), whose FPS decisions are taken in fp32 as in the kernels;
+ *     buffer (Eq. 9), compressed by the same fp64 FPS (Algorithm 1);
  *   - cosine with a zero vector is 0 (FPS) / the query is skipped (assignment);
  *   - argmin / argmax ties go to the lowest index;
  *   - RoPE uses the rotate-half pairing (i, i + d/2) with
@@ -120,69 +120,85 @@ static double* widen_rows(const uint16_t* q, int n, int d) {
  *   while fewer than m picked:
  *     r   = argmin over unpicked j of S_j;   pick r
  *     S_j = max(S_j, cos(q_j, q_r)) for the unpicked j
- * picks[k] is the k-th selected row.  gap[k] is the distance from the chosen
- * value to the runner-up value of the same argmin (+inf when there is none),
- * which the parity tests use to recognise ties.
+ * Ties go to the lowest index.  picks[k] is the k-th selected row.  gap[k] is
+ * the distance from the minimum of step k to the runner-up value (+inf when
+ * there is none) and alt[k] the runner-up's row (-1 when there is none): the
+ * parity tests use them to recognise near-ties.
+ *
+ * Adoption (test harness only): where forced is not NULL and forced[k] >= 0,
+ * step k takes row forced[k] instead of the argmin - the choice another
+ * implementation, whose similarities carry rounding errors, may make at a
+ * near-tie - and the farthest-point loop continues from it.  margin[k]
+ * receives the value of the row taken minus the minimum (0 for the argmin),
+ * and vals[k * N + j] the value step k minimises for row j (+inf for rows
+ * picked before it).  A forced row that is out of range or already picked
+ * makes the call return -1.  alt, margin and vals may be NULL.
  * Returns the number of picks (min(m, N)).
  */
-int bkvo_fps(const uint16_t* q, int N, int d, int m, int32_t* picks, double* gap) {
+int bkvo_fps_adopt(const uint16_t* q, int N, int d, int m, const int32_t* forced, int32_t* picks, double* gap,
+                   int32_t* alt, double* margin, double* vals) {
   if (m > N) m = N;
   if (m <= 0) return 0;
   double* x = widen_rows(q, N, d);
-  double* S = (double*)malloc(sizeof(double) * (size_t)N);
+  double* val = (double*)malloc(sizeof(double) * (size_t)N); /* the quantity minimised at the current step */
   char* sel = (char*)calloc((size_t)N, 1);
+  int got = m;
 
-  /* average cosine similarity of every query to the whole set */
-  int p = -1;
-  double best = INFINITY, second = INFINITY;
+  /* step 0 minimises the average cosine similarity of every query to the whole set */
   for (int i = 0; i < N; ++i) {
     double sum = 0.0;
     for (int j = 0; j < N; ++j) sum = sum + cosine(x + (size_t)i * d, x + (size_t)j * d, d, NULL);
-    double avg = sum / (double)N;
-    if (avg < best) {
-      second = best;
-      best = avg;
-      p = i;
-    } else if (avg < second) {
-      second = avg;
-    }
+    val[i] = sum / (double)N;
   }
-  if (p < 0) p = 0; /* only reachable with non-finite inputs */
-  picks[0] = p;
-  gap[0] = second - best;
-  sel[p] = 1;
-  for (int j = 0; j < N; ++j) S[j] = cosine(x + (size_t)j * d, x + (size_t)p * d, d, NULL);
-
-  for (int k = 1; k < m; ++k) {
-    int r = -1;
+  for (int k = 0; k < m; ++k) {
+    int r = -1, r2 = -1;
     double b1 = INFINITY, b2 = INFINITY;
     for (int j = 0; j < N; ++j) {
       if (sel[j]) continue;
-      if (S[j] < b1) {
+      if (val[j] < b1) {
         b2 = b1;
-        b1 = S[j];
+        r2 = r;
+        b1 = val[j];
         r = j;
-      } else if (S[j] < b2) {
-        b2 = S[j];
+      } else if (val[j] < b2) {
+        b2 = val[j];
+        r2 = j;
       }
     }
     if (r < 0) { /* only reachable with non-finite inputs */
-      m = k;
+      got = k;
       break;
     }
-    picks[k] = r;
+    if (vals)
+      for (int j = 0; j < N; ++j) vals[(size_t)k * N + j] = sel[j] ? INFINITY : val[j];
+    int c = r;
+    if (forced && forced[k] >= 0) {
+      c = forced[k];
+      if (c >= N || sel[c]) {
+        got = -1;
+        break;
+      }
+    }
+    picks[k] = c;
     gap[k] = b2 - b1;
-    sel[r] = 1;
+    if (alt) alt[k] = r2;
+    if (margin) margin[k] = val[c] - b1;
+    sel[c] = 1;
+    /* S_j: the similarity to the first pick, then the running maximum over the picks */
     for (int j = 0; j < N; ++j) {
       if (sel[j]) continue;
-      double c = cosine(x + (size_t)j * d, x + (size_t)r * d, d, NULL);
-      if (c > S[j]) S[j] = c;
+      double cj = cosine(x + (size_t)j * d, x + (size_t)c * d, d, NULL);
+      if (k == 0 || cj > val[j]) val[j] = cj;
     }
   }
   free(sel);
-  free(S);
+  free(val);
   free(x);
-  return m;
+  return got;
+}
+
+int bkvo_fps(const uint16_t* q, int N, int d, int m, int32_t* picks, double* gap) {
+  return bkvo_fps_adopt(q, N, d, m, NULL, picks, gap, NULL, NULL, NULL);
 }
 
 /* ------------------------------------------------------------------ */
@@ -190,127 +206,61 @@ int bkvo_fps(const uint16_t* q, int N, int d, int m, int32_t* picks, double* gap
 /* ------------------------------------------------------------------ */
 
 /*
- * Algorithm 1 with every similarity taken in fp32, the precision of the
- * buffer kernels (the argmins are integer decisions; both sides take them in
- * the same precision, and the pins compare them with the fp64 bkvo_fps):
- *   dot32(a, b) = fmaf(a_{d-1}, b_{d-1}, ... fmaf(a_0, b_0, 0.f))    (i increasing)
- *   n_a         = sqrtf(dot32(a, a))
- *   cos32(a, b) = dot32(a, b) / (n_a * n_b), or 0 when a norm is 0
- *   avg_i       = (sum over j = 0 .. N-1 of cos32(q_i, q_j), fp32, j increasing) / N
- * then the same first pick, S_j and farthest-point loop as bkvo_fps, ties to
- * the lowest index.  gap[k] is the runner-up distance of the k-th argmin.
- */
-static float dot32(const float* a, const float* b, int d) {
-  float s = 0.f;
-  for (int i = 0; i < d; ++i) s = fmaf(a[i], b[i], s);
-  return s;
-}
-
-int bkvo_fps32(const uint16_t* q, int N, int d, int m, int32_t* picks, double* gap) {
-  if (m > N) m = N;
-  if (m <= 0) return 0;
-  float* x = (float*)malloc(sizeof(float) * (size_t)N * (size_t)d);
-  for (size_t i = 0; i < (size_t)N * (size_t)d; ++i) x[i] = (float)bkvo_bf16_to_f64(q[i]);
-  float* nrm = (float*)malloc(sizeof(float) * (size_t)N);
-  float* cs = (float*)malloc(sizeof(float) * (size_t)N * (size_t)N);
-  float* S = (float*)malloc(sizeof(float) * (size_t)N);
-  char* sel = (char*)calloc((size_t)N, 1);
-  for (int i = 0; i < N; ++i) nrm[i] = sqrtf(dot32(x + (size_t)i * d, x + (size_t)i * d, d));
-  for (int i = 0; i < N; ++i)
-    for (int j = 0; j < N; ++j) {
-      const float den = nrm[i] * nrm[j];
-      cs[(size_t)i * N + j] = (nrm[i] == 0.f || nrm[j] == 0.f)
-                                  ? 0.f
-                                  : dot32(x + (size_t)i * d, x + (size_t)j * d, d) / den;
-    }
-  int p = -1;
-  float best = INFINITY, second = INFINITY;
-  for (int i = 0; i < N; ++i) {
-    float sum = 0.f;
-    for (int j = 0; j < N; ++j) sum = sum + cs[(size_t)i * N + j];
-    const float avg = sum / (float)N;
-    if (avg < best) {
-      second = best;
-      best = avg;
-      p = i;
-    } else if (avg < second) {
-      second = avg;
-    }
-  }
-  if (p < 0) p = 0; /* only reachable with non-finite inputs */
-  picks[0] = p;
-  gap[0] = (double)second - (double)best;
-  sel[p] = 1;
-  for (int j = 0; j < N; ++j) S[j] = cs[(size_t)j * N + p];
-  for (int k = 1; k < m; ++k) {
-    int r = -1;
-    float b1 = INFINITY, b2 = INFINITY;
-    for (int j = 0; j < N; ++j) {
-      if (sel[j]) continue;
-      if (S[j] < b1) {
-        b2 = b1;
-        b1 = S[j];
-        r = j;
-      } else if (S[j] < b2) {
-        b2 = S[j];
-      }
-    }
-    if (r < 0) { /* only reachable with non-finite inputs */
-      m = k;
-      break;
-    }
-    picks[k] = r;
-    gap[k] = (double)b2 - (double)b1;
-    sel[r] = 1;
-    for (int j = 0; j < N; ++j) {
-      if (sel[j]) continue;
-      const float c = cs[(size_t)j * N + r];
-      if (c > S[j]) S[j] = c;
-    }
-  }
-  free(sel);
-  free(S);
-  free(cs);
-  free(nrm);
-  free(x);
-  return m;
-}
-
-/*
  * The fill-and-compress buffer of one query head (Eq. 9): every new query is
  * appended in order; when the buffer holds b_max queries it is replaced by
- * its FPS selection of b_min queries, in pick order.
+ * its FPS selection (Algorithm 1, fp64 similarities as in bkvo_fps) of b_min
+ * queries, in pick order.
  *   buf     bf16 [b_max][d], rows [0, *size) in use; updated in place.
  *   q_new   bf16 [n_new][d].
- *   events  if not NULL, receives for each compression its b_min picks
- *           (indices into the full buffer) and gaps, events_cap compressions at most.
- * Returns the number of compressions.
+ *   forced  NULL, or [events_cap][b_min] picks dictated to the compressions
+ *           (-1: the argmin), passed to bkvo_fps_adopt (test harness only).
+ *   ev_*    if not NULL, receive for each compression (events_cap at most) its
+ *           b_min picks (indices into the full buffer), gaps, runner-up rows,
+ *           margins and candidate values ([b_min][b_max] per compression), as
+ *           bkvo_fps_adopt reports them.
+ * Returns the number of compressions, or -1 if a forced pick was invalid.
  */
 int bkvo_cfps_update(uint16_t* buf, int32_t* size, int b_min, int b_max, const uint16_t* q_new, int n_new, int d,
-                     int32_t* ev_picks, double* ev_gaps, int events_cap) {
-  int n_ev = 0;
-  int32_t* picks = (int32_t*)malloc(sizeof(int32_t) * (size_t)(b_min > 0 ? b_min : 1));
-  double* gaps = (double*)malloc(sizeof(double) * (size_t)(b_min > 0 ? b_min : 1));
+                     const int32_t* forced, int32_t* ev_picks, double* ev_gaps, int32_t* ev_alts, double* ev_margins,
+                     double* ev_vals, int events_cap) {
+  int n_ev = 0, bad = 0;
+  const size_t nm = (size_t)(b_min > 0 ? b_min : 1);
+  int32_t* picks = (int32_t*)malloc(sizeof(int32_t) * nm);
+  double* gaps = (double*)malloc(sizeof(double) * nm);
+  int32_t* alts = (int32_t*)malloc(sizeof(int32_t) * nm);
+  double* margins = (double*)malloc(sizeof(double) * nm);
+  double* vals = (double*)malloc(sizeof(double) * nm * (size_t)b_max);
   uint16_t* tmp = (uint16_t*)malloc(sizeof(uint16_t) * (size_t)b_max * (size_t)d);
-  for (int n = 0; n < n_new; ++n) {
+  for (int n = 0; n < n_new && !bad; ++n) {
     memcpy(buf + (size_t)(*size) * d, q_new + (size_t)n * d, sizeof(uint16_t) * (size_t)d);
     *size += 1;
     if (*size >= b_max) {
-      int got = bkvo_fps32(buf, *size, d, b_min, picks, gaps);
+      const int32_t* f = (forced && n_ev < events_cap) ? forced + (size_t)n_ev * nm : NULL;
+      int got = bkvo_fps_adopt(buf, *size, d, b_min, f, picks, gaps, alts, margins, vals);
+      if (got < 0) {
+        bad = 1;
+        break;
+      }
       for (int k = 0; k < got; ++k) memcpy(tmp + (size_t)k * d, buf + (size_t)picks[k] * d, sizeof(uint16_t) * (size_t)d);
       memcpy(buf, tmp, sizeof(uint16_t) * (size_t)got * (size_t)d);
-      if (ev_picks && n_ev < events_cap) {
-        memcpy(ev_picks + (size_t)n_ev * b_min, picks, sizeof(int32_t) * (size_t)got);
-        memcpy(ev_gaps + (size_t)n_ev * b_min, gaps, sizeof(double) * (size_t)got);
+      if (n_ev < events_cap) {
+        if (ev_picks) memcpy(ev_picks + (size_t)n_ev * nm, picks, sizeof(int32_t) * (size_t)got);
+        if (ev_gaps) memcpy(ev_gaps + (size_t)n_ev * nm, gaps, sizeof(double) * (size_t)got);
+        if (ev_alts) memcpy(ev_alts + (size_t)n_ev * nm, alts, sizeof(int32_t) * (size_t)got);
+        if (ev_margins) memcpy(ev_margins + (size_t)n_ev * nm, margins, sizeof(double) * (size_t)got);
+        if (ev_vals) memcpy(ev_vals + (size_t)n_ev * nm * b_max, vals, sizeof(double) * (size_t)got * b_max);
       }
       ++n_ev;
       *size = got;
     }
   }
   free(tmp);
+  free(vals);
+  free(margins);
+  free(alts);
   free(gaps);
   free(picks);
-  return n_ev;
+  return bad ? -1 : n_ev;
 }
 
 /* ------------------------------------------------------------------ */

@@ -54,8 +54,8 @@ _SIGS = {
     "bkvo_score": (None, [_P, _P, _I, _P, _I, _I, _P]),
     "bkvo_score_agg": (None, [_P, _P, _I, _P, _I, _I, _I, _P]),
     "bkvo_score_mask": (None, [_P, _P, _P, _I, _P, _P, _I, _I, _I, _P]),
-    "bkvo_fps32": (_I, [_P, _I, _I, _I, _P, _P]),
-    "bkvo_cfps_update": (_I, [_P, _P, _I, _I, _P, _I, _I, _P, _P, _I]),
+    "bkvo_fps_adopt": (_I, [_P, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
+    "bkvo_cfps_update": (_I, [_P, _P, _I, _I, _P, _I, _I, _P, _P, _P, _P, _P, _P, _I]),
     "bkvo_select": (_I, [_P, _I, _I, _I, _I, _P, _P]),
     "bkvo_gather": (None, [_P, _P, _P, _I, _I]),
     "bkvo_step_many": (_I, [_P, _I, _I, _I, _I, _I, _I, _I, _P, _I, _P, _P, _I64, _D, _I, _I,
@@ -124,33 +124,72 @@ def fps(q_bits: np.ndarray, m: int, lib=None):
     return picks[:got].copy(), gaps[:got].copy()
 
 
-def fps32(q_bits: np.ndarray, m: int, lib=None):
-    """Algorithm 1 with the similarities in fp32 (sequential fused dot products), the
-    precision of the Continual FPS kernels.  Returns (picks, gaps)."""
+def fps_adopt(q_bits: np.ndarray, m: int, forced: np.ndarray | None = None, lib=None):
+    """Algorithm 1 in fp64 where forced[k] >= 0 dictates the k-th pick (a choice another implementation
+    made at a near-tie; test harness only).  Returns (picks, gaps, alts, margins, vals): the runner-up
+    distance and row of each step's argmin, how far the row taken lies above the minimum, and the value
+    each step minimises per row ([m, N], +inf for rows already taken).  Raises ValueError for a forced
+    row that is out of range or already taken."""
     q = _c(q_bits, np.uint16)
     n, d = q.shape
-    picks = np.full(max(m, 1), -1, np.int32)
-    gaps = np.zeros(max(m, 1), np.float64)
-    got = (lib or load()).bkvo_fps32(_p(q), n, d, m, _p(picks), _p(gaps))
-    return picks[:got].copy(), gaps[:got].copy()
+    k = max(m, 1)
+    f = None if forced is None else _c(np.asarray(forced).reshape(-1)[:k], np.int32)
+    if f is not None and f.shape[0] < k:
+        f = np.concatenate([f, np.full(k - f.shape[0], -1, np.int32)])
+    picks = np.full(k, -1, np.int32)
+    gaps = np.zeros(k, np.float64)
+    alts = np.full(k, -1, np.int32)
+    margins = np.zeros(k, np.float64)
+    vals = np.zeros((k, max(n, 1)), np.float64)
+    got = (lib or load()).bkvo_fps_adopt(_p(q), n, d, m, _p(f), _p(picks), _p(gaps), _p(alts), _p(margins),
+                                         _p(vals))
+    if got < 0:
+        raise ValueError("a forced FPS pick is out of range or already taken")
+    return picks[:got].copy(), gaps[:got].copy(), alts[:got].copy(), margins[:got].copy(), vals[:got, :n].copy()
 
 
-def cfps_update(buf_bits: np.ndarray, size: int, b_min: int, b_max: int, q_new_bits: np.ndarray, lib=None):
+def cfps_events(size: int, b_min: int, b_max: int, n_new: int) -> int:
+    """Compressions of a Continual FPS buffer of `size` rows over n_new arrivals."""
+    n = 0
+    for _ in range(n_new):
+        size += 1
+        if size >= b_max:
+            size, n = b_min, n + 1
+    return n
+
+
+def cfps_update(buf_bits: np.ndarray, size: int, b_min: int, b_max: int, q_new_bits: np.ndarray, lib=None,
+                forced: np.ndarray | None = None) -> dict:
     """Continual FPS (Eq. 9) of one query head: append each new query; at b_max queries
-    compress the buffer to its FPS selection of b_min.  buf_bits: uint16 [>= size, d].
-    Returns (buffer uint16 [b_max, d] with rows [0, size) in use, size, picks [events, b_min],
-    gaps [events, b_min])."""
+    compress the buffer to its fp64 FPS selection of b_min.  buf_bits: uint16 [>= size, d].
+    forced: None or [events, b_min] dictated picks (-1 = the argmin; test harness only).
+    Returns dict(buf uint16 [b_max, d] with rows [0, size) in use, size, and per compression
+    picks / gaps / alts / margins [events, b_min] and vals [events, b_min, b_max])."""
     d = q_new_bits.shape[-1]
     buf = np.zeros((b_max, d), np.uint16)
     buf[:size] = buf_bits[:size]
     q = _c(q_new_bits.reshape(-1, d), np.uint16)
     n_new = q.shape[0]
-    cap = n_new // max(b_max - b_min, 1) + 2
-    ev_p = np.full((cap, max(b_min, 1)), -1, np.int32)
-    ev_g = np.zeros((cap, max(b_min, 1)), np.float64)
+    cap = cfps_events(size, b_min, b_max, n_new)
+    w = max(b_min, 1)
+    shape = (max(cap, 1), w)
+    ev_p = np.full(shape, -1, np.int32)
+    ev_g = np.zeros(shape, np.float64)
+    ev_a = np.full(shape, -1, np.int32)
+    ev_m = np.zeros(shape, np.float64)
+    ev_v = np.zeros(shape + (b_max,), np.float64)
+    f = None
+    if forced is not None:
+        f = np.full(shape, -1, np.int32)
+        fa = np.asarray(forced, np.int32).reshape(-1, w)[:shape[0]]
+        f[:fa.shape[0]] = fa
     sz = np.array([size], np.int32)
-    n_ev = (lib or load()).bkvo_cfps_update(_p(buf), _p(sz), b_min, b_max, _p(q), n_new, d, _p(ev_p), _p(ev_g), cap)
-    return buf, int(sz[0]), ev_p[:n_ev].copy(), ev_g[:n_ev].copy()
+    n_ev = (lib or load()).bkvo_cfps_update(_p(buf), _p(sz), b_min, b_max, _p(q), n_new, d, _p(f), _p(ev_p),
+                                            _p(ev_g), _p(ev_a), _p(ev_m), _p(ev_v), shape[0])
+    if n_ev < 0:
+        raise ValueError("a forced FPS pick is out of range or already taken")
+    return dict(buf=buf, size=int(sz[0]), picks=ev_p[:n_ev].copy(), gaps=ev_g[:n_ev].copy(),
+                alts=ev_a[:n_ev].copy(), margins=ev_m[:n_ev].copy(), vals=ev_v[:n_ev].copy())
 
 
 def init_beacons(q_bits: np.ndarray, nb: int, lib=None):

@@ -2,9 +2,12 @@
 
 Every query head is checked: the FPS seeding (fp64 similarities; picks equal up
 to ties below 1e-12), the fill-and-compress buffer after a call of many new
-queries (fp32 decisions, taken with the same operations on both sides, so the
-buffers must be identical), the compress on the resulting beacons (scores,
-kept set, compacted rows, as in tests/parity.py) and the post-eviction merge.
+queries, the compress on the resulting beacons (scores, kept set, compacted
+rows, as in tests/parity.py) and the post-eviction merge.  The buffer, beacon
+and merge FPS steps are compared with Algorithm 1 in fp64: the kernels decide
+from fp32 similarities, so where the fp64 runner-up lies within
+tests/parity.cfps_tie_bound of the minimum either row is accepted and the
+oracle continues from the GPU's choice (tests/parity.search_branches).
 """
 import numpy as np
 import pytest
@@ -75,7 +78,7 @@ def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False, 
     buf2 = buf2.view(torch.int16).numpy().view(np.uint16).reshape(-1, b_max, d)
     size0, size1, size2 = (x.numpy().reshape(-1) for x in (size0, size1, size2))
     heads = (insts[:, None] * G + np.arange(G)[None, :]).reshape(-1)
-    fps_ties = 0
+    fps_ties = buf_ties = 0
     for h in heads:
         # ---- seeding: fp64 FPS of the head's prompt queries
         picks, gaps = O.fps(q_init[h], b_min, lib)
@@ -84,16 +87,15 @@ def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False, 
             first = next(k for k in range(b_min) if not np.array_equal(buf0[h, k], q_init[h][picks[k]]))
             assert gaps[first] < P.ASSIGN_TIE, f"head {h}: seed pick {first} differs, fp64 gap {gaps[first]:.2e}"
             fps_ties += 1
-        # ---- update from the GPU's seed: identical fp32 decisions
-        want, wsize, _, _ = O.cfps_update(buf0[h], int(size0[h]), b_min, b_max, q_new[h], lib)
-        assert size1[h] == wsize, f"head {h}: size {size1[h]} vs {wsize}"
-        np.testing.assert_array_equal(buf1[h, :wsize], want[:wsize], err_msg=f"head {h}: buffer after update")
+        # ---- update from the GPU's seed: fp64 Eq. 9 up to near-ties of the fp32 decisions
+        buf_ties += P.match_cfps_update(buf0[h], int(size0[h]), b_min, b_max, q_new[h], buf1[h], int(size1[h]), lib,
+                                        tag=f"head {h}: buffer after update")
 
     # every head: the sizes of a head depend only on the call's lengths
     assert np.all(size0 == b_min)
     assert np.all(size1 == size1[heads[0]]) and np.all(size2 == size2[heads[0]])
 
-    rel_max, swaps = 0.0, 0
+    rel_max, swaps, cmp_ties = 0.0, 0, 0
     kept_h = kept.view(n_inst, budget).cpu().numpy()
     s_h = scores.view(n_inst, wl.capacity).cpu().numpy()
     if L > budget:  # every instance: ascending, the recent window kept
@@ -101,12 +103,12 @@ def _run_cfps(wl, seed, b_min, L=None, budget=None, n_new=None, mean_agg=False, 
         assert np.all(kept_h[:, budget - W:] == np.arange(L - W, L))
     for i, e in enumerate(insts):
         hs = slice(e * G, (e + 1) * G)
-        r, sw = P.check_cfps_compress(wl, b_min, buf1[hs], size1[hs], q_rec[hs], inp["recent_pos"], inp["t_pos"],
-                                      Kb[i], Vb[i], K1[i], V1[i], kept_h[e], s_h[e], L, budget, buf2[hs], size2[hs],
-                                      lib, tag=f"instance {e}", mean=mean_agg, causal=causal)
-        rel_max, swaps = max(rel_max, r), swaps + sw
-    print(f"{wl.name}: {len(heads)} heads checked, seed ties {fps_ties}, max score rel err {rel_max:.2e}, "
-          f"swaps {swaps}")
+        r, sw, t = P.check_cfps_compress(wl, b_min, buf1[hs], size1[hs], q_rec[hs], inp["recent_pos"],
+                                         inp["t_pos"], Kb[i], Vb[i], K1[i], V1[i], kept_h[e], s_h[e], L, budget,
+                                         buf2[hs], size2[hs], lib, tag=f"instance {e}", mean=mean_agg, causal=causal)
+        rel_max, swaps, cmp_ties = max(rel_max, r), swaps + sw, cmp_ties + t
+    print(f"{wl.name}: {len(heads)} heads checked, seed ties {fps_ties}, buffer ties {buf_ties}, "
+          f"beacon/merge ties {cmp_ties}, max score rel err {rel_max:.2e}, swaps {swaps}")
 
 
 @pytest.mark.parametrize("wl,b_min,seed", [

@@ -12,9 +12,10 @@ heads per KV head, drifting query clusters) after a 128-token prompt:
     (bkv_compress with the frozen beacons and the recent queries), and each
     buffer becomes the FPS selection of its beacons and recent queries.
 
-Every update is checked against the oracle's buffer (identical fp32
-decisions) and every compress as in tests/parity.py, always from the state the
-GPU carried forward.
+Every update is checked against the oracle's fp64 buffer (Eq. 9, Algorithm 1)
+up to near-ties of the kernels' fp32 decisions (tests/parity.search_branches),
+and every compress as in tests/parity.py, always from the state the GPU
+carried forward.
 """
 import numpy as np
 import pytest
@@ -62,7 +63,7 @@ def test_algorithm2_trace_every_step(steps, b_min, kv_min, kv_grow):
         buf, sizes = bk.cfps_state()
         return _bits(buf).reshape(-1, b_max, d), sizes.cpu().numpy().reshape(-1)
 
-    updates = compresses = swaps = 0
+    updates = compresses = swaps = ties = 0
     worst = 0.0
     try:
         bk.init_beacons(q_init)
@@ -78,9 +79,8 @@ def test_algorithm2_trace_every_step(steps, b_min, kv_min, kv_grow):
                 nbuf, nsize = state()
                 qh = _bits(q).reshape(-1, 1, d)                     # [heads, 1, d]
                 for h in range(qh.shape[0]):
-                    want, wsize, _, _ = O.cfps_update(buf[h], int(size[h]), b_min, b_max, qh[h], lib)
-                    assert nsize[h] == wsize, f"step {step} head {h}: size {nsize[h]} vs {wsize}"
-                    np.testing.assert_array_equal(nbuf[h, :wsize], want[:wsize], err_msg=f"step {step} head {h}")
+                    ties += P.match_cfps_update(buf[h], int(size[h]), b_min, b_max, qh[h], nbuf[h], int(nsize[h]),
+                                                lib, tag=f"step {step} head {h}")
                 buf, size = nbuf, nsize
                 updates += 1
             else:                                                    # recent phase (beacons frozen)
@@ -102,10 +102,10 @@ def test_algorithm2_trace_every_step(steps, b_min, kv_min, kv_grow):
                 qr = _bits(q_recent).reshape(-1, W, d)
                 for e in range(n_inst):
                     hs = slice(e * G, (e + 1) * G)
-                    r, sw = P.check_cfps_compress(wl, b_min, buf[hs], size[hs], qr[hs], recent_pos, pos, K0[e], V0[e],
-                                                  K1[e], V1[e], kept_h[e], s_h[e], L, kv_min, nbuf[hs], nsize[hs],
-                                                  lib, tag=f"step {step} instance {e}")
-                    worst, swaps = max(worst, r), swaps + sw
+                    r, sw, t = P.check_cfps_compress(wl, b_min, buf[hs], size[hs], qr[hs], recent_pos, pos, K0[e],
+                                                     V0[e], K1[e], V1[e], kept_h[e], s_h[e], L, kv_min, nbuf[hs],
+                                                     nsize[hs], lib, tag=f"step {step} instance {e}")
+                    worst, swaps, ties = max(worst, r), swaps + sw, ties + t
                 buf, size = nbuf, nsize
                 L = kv_min
                 recent, recent_pos = [], []
@@ -114,6 +114,6 @@ def test_algorithm2_trace_every_step(steps, b_min, kv_min, kv_grow):
     finally:
         bk.close()
     print(f"trace (Algorithm 2, Continual FPS): {steps} steps, {updates} updates, {compresses} compresses, "
-          f"worst score rel err {worst:.2e}, boundary swaps {swaps}")
+          f"worst score rel err {worst:.2e}, boundary swaps {swaps}, FPS near-tie departures {ties}")
     first = kv_max - wl.prefill                                      # steps until the first compress
     assert compresses == 1 + (steps - first) // kv_grow

@@ -32,8 +32,8 @@ _ROPE = [(TN.test_rope_is_complex_rotation_of_rotate_half_pairs, {}),
          (TN.test_rope_preserves_norm_and_relative_position, {})]
 _FPS = [(TB.test_fps_matches_maxmin_brute_force, dict(seed=s)) for s in range(6)] + [
     (TB.test_fps_orthonormal_basis_ties_go_to_lowest_index, {}), (TB.test_fps_outlier_first, {})]
-_CFPS = [(TC.test_fps32_agrees_with_fp64_away_from_ties, dict(seed=s)) for s in range(8)] + [
-    (TC.test_fps32_orthonormal_basis_takes_indices_in_order, {}), (TC.test_fps32_zero_query_has_zero_similarity, {}),
+_CFPS = [(TC.test_fps_adopt_continues_from_a_dictated_pick, dict(seed=s)) for s in range(6)] + [
+    (TC.test_fps_orthonormal_basis_takes_indices_in_order, {}), (TC.test_fps_zero_query_has_zero_similarity, {}),
     (TC.test_cfps_buffer_matches_fp64_brute_force_simulation, {}), (TC.test_cfps_closed_forms, {})]
 _UPD = [(TB.test_update_planted_assignment_uses_cosine_not_dot, {}),
         (TB.test_update_single_beacon_is_global_mean, {}), (TB.test_update_centroid_is_mean_of_assigned, {})]
@@ -55,13 +55,11 @@ MUTANTS = [
     ("rope_interleaved_pairs", "double x1 = x[i], x2 = x[i + h];", "double x1 = x[2 * i], x2 = x[2 * i + 1];",
      _ROPE),
     ("rope_frequency_exponent", "-(double)(2 * i) / (double)d", "-(double)(i) / (double)d", _ROPE),
-    ("fps_min_update", "d, NULL);\n      if (c > S[j]) S[j] = c;", "d, NULL);\n      if (c < S[j]) S[j] = c;", _FPS),
-    ("fps_first_pick_argmax", "double avg = sum / (double)N;\n    if (avg < best) {",
-     "double avg = sum / (double)N;\n    if (-avg < best) {", _FPS),
-    ("fps32_dot_without_norms", ": dot32(x + (size_t)i * d, x + (size_t)j * d, d) / den;",
-     ": dot32(x + (size_t)i * d, x + (size_t)j * d, d);", _CFPS),
-    ("fps32_first_pick_argmax", "const float avg = sum / (float)N;\n    if (avg < best) {",
-     "const float avg = -sum / (float)N;\n    if (avg < best) {", _CFPS),
+    ("fps_min_update", "if (k == 0 || cj > val[j]) val[j] = cj;", "if (k == 0 || cj < val[j]) val[j] = cj;", _FPS),
+    ("fps_first_pick_argmax", "val[i] = sum / (double)N;", "val[i] = -sum / (double)N;", _FPS),
+    ("fps_forced_pick_ignored", "      c = forced[k];\n", "      c = r;\n", _CFPS),
+    ("fps_first_similarity_not_reset", "if (k == 0 || cj > val[j]) val[j] = cj;", "if (cj > val[j]) val[j] = cj;",
+     _FPS + _CFPS),
     ("cfps_compress_one_early", "    if (*size >= b_max) {", "    if (*size >= b_max - 1) {", _CFPS),
     ("cfps_keeps_arrival_order", "memcpy(tmp + (size_t)k * d, buf + (size_t)picks[k] * d,",
      "memcpy(tmp + (size_t)k * d, buf + (size_t)k * d,", _CFPS),
