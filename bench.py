@@ -13,10 +13,17 @@ Every step is bracketed by CUDA events on the stream the library launches on.
 
     python bench.py [--gpus N --steps K --warmup W] [--impl reference]
 
---config 3 / 4 time the same step on the Llama-8B and Qwen3-14B shapes.
+The default run also times, after the headline line's own measurement, the
+Llama-8B and Qwen3-14B steps and the whole Qwen3-8B decode trace (32768
+steps), and reports each under "configs" with its fraction of its own step
+roofline (--no-extra-configs skips them).
+
+--config 3 / 4 time the same step on the Llama-8B and Qwen3-14B shapes alone.
 --config 5 (or --trace-steps N) runs the long decode trace instead: one beacon
-update per decode step and a compress whenever the cache reaches L rows, timed
-as the total device time of the library calls over the trace (trace_main).
+update per decode step (with Continual FPS beacons, only in Algorithm 2's
+observation phase) and a compress whenever the cache reaches B_max rows, timed
+as the total device time of the library calls over the trace (trace_bench).
+--bmin-ratio 0.875 sets B_max = budget / 0.875, the paper's B_min = 7/8 B_max.
 
 Prints one JSON line (rank 0).  --impl reference times the CPU oracle (the
 plain fp64 restatement of the method) on the host cores instead.
@@ -61,6 +68,13 @@ def parse():
                     help="Continual FPS: beacons per query head (the buffer holds this + window queries)")
     ap.add_argument("--trace-steps", type=int, default=0,
                     help="decode steps of the long-trace mode (0: the workload's own; config 5 runs a trace)")
+    ap.add_argument("--bmin-ratio", type=float, default=1.0,
+                    help="trace mode: B_min / B_max; B_min is the workload's budget and B_max = budget / ratio "
+                         "(1.0: the workload's own L, e.g. 7/8 = 0.875 as in the paper's setting)")
+    ap.add_argument("--extra-steps", type=int, default=30, help="timed steps of each additional workload")
+    ap.add_argument("--no-extra-configs", action="store_true",
+                    help="time only the headline workload (by default the Qwen3-4B run also times the "
+                         "Llama-8B and Qwen3-14B steps and the Qwen3-8B decode trace)")
     return ap.parse_args()
 
 
@@ -207,7 +221,7 @@ def reference_arm(args, wl, rank: int) -> None:
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(times),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": config_block(wl, args.gpus),
+        "config": dict(config_block(wl, args.gpus), beacon_mode=args.beacons),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -275,6 +289,22 @@ def rank_seed(seed: int, rank: int) -> int:
 
 
 # ------------------------------------------------------------------ main GPU bench
+class Job:
+    """Rank, device and the timing barrier of one bench process."""
+
+    def __init__(self, rank: int, world: int, local_rank: int):
+        import torch
+        self.rank, self.world, self.local_rank = rank, world, local_rank
+        self.dev = torch.device("cuda", local_rank)
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        self.gpu_index = int(vis.split(",")[local_rank]) if vis and vis.split(",")[0].isdigit() else local_rank
+
+    def barrier(self):
+        if self.world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+
 def main():
     args = parse()
     from paper_2609_04971_gb300.workloads import WORKLOADS
@@ -291,25 +321,94 @@ def main():
     if args.impl == "reference":
         reference_arm(args, wl, rank)
         return
-    if args.trace_steps or wl.trace_steps:
-        trace_main(args, wl, rank, world, local_rank, cfps)
-        return
 
     import torch
     import torch.distributed as dist
+    torch.cuda.set_device(local_rank)
+    job = Job(rank, world, local_rank)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=job.dev)
+    trace = bool(args.trace_steps or wl.trace_steps)
+    if trace:
+        out = trace_bench(args, wl, job, cfps, args.trace_steps or wl.trace_steps)
+    else:
+        out = step_bench(args, wl, job, cfps, args.steps, args.warmup, with_e2e=not args.no_e2e,
+                         with_cpu=rank == 0 and world == 1 and not args.no_cpu_baseline)
+    # the other single-GPU workloads, after the headline line's own measurement (one GPU only)
+    if world == 1 and not args.no_extra_configs and not args.layers and not cfps and args.config == 2 \
+            and not args.trace_steps:
+        out["configs"] = extra_configs(args, job)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def release_memory():
+    import gc
+
+    import torch
+    gc.collect()
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+
+
+def extra_configs(args, job) -> dict:
+    """Llama-8B and Qwen3-14B steps (30 timed steps each) and the full Qwen3-8B decode trace, each
+    summarised by its step time, its fraction of the step roofline and its dominant kernel."""
+    from paper_2609_04971_gb300.workloads import WORKLOADS
+    res = {}
+    for c in (3, 4, 5):
+        release_memory()
+        wl = WORKLOADS[c]
+        if wl.trace_steps:
+            o = trace_bench(args, wl, job, False, wl.trace_steps)
+        else:
+            o = step_bench(args, wl, job, False, args.extra_steps, max(3, args.warmup), with_e2e=False,
+                           with_cpu=False)
+        res[str(c)] = config_summary(o)
+    release_memory()
+    return res
+
+
+def config_summary(o: dict) -> dict:
+    r = o.get("roofline") or {}
+    s = {"workload": o["config"]["workload"], "metric": o["metric"], "value": o["value"], "unit": o["unit"],
+         "steps": o["steps"], "ms_per_step": o["ms_per_step"],
+         "step_roofline_ms": o["step_roofline"]["roofline_ms"], "step_roofline_frac": o["step_roofline"]["frac"],
+         "dominant_kernel": r.get("kernel"), "dominant_frac_of_hbm": r.get("frac"),
+         "kernels": {k: {kk: v[kk] for kk in ("ms_per_launch", "launches", "alg_bytes_per_launch", "frac_of_hbm")
+                         if kk in v} for k, v in o["kernels"].items()},
+         "gpu_launches": o["gpu_launches"], "clocks": o["clocks"]}
+    if "trace" in o:
+        s["trace"] = o["trace"]
+        s["compresses"] = o["config"]["compresses"]
+    return s
+
+
+def kernel_table(prof: dict, alg_bytes: dict, steps: int, hbm_gbs: float) -> dict:
+    """Per kernel: mean launch time and algorithmic bytes per launch over the measured launches.
+    alg_bytes holds each kernel's algorithmic bytes per step; with more than 64 scoring queries the
+    score kernel runs twice per step and its bytes are shared by both launches."""
+    kernels = {}
+    for name, b in alg_bytes.items():
+        ms, n = prof.get(name, (0.0, 0))
+        if n:
+            per = ms / n
+            bl = b * steps / n
+            kernels[name] = {"ms_per_launch": per, "launches": n, "alg_bytes_per_launch": bl,
+                             "achieved_gbs": bl / (per * 1e-3) / 1e9, "frac_of_hbm": bl / (per * 1e-3) / 1e9 / hbm_gbs}
+    return kernels
+
+
+def step_bench(args, wl, job, cfps: bool, steps: int, warmup: int, with_e2e: bool, with_cpu: bool) -> dict:
+    """One update + compress per step over every instance of the workload, inputs resident in HBM."""
+    import torch
     from paper_2609_04971_gb300 import bkv, synth
 
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    if world > 1:
-        dist.init_process_group("nccl", device_id=dev)
-
-    def barrier():
-        if world > 1:
-            dist.barrier()
-
+    dev, world = job.dev, job.world
     hbm_gbs, bf16_tflops, peak_src = peaks()
-    inp = synth.step_inputs(wl, rank_seed(args.seed, rank), dev)
+    inp = synth.step_inputs(wl, rank_seed(args.seed, job.rank), dev)
     K, V = inp["K"], inp["V"]
     L, budget = wl.L, wl.budget
     new_k = K[:, :, :, budget:L].clone()      # "new tokens" written back after every compress
@@ -332,35 +431,33 @@ def main():
         bk.compress(K, V, L=L, budget=budget, t_pos=t_pos, q_recent=inp["q_recent"],
                     recent_pos=[p + (L - budget) * i for p in inp["recent_pos"]], kept_out=kept)
 
-    for i in range(args.warmup):
+    for i in range(warmup):
         prepare(i)
         step(i)
     bk.sync()
     bkv.bkv_profile_read(bk.ctx)
     bkv.bkv_profile_enable(bk.ctx, True)
 
-    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
-    gpu_index = int(vis.split(",")[local_rank]) if vis and vis.split(",")[0].isdigit() else local_rank
-    sampler = ClockSampler(gpu_index)
+    sampler = ClockSampler(job.gpu_index)
     sampler.start()
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-    barrier()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    job.barrier()
     torch.cuda.synchronize()
-    for i in range(args.steps):
-        prepare(args.warmup + i)
+    for i in range(steps):
+        prepare(warmup + i)
         ev[i][0].record()
-        step(args.warmup + i)
+        step(warmup + i)
         ev[i][1].record()
     torch.cuda.synchronize()
-    barrier()
+    job.barrier()
     clocks = sampler.stop()
     bk.sync()
     prof = bkv.bkv_profile_read(bk.ctx)
     bkv.bkv_profile_enable(bk.ctx, False)
     step_ms = [a.elapsed_time(b) for a, b in ev]
     total_ms = max_over_ranks(sum(step_ms), world, dev)
-    ms_per_step = total_ms / args.steps
-    value = aggregate_throughput(wl.tokens_per_step(), world, args.steps, total_ms)
+    ms_per_step = total_ms / steps
+    value = aggregate_throughput(wl.tokens_per_step(), world, steps, total_ms)
 
     # per-kernel roofline (algorithmic bytes per launch / measured duration per launch)
     d = wl.head_dim
@@ -374,17 +471,11 @@ def main():
     if cfps:  # three launches per step: buffer update, beacon selection, merge; accounted per step
         ms, n = prof.get("cfps", (0.0, 0))
         b = cfps_bytes(wl)
-        per = ms / args.steps
+        per = ms / steps
         kernels["cfps"] = {"ms_per_step": per, "launches": n, "alg_bytes_per_step": b,
                            "achieved_gbs": b / (per * 1e-3) / 1e9, "frac_of_hbm": b / (per * 1e-3) / 1e9 / hbm_gbs,
                            "note": "per step: update (n_new queries per head) + beacon FPS + post-eviction merge"}
-    for name, b in alg_bytes.items():  # b: algorithmic bytes per step, shared by the step's launches
-        ms, n = prof.get(name, (0.0, 0))
-        if n:
-            per = ms / n
-            bl = b * args.steps / n  # more than 64 scoring queries: two score launches per step read K twice
-            kernels[name] = {"ms_per_launch": per, "launches": n, "alg_bytes_per_launch": bl,
-                             "achieved_gbs": bl / (per * 1e-3) / 1e9, "frac_of_hbm": bl / (per * 1e-3) / 1e9 / hbm_gbs}
+    kernels.update(kernel_table(prof, alg_bytes, steps, hbm_gbs))
     ms, n = prof.get("rope_stage", (0.0, 0))
     if n:  # the rotary table of a compress, 24 (W + 1) d / 2 bytes copied from pinned host memory
         kernels["rope_stage"] = {"ms_per_launch": ms / n, "launches": n}
@@ -405,10 +496,10 @@ def main():
     launches = sum(n for _, n in prof.values())
 
     out = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps,
+        "warmup": warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": dict(config_block(wl, world), beacon_mode=args.beacons),
+        "config": dict(config_block(wl, world), beacon_mode=args.beacons if cfps else "centroid"),
         "roofline": roofline,
         "step_roofline": {"alg_bytes": step_bytes, "alg_flops": step_flops,
                           "roofline_ms": step_roof_s * 1e3, "frac": step_roof_s * 1e3 / ms_per_step},
@@ -419,16 +510,13 @@ def main():
     }
 
     # end to end through the public API with host buffers
-    if not args.no_e2e:
-        out["e2e"] = e2e(bk, wl, inp, args, dev, world, barrier)
+    if with_e2e:
+        out["e2e"] = e2e(bk, wl, inp, args, dev, world, job.barrier)
     del new_k, new_v, flush
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if with_cpu:
         out["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds, args.seed)
     bk.close()
-    if rank == 0:
-        print(json.dumps(out), flush=True)
-    if world > 1:
-        dist.destroy_process_group()
+    return out
 
 
 # ------------------------------------------------------------------ long decode trace
@@ -447,38 +535,50 @@ def trace_schedule(prefill: int, budget: int, grow: int, steps: int) -> list[int
     return sched
 
 
-def trace_main(args, wl, rank: int, world: int, local_rank: int, cfps: bool) -> None:
+def trace_phases(prefill: int, b_min: int, b_max: int, window: int, steps: int) -> list[str]:
+    """Algorithm 2's phase of every decode step, by the cache length L after the step's token is
+    appended: 'obs' while L <= B_max - n_recent (the query feeds the observation buffer), 'recent'
+    while B_max - n_recent < L <= B_max (the query is kept with its position for the next eviction);
+    the step at which L = B_max also evicts down to B_min."""
+    out, L = [], prefill
+    for _ in range(steps):
+        L += 1
+        out.append("obs" if L <= b_max - window else "recent")
+        if L >= b_max:
+            L = b_min
+    return out
+
+
+def trace_bench(args, wl, job, cfps: bool, steps: int) -> dict:
     """Long decode trace.  After a prompt of wl.prefill tokens (FPS-seeded beacons), every decode step
-    adds one pre-RoPE query per query head (one beacon update with n_new = 1) and one K / V row; when
-    the cache reaches wl.L rows it is compressed to wl.budget.  The timed quantity is the compression
-    overhead of the whole trace: the device time of every bkv_update_beacons and bkv_compress call, each
-    bracketed by CUDA events on the library's stream.  The model's own work between them (appending the
-    K / V row, building the recent-query block) runs outside the events.  Queries and K / V rows cycle
-    through TRACE_POOL pre-generated decode steps (drifting clusters within the pool), so that host-side
-    input generation does not pace the trace."""
+    adds one pre-RoPE query per query head and one K / V row; when the cache reaches B_max = wl.L rows it
+    is compressed to B_min = wl.budget (Algorithm 2).  With running-mean centroids every decode query
+    updates the beacons.  With Continual FPS buffers the queries follow Algorithm 2's phases: they feed
+    the buffers while L <= B_max - n_recent, the beacons are then fixed (the library selects them from
+    the unchanged buffer at the eviction), and the last n_recent queries are kept with their positions
+    for the eviction and the merge that follows it.  The timed quantity is the compression overhead of
+    the whole trace: the device time of every bkv_update_beacons and bkv_compress call, each bracketed
+    by CUDA events on the library's stream.  The model's own work between them (appending the K / V
+    row, building the recent-query block) runs outside the events.  Queries and K / V rows cycle through
+    TRACE_POOL pre-generated decode steps (drifting clusters within the pool), so that host-side input
+    generation does not pace the trace."""
     import collections
 
     import torch
-    import torch.distributed as dist
     from paper_2609_04971_gb300 import bkv, synth
 
-    steps = args.trace_steps or wl.trace_steps
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    if world > 1:
-        dist.init_process_group("nccl", device_id=dev)
-
-    def barrier():
-        if world > 1:
-            dist.barrier()
-
+    dev, world = job.dev, job.world
+    if args.bmin_ratio < 1.0:  # B_min = ratio * B_max, with B_min the workload's budget
+        b_max = int(round(wl.budget / args.bmin_ratio))
+        wl = wl.scaled(L=b_max, name=f"{wl.name}_Bmax{b_max}")
     hbm_gbs, bf16_tflops, peak_src = peaks()
     nl, B, Hkv, d, W = wl.n_layers, wl.batch, wl.n_kv_heads, wl.head_dim, wl.window
     cap, budget = wl.L, wl.budget
     sched = trace_schedule(wl.prefill, budget, cap - budget, steps)
+    phases = trace_phases(wl.prefill, budget, cap, W, steps)
     if sched and sched[0] + 1 < W:
         raise SystemExit("trace: the first compress comes before the recent window has filled")
-    seed = rank_seed(args.seed, rank)
+    seed = rank_seed(args.seed, job.rank)
     gen = synth.TraceGen(wl, seed, dev)
     q_init, k0, v0 = gen.prefill()
     pool = max(W, 1, min(TRACE_POOL, steps))   # the warm-up compress takes its W recent queries from the pool
@@ -518,25 +618,26 @@ def trace_main(args, wl, rank: int, world: int, local_rank: int, cfps: bool) -> 
     ev_u = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(drain)]
     ev_c = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
             for _ in range(len(sched))]
-    upd_ms = 0.0
+    upd_ms, n_upd = 0.0, 0
     hist = collections.deque(maxlen=W)   # (query [nl, B, Hq, d], absolute position) of the latest steps
     L, pos, c = wl.prefill, wl.prefill, 0
     compress_at = set(sched)
     prof = {name: (0.0, 0) for name in bkv.KERNEL_NAMES}
 
-    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
-    gpu_index = int(vis.split(",")[local_rank]) if vis and vis.split(",")[0].isdigit() else local_rank
-    sampler = ClockSampler(gpu_index)
+    sampler = ClockSampler(job.gpu_index)
     sampler.start()
-    barrier()
+    job.barrier()
     torch.cuda.synchronize()
     wall0 = time.perf_counter()
+    pending = 0  # update events recorded since the last drain
     for s in range(steps):
         j = s % pool
-        e0, e1 = ev_u[s % drain]
-        e0.record()
-        bk.update(q_pool[j])
-        e1.record()
+        if not cfps or phases[s] == "obs":
+            e0, e1 = ev_u[pending]
+            e0.record()
+            bk.update(q_pool[j])
+            e1.record()
+            pending += 1
         K[:, :, :, L].copy_(k_pool[j])
         V[:, :, :, L].copy_(v_pool[j])
         hist.append((q_pool[j, :, :, :, 0], pos))
@@ -551,14 +652,17 @@ def trace_main(args, wl, rank: int, world: int, local_rank: int, cfps: bool) -> 
             b.record()
             c += 1
             L = budget
-        if s % drain == drain - 1 or s == steps - 1:
-            ev_u[s % drain][1].synchronize()
-            upd_ms += sum(x.elapsed_time(y) for x, y in ev_u[:s % drain + 1])
+        if pending == drain or s == steps - 1:
+            if pending:
+                ev_u[pending - 1][1].synchronize()
+                upd_ms += sum(x.elapsed_time(y) for x, y in ev_u[:pending])
+                n_upd += pending
+                pending = 0
             for name, (ms, n) in bkv.bkv_profile_read(bk.ctx).items():  # recycles the library's events
                 prof[name] = (prof[name][0] + ms, prof[name][1] + n)
     torch.cuda.synchronize()
     wall_s = time.perf_counter() - wall0
-    barrier()
+    job.barrier()
     clocks = sampler.stop()
     bk.sync()
     bkv.bkv_profile_enable(bk.ctx, False)
@@ -571,8 +675,8 @@ def trace_main(args, wl, rank: int, world: int, local_rank: int, cfps: bool) -> 
         upd_bytes = 2 * wl.n_layers * wl.batch * wl.n_q_heads * d * 2
     else:
         upd_bytes = wl.update_bytes(1)
-    trace_bytes = len(sched) * wl.compress_bytes() + steps * upd_bytes
-    trace_flops = len(sched) * wl.compress_flops() + (0 if cfps else steps * wl.update_flops(1))
+    trace_bytes = len(sched) * wl.compress_bytes() + n_upd * upd_bytes
+    trace_flops = len(sched) * wl.compress_flops() + (0 if cfps else n_upd * wl.update_flops(1))
     roof_ms = 1e3 * max(trace_bytes / (hbm_gbs * 1e9), trace_flops / (bf16_tflops * 1e12))
     per_launch_bytes = {"qobs": wl.n_inst * wl.group * W * d * 2, "score": wl.n_inst * cap * d * 2,
                         "select_gather": wl.n_inst * (budget * d * 2 * 4 + budget * 4)}
@@ -584,7 +688,7 @@ def trace_main(args, wl, rank: int, world: int, local_rank: int, cfps: bool) -> 
             continue
         k = {"ms_per_launch": ms / n, "launches": n, "ms_total": ms}
         if name in per_launch_bytes:
-            bl = per_launch_bytes[name] * (len(sched) if name != "update" else steps) / n
+            bl = per_launch_bytes[name] * (len(sched) if name != "update" else n_upd) / n
             k.update(alg_bytes_per_launch=bl, achieved_gbs=bl / (ms / n * 1e-3) / 1e9,
                      frac_of_hbm=bl / (ms / n * 1e-3) / 1e9 / hbm_gbs)
         kernels[name] = k
@@ -597,30 +701,26 @@ def trace_main(args, wl, rank: int, world: int, local_rank: int, cfps: bool) -> 
         traffic = None if dom == "update" else traffic_from_profiles(dom, wl.n_inst)
         roofline = {"bound": "hbm", "kernel": dom, "achieved": kd["achieved_gbs"], "peak": hbm_gbs, "unit": "GB/s",
                     "frac": kd["achieved_gbs"] / hbm_gbs, "traffic": traffic, "peak_source": f"{peak_src} hbm_gbs"}
-    out = {
+    return {
         "metric": METRIC, "value": tokens / (total_ms / 1e3), "unit": UNIT, "n_gpus": world, "steps": steps,
         "warmup": args.warmup, "ms_per_step": total_ms / steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": dict(config_block(wl, world), beacon_mode=args.beacons, decode_steps=steps,
-                       compresses=len(sched), query_pool_steps=pool,
-                       l2="K/V working set 10 GB > L2; no flush between decode steps"),
+        "config": dict(config_block(wl, world), beacon_mode=args.beacons if cfps else "centroid",
+                       decode_steps=steps, compresses=len(sched), beacon_updates=n_upd, b_max=cap, b_min=budget,
+                       query_pool_steps=pool, l2="K/V working set 10 GB > L2; no flush between decode steps"),
         "roofline": roofline,
         "step_roofline": {"alg_bytes": trace_bytes, "alg_flops": trace_flops, "roofline_ms": roof_ms,
                           "frac": roof_ms / total_ms,
-                          "note": "whole trace: every compress plus one update per decode step"
+                          "note": "whole trace: every compress plus every beacon update"
                                   + ("; Continual FPS updates counted as query read + buffer append only"
                                      if cfps else "")},
         "trace": {"overhead_s": total_ms / 1e3, "overhead_us_per_decode_step": 1e3 * total_ms / steps,
-                  "update_us_per_step": 1e3 * upd_ms / steps,
+                  "update_us_per_call": 1e3 * upd_ms / max(n_upd, 1),
                   "compress_ms_mean": statistics.mean(cmp_ms) if cmp_ms else 0.0,
                   "wall_s": wall_s},
         "kernels": kernels, "gpu_launches": sum(n for _, n in prof.values()), "clocks": clocks,
         "e2e": None, "e2e_note": "trace mode: device-resident inputs only",
     }
-    if rank == 0:
-        print(json.dumps(out), flush=True)
-    if world > 1:
-        dist.destroy_process_group()
 
 
 def e2e(bk, wl, inp, args, dev, world, barrier) -> dict:

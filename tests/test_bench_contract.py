@@ -37,3 +37,23 @@ def test_trace_schedule_of_the_long_trace():
     assert len(sched) == 225 and sched[0] == T.L - T.prefill - 1
     assert all(b - a == T.L - T.budget for a, b in zip(sched, sched[1:]))
     assert bench.trace_schedule(10, 8, 4, 1) == [] and bench.trace_schedule(10, 8, 4, 6) == [1, 5]
+
+
+def test_trace_phases_follow_algorithm_2():
+    """Algorithm 2: a decode step feeds the observation buffer while the cache (after its token) holds at
+    most B_max - n_recent rows, keeps its query as a recent one while it holds more, and the step that
+    reaches B_max evicts to B_min.  Here B_min = 8, B_max = 12, n_recent = 2, a 5-row prompt."""
+    import bench
+    ph = bench.trace_phases(prefill=5, b_min=8, b_max=12, window=2, steps=14)
+    # L after each step: 6..12 (evict), 9, 10, 11, 12 (evict), 9, 10, 11
+    assert ph == ["obs"] * 5 + ["recent"] * 2 + ["obs"] * 2 + ["recent"] * 2 + ["obs"] * 2 + ["recent"]
+    sched = bench.trace_schedule(5, 8, 4, 14)
+    assert sched == [6, 10]
+    # every eviction is preceded by exactly n_recent recent-phase steps
+    for s in sched:
+        assert ph[s - 1:s + 1] == ["recent", "recent"] and ph[s - 2] == "obs"
+    # the paper's 7/8 ratio on the long trace: B_min 4096 -> B_max 4681, n_recent 8
+    ph = bench.trace_phases(128, 4096, 4681, 8, 32768)
+    sched = bench.trace_schedule(128, 4096, 4681 - 4096, 32768)
+    assert all(ph[s] == "recent" and ph[s - 7] == "recent" and ph[s - 8] == "obs" for s in sched)
+    assert sum(p == "recent" for p in ph) >= 8 * len(sched)
