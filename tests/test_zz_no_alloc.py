@@ -80,3 +80,44 @@ def test_static_compress_rejects_requests_beyond_its_scratch():
     with pytest.raises(bkv.BkvError) as ei:
         bkv.bkv_compress_static(cfg, cent, counts, K, K, wl.L, wl.budget, wl.L - 1, q, list(range(wl.window)), kept)
     assert ei.value.code == bkv.BKV_EINVAL and "scratch" in str(ei.value)
+
+
+def test_static_compress_leaves_free_device_memory_unchanged():
+    """The property callers rely on: after one warm-up call (which sets the device up and loads the
+    kernels), further calls change the device's free memory by nothing.  Every tensor is allocated,
+    and the context used to build the beacon state is destroyed, before the first reading."""
+    from paper_2609_04971_gb300 import bkv, synth
+    wl = QWEN3_4B.scaled(name="static_mem", n_layers=1, batch=2, L=1000, budget=700)
+    dev = torch.device("cuda")
+    inp = synth.step_inputs(wl, 28, dev)
+    bk = bkv.BeaconKV.for_workload(wl)
+    try:
+        bk.init_beacons(inp["q_init"])
+        bk.update(inp["q_new"])
+        cent, _, counts = bk.state()
+        bk.sync()
+    finally:
+        bk.close()
+    K0, V0 = inp["K"].clone(), inp["V"].clone()
+    K, V = K0.clone(), V0.clone()
+    kept = torch.empty(wl.n_layers, wl.batch, wl.n_kv_heads, wl.budget, dtype=torch.int32, device=dev)
+    scores = torch.empty(wl.n_layers, wl.batch, wl.n_kv_heads, wl.capacity, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+
+    def call():
+        bkv.bkv_compress_static(bk.cfg, cent, counts, K, V, wl.L, wl.budget, inp["t_pos"], inp["q_recent"],
+                                inp["recent_pos"], kept, scores, status)
+
+    call()
+    torch.cuda.synchronize()
+    kept_first = kept.clone()
+    free0, _ = torch.cuda.mem_get_info(dev)
+    for _ in range(3):
+        K.copy_(K0)
+        V.copy_(V0)
+        call()
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info(dev)
+    assert free1 == free0, f"free device memory changed by {free0 - free1} bytes over three calls"
+    assert int(status.item()) == 0
+    assert torch.equal(kept, kept_first)
