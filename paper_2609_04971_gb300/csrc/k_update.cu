@@ -27,9 +27,11 @@
 // exact for 2^-31 <= |x| < 2^14, the conversion to fixed point per beacon
 // change rather than per element); re-decided rows are converted directly.
 // The per-call sum is exact and independent of the order.  It is then
-// added once to the fp64 running sum (the only fp64 operation per element
-// besides the int64 conversion), and c = fp32(sum / count) to within one fp32
-// ulp from double-float arithmetic on the sum's bits.
+// added once to the fp64 running sum, correctly rounded (fold_sum_fp64: one
+// fp64 addition while the call's sum is exact in fp64, fold_sum's exact
+// integer addition beyond; the bookkeeping warps that fold have the fp64 pipe
+// to themselves), and c = fp32(sum / count) to within one fp32 ulp from
+// double-float arithmetic on the sum's bits.
 //
 // Warp roles (26 warps): warp 0 TMA producer; warp 1 TMEM allocation and MMA
 // issue; warps 2..5 screeners (one per TMEM lane quarter: decisions, the
@@ -610,7 +612,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
         const int ai = b * D + (col % kCols) * 32 + col / kCols;  // the accumulator cell of (b, col)
         if (add_cnt[pb][b] > 0) {
           const size_t gi = static_cast<size_t>(e) * cells + c;
-          const double s_new = __dadd_rn(sums_sm[c], fixed40_to_double(acc_i[ai]));
+          const double s_new = fold_sum_fp64(sums_sm[c], acc_i[ai]);
           a.sums[gi] = s_new;
           a.cent[gi] = centroid_value(s_new, rcp_sh[b]);
         }

@@ -103,11 +103,84 @@ __device__ __forceinline__ double fixed40_to_double(long long acc) {
   return __longlong_as_double(__double_as_longlong(__ll2double_rn(acc)) - (40LL << 52));
 }
 
+// The double nearest to t * 2^-40 (ties to even) for 0 < |t| < 2^63, from integer operations
+// only: the leading bit fixes the exponent, the bits below the 53-bit significand are rounded.
+__device__ __forceinline__ double fixed40_round(long long t) {
+  const unsigned long long sign = t < 0 ? (1ull << 63) : 0ull;
+  const unsigned long long a = t < 0 ? 0ull - static_cast<unsigned long long>(t) : static_cast<unsigned long long>(t);
+  int msb = 63 - __clzll(static_cast<long long>(a));
+  unsigned long long mant;
+  if (msb <= 52) {
+    mant = a << (52 - msb);
+  } else {
+    const int sh = msb - 52;
+    mant = a >> sh;
+    const unsigned long long rem = a & ((1ull << sh) - 1ull), half = 1ull << (sh - 1);
+    if (rem > half || (rem == half && (mant & 1ull))) ++mant;
+    if (mant >> 53) {
+      mant >>= 1;
+      ++msb;
+    }
+  }
+  const unsigned long long e = static_cast<unsigned long long>(msb - 40 + 1023);
+  return __longlong_as_double(static_cast<long long>(sign | (e << 52) | (mant & ((1ull << 52) - 1ull))));
+}
+
+// s + acc * 2^-40 rounded to the nearest double (ties to even), the running sum after a call
+// whose exact sum is acc (fixed point, 40 fractional bits).  fp64 arithmetic is slow on this
+// part, so the common case stays in integers: when s is a multiple of 2^-40 below 2^22 in
+// magnitude (every sum built from queries of 2^-31 or more is) and |acc| < 2^61, s becomes the
+// integer s * 2^40, the two integers are added exactly and the total is rounded once.  This is
+// the correctly rounded sum, as an fp64 addition of s and acc * 2^-40 (exact below 2^53) gives.
+// Other values take the fp64 route.
+__device__ __forceinline__ double fold_sum(double s, long long acc) {
+  if (acc == 0) return s;
+  const unsigned long long bits = static_cast<unsigned long long>(__double_as_longlong(s));
+  const int e = static_cast<int>((bits >> 52) & 0x7ff);
+  const long long lim = 1LL << 61;
+  if (acc > -lim && acc < lim && e < 1023 + 22) {
+    long long f = 0;
+    bool ok = true;
+    if (e != 0) {
+      const unsigned long long m = (bits & ((1ull << 52) - 1ull)) | (1ull << 52);
+      const int sh = e - 1035;  // s * 2^40 = m * 2^(e - 1075 + 40)
+      if (sh >= 0) {
+        f = static_cast<long long>(m << sh);
+      } else if (sh > -53 && (m & ((1ull << -sh) - 1ull)) == 0ull) {
+        f = static_cast<long long>(m >> -sh);
+      } else {
+        ok = false;  // not a multiple of 2^-40
+      }
+      if (bits >> 63) f = -f;
+    } else {
+      ok = (bits << 1) == 0ull;  // +-0; subnormals take the fp64 route
+    }
+    if (ok) {
+      const long long t = f + acc;
+      return t == 0 ? 0.0 : fixed40_round(t);
+    }
+  }
+  return __dadd_rn(s, fixed40_to_double(acc));
+}
+
+// fold_sum for warps that have the fp64 pipe to themselves: below 2^53, acc * 2^-40 is exact in
+// fp64 and one fp64 addition rounds the sum once, so the result is fold_sum's, without its integer
+// instructions; larger sums take fold_sum (which rounds once where the fp64 route would round twice).
+__device__ __forceinline__ double fold_sum_fp64(double s, long long acc) {
+  const long long lim = 1LL << 53;
+  if (acc > -lim && acc < lim) return acc == 0 ? s : __dadd_rn(s, fixed40_to_double(acc));
+  return fold_sum(s, acc);
+}
+
 // 1 / n for a count n >= 1 as a double-float: the correctly rounded fp32 reciprocal of n
 // refined by one Newton-Raphson step r' = r + r (1 - n r), the residual formed exactly.
 __device__ __forceinline__ DF count_reciprocal(long long n) {
-  const float nf = static_cast<float>(n);                      // n rounded (exact below 2^24)
-  const float nl = static_cast<float>(n - static_cast<long long>(nf));
+  // 64-bit integer <-> float conversions run on the slow fp64 unit of this part: counts below 2^31
+  // (all practical ones) take the 32-bit forms, which give the same values
+  const bool small = n < (1LL << 31);
+  const float nf = small ? __int2float_rn(static_cast<int>(n)) : static_cast<float>(n);  // exact below 2^24
+  const long long nfi = small ? static_cast<long long>(__float2int_rn(nf)) : static_cast<long long>(nf);
+  const float nl = small ? __int2float_rn(static_cast<int>(n - nfi)) : static_cast<float>(n - nfi);
   const float r = __frcp_rn(nf);
   const float p = __fmul_rn(nf, r);
   const float pe = __fmaf_rn(nl, r, __fmaf_rn(nf, r, -p));     // n r - p
@@ -133,8 +206,9 @@ __device__ __forceinline__ float centroid_value(double s, DF rcp) {
   const unsigned long long m = (bits & ((1ull << 52) - 1)) | (1ull << 52);  // 53-bit significand
   const unsigned long long m_hi = (m + (1ull << 28) - 1 + ((m >> 29) & 1)) >> 29;  // m / 2^29, nearest even
   const long long rem = static_cast<long long>(m) - static_cast<long long>(m_hi << 29);  // |rem| <= 2^28
-  float hi = __fmul_rn(static_cast<float>(m_hi), pow2f(e - 1046));  // exact: m_hi <= 2^24
-  float lo = __fmul_rn(static_cast<float>(rem), pow2f(e - 1075));
+  // 32-bit conversions (m_hi <= 2^24 and |rem| <= 2^28 fit; 64-bit ones run on the slow fp64 unit)
+  float hi = __fmul_rn(__uint2float_rn(static_cast<uint32_t>(m_hi)), pow2f(e - 1046));  // exact: m_hi <= 2^24
+  float lo = __fmul_rn(__int2float_rn(static_cast<int>(rem)), pow2f(e - 1075));  // rem rounded to fp32
   if (bits >> 63) {
     hi = -hi;
     lo = -lo;

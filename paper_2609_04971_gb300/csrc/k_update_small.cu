@@ -6,11 +6,12 @@
 // too small for the batched kernel's pipeline (TMA ring, MMA screening,
 // accumulator and bookkeeping warps), whose per-instance handoffs then bound
 // the call.  The warp stages the call's queries in shared memory as fp32 and
-// gives each lane one beacon:
-//   screening: lane b streams centroid b's row from HBM once and forms, in
-//     column order, its squared norm and its dot with every query; the
-//     screened value of (query r, beacon b) is dot * rsqrtf(|c_b|^2), whose
-//     error is far below 1e-4 |q|.  No cross-lane reduction is needed, and the
+// gives each centroid row R = 32 / nb lanes (nb rounded up to a power of two):
+//   screening: the R lanes of beacon b stream its row from HBM once, in
+//     interleaved 16-byte chunks (adjacent lanes read adjacent chunks), and
+//     form its squared norm and its dot with every query, added over the R
+//     lanes at the end; the screened value of (query r, beacon b) is
+//     dot * rsqrtf(|c_b|^2), whose error is far below 1e-4 |q|.  The
 //     centroids are never held in shared memory, so every instance of a
 //     decode step fits in one wave;
 //   decision: lane r scans the screened values of query r in beacon order for
@@ -21,8 +22,9 @@
 //     both kernels take the same decisions;
 //   sums: per touched beacon, the rows assigned to it are added as the same
 //     three exact fp32 parts, turned into round(sum * 2^40), added once to the
-//     fp64 running sum, and c = fp32(sum / count) to within one ulp from
-//     double-float arithmetic, as in the batched kernel's fold.  The running
+//     fp64 running sum (fold_sum: exact integer addition and one rounding, no
+//     fp64 arithmetic in the common case), and c = fp32(sum / count) to within
+//     one ulp from double-float arithmetic, as in the batched kernel's fold.  The running
 //     sums of every touched beacon are prefetched into L2 at once.
 // All queries of the call see the centroids as they were at call start.
 #include "bkv_device.cuh"
@@ -34,6 +36,7 @@ namespace {
 
 struct SmallArgs {
   int n_inst, nq, nb;
+  int lg_rows;             // log2 of the lanes that share one centroid row (32 / nb rounded up to a power of 2)
   const __nv_bfloat16* q;  // [n_inst * nq][D] (the G query heads of an instance are adjacent)
   float* cent;             // [n_inst][nb][D]
   double* sums;            // [n_inst][nb][D]
@@ -46,6 +49,7 @@ struct SmallArgs {
 //                       16-byte reads of the norm pass conflict-free
 //   sc    [NQ][33]      screened value of (query r, beacon b) at r * 33 + b
 //   cninv [kMaxBeacons] double-float 1 / |c_b| (exact re-decisions only)
+//   qn2   [NQ]          the queries' squared norms
 template <int D, int NQ>
 struct SmallLayout {
   static constexpr int kPitch = D + 4;
@@ -53,7 +57,8 @@ struct SmallLayout {
   static constexpr int kQs = 0;
   static constexpr int kSc = NQ * kPitch;
   static constexpr int kCninv = kSc + NQ * kScPitch;             // even: DF-aligned
-  static constexpr int kPerWarp = kCninv + 2 * kMaxBeacons;      // a multiple of 4: float4-aligned warps
+  static constexpr int kQn2 = kCninv + 2 * kMaxBeacons;
+  static constexpr int kPerWarp = kQn2 + NQ;                      // a multiple of 4: float4-aligned warps
   static constexpr int kWarps = NQ <= 8 ? 8 : 4;
   static_assert(kSc % 4 == 0 && kCninv % 2 == 0 && kPerWarp % 4 == 0, "shared-memory alignment");
 };
@@ -75,33 +80,55 @@ __global__ void __launch_bounds__(32 * SmallLayout<D, NQ>::kWarps, NQ <= 8 ? 4 :
   float* qs = small_sh + static_cast<size_t>(w) * Lay::kPerWarp + Lay::kQs;
   float* sc = small_sh + static_cast<size_t>(w) * Lay::kPerWarp + Lay::kSc;
   DF* cninv = reinterpret_cast<DF*>(small_sh + static_cast<size_t>(w) * Lay::kPerWarp + Lay::kCninv);
+  float* qn2s = small_sh + static_cast<size_t>(w) * Lay::kPerWarp + Lay::kQn2;
   const size_t cbase = static_cast<size_t>(e) * nb * D;
   const __nv_bfloat16* qe = a.q + static_cast<size_t>(e) * nq * D;
   const long long cnt_lane = lane < nb ? a.counts[static_cast<size_t>(e) * nb + lane] : 0;  // lane b: beacon b's count
 
-  // ---- the call's queries, bf16 -> fp32 (exact), 8 values per 16-byte load; rows nq..NQ-1 are zero
+  // ---- the call's queries, bf16 -> fp32 (exact), 8 values per 16-byte load; rows nq..NQ-1 are zero.
+  // A row is D / 8 consecutive lanes' loads, so its squared norm (for the screening margin) is a sum
+  // over those lanes: a butterfly over D / 8 lanes, written to qn2 by the row's first lane.
+  static_assert(32 % (D / 8) == 0, "a row's loads stay inside one warp");
   for (int i = lane; i < NQ * D / 8; i += 32) {
     const int r = i / (D / 8), c = (i % (D / 8)) * 8;
     uint4 v = make_uint4(0u, 0u, 0u, 0u);
     if (r < nq) v = reinterpret_cast<const uint4*>(qe)[i];
+    const float4 x0 = make_float4(__uint_as_float(v.x << 16), __uint_as_float(v.x & 0xffff0000u),
+                                  __uint_as_float(v.y << 16), __uint_as_float(v.y & 0xffff0000u));
+    const float4 x1 = make_float4(__uint_as_float(v.z << 16), __uint_as_float(v.z & 0xffff0000u),
+                                  __uint_as_float(v.w << 16), __uint_as_float(v.w & 0xffff0000u));
     float4* dst = reinterpret_cast<float4*>(qs + r * P + c);
-    dst[0] = make_float4(__uint_as_float(v.x << 16), __uint_as_float(v.x & 0xffff0000u), __uint_as_float(v.y << 16),
-                         __uint_as_float(v.y & 0xffff0000u));
-    dst[1] = make_float4(__uint_as_float(v.z << 16), __uint_as_float(v.z & 0xffff0000u), __uint_as_float(v.w << 16),
-                         __uint_as_float(v.w & 0xffff0000u));
+    dst[0] = x0;
+    dst[1] = x1;
+    float p = x0.x * x0.x;
+    p = fmaf(x0.y, x0.y, p);
+    p = fmaf(x0.z, x0.z, p);
+    p = fmaf(x0.w, x0.w, p);
+    p = fmaf(x1.x, x1.x, p);
+    p = fmaf(x1.y, x1.y, p);
+    p = fmaf(x1.z, x1.z, p);
+    p = fmaf(x1.w, x1.w, p);
+#pragma unroll
+    for (int o = 1; o < D / 8; o <<= 1) p += __shfl_xor_sync(0xffffffffu, p, o);
+    if ((i % (D / 8)) == 0) qn2s[r] = p;
   }
   __syncwarp();
 
-  // ---- lane b: centroid b's squared norm and its dot with every query, in column order
-  const bool has_row = lane < nb;
-  const float4* crow = reinterpret_cast<const float4*>(a.cent + cbase + static_cast<size_t>(has_row ? lane : 0) * D);
+  // ---- R lanes per centroid row (R = 32 / nb rounded up to a power of two): lane l takes row
+  // l / R and its 16-byte chunks l % R, l % R + R, ... (adjacent lanes read adjacent chunks), forming
+  // the row's squared norm and its dot with every query; the R partial sums are then added
+  const int lg_r = a.lg_rows;
+  const int R = 1 << lg_r;
+  const int row = lane >> lg_r, part = lane & (R - 1);
+  const bool has_row = row < nb;
+  const float4* crow = reinterpret_cast<const float4*>(a.cent + cbase + static_cast<size_t>(has_row ? row : 0) * D);
   float acc[NQ];
 #pragma unroll
   for (int r = 0; r < NQ; ++r) acc[r] = 0.f;
   float n2 = 0.f;
   int nz = 0;
 #pragma unroll(NQ <= 4 ? 4 : 2)
-  for (int k = 0; k < D / 4; ++k) {
+  for (int k = part; k < D / 4; k += R) {
     const float4 c = has_row ? crow[k] : make_float4(0.f, 0.f, 0.f, 0.f);
     n2 = fmaf(c.x, c.x, n2);
     n2 = fmaf(c.y, c.y, n2);
@@ -110,36 +137,38 @@ __global__ void __launch_bounds__(32 * SmallLayout<D, NQ>::kWarps, NQ <= 8 ? 4 :
     nz |= (c.x != 0.f) | (c.y != 0.f) | (c.z != 0.f) | (c.w != 0.f);
 #pragma unroll
     for (int r = 0; r < NQ; ++r) {
-      const float4 x = *reinterpret_cast<const float4*>(qs + r * P + 4 * k);  // same address in every lane
+      const float4 x = *reinterpret_cast<const float4*>(qs + r * P + 4 * k);  // R distinct addresses per warp
       acc[r] = fmaf(x.x, c.x, acc[r]);
       acc[r] = fmaf(x.y, c.y, acc[r]);
       acc[r] = fmaf(x.z, c.z, acc[r]);
       acc[r] = fmaf(x.w, c.w, acc[r]);
     }
   }
-  const bool valid = has_row && cnt_lane > 0 && nz;  // count > 0 and a nonzero centroid
-  const uint32_t vmask = __ballot_sync(0xffffffffu, valid);
+  for (int o = 1; o < R; o <<= 1) {
+    n2 += __shfl_xor_sync(0xffffffffu, n2, o);
+    nz |= __shfl_xor_sync(0xffffffffu, nz, o);
+#pragma unroll
+    for (int r = 0; r < NQ; ++r) acc[r] += __shfl_xor_sync(0xffffffffu, acc[r], o);
+  }
+  const long long cnt_row = __shfl_sync(0xffffffffu, cnt_lane, row & 31);  // lane b holds beacon b's count
+  const bool valid = has_row && cnt_row > 0 && nz;  // count > 0 and a nonzero centroid
+  // every lane takes part in the shuffle (row b's validity from its first lane); lane b < nb votes it
+  const bool valid_b = __shfl_sync(0xffffffffu, valid, (lane << lg_r) & 31);
+  const uint32_t vmask = __ballot_sync(0xffffffffu, lane < nb && valid_b);
   const bool degenerate = __any_sync(0xffffffffu, valid && !(n2 > 1e-30f && n2 < 1e30f));
   const float inv = valid ? rsqrtf(n2) : 0.f;
+  if (part == 0) {
 #pragma unroll
-  for (int r = 0; r < NQ; ++r)
-    if (r < nq) sc[r * SP + lane] = valid ? acc[r] * inv : -INFINITY;
+    for (int r = 0; r < NQ; ++r)
+      if (r < nq) sc[r * SP + row] = valid ? acc[r] * inv : -INFINITY;
+  }
   __syncwarp();
 
   // ---- lane r: decision for query r against the centroids at call start
   int dec = -1;
   bool need_exact = false;
   if (lane < nq) {
-    const float* qr = qs + lane * P;
-    float qn2 = 0.f;
-#pragma unroll 8
-    for (int k = 0; k < D / 4; ++k) {
-      const float4 x = *reinterpret_cast<const float4*>(qr + 4 * k);
-      qn2 = fmaf(x.x, x.x, qn2);
-      qn2 = fmaf(x.y, x.y, qn2);
-      qn2 = fmaf(x.z, x.z, qn2);
-      qn2 = fmaf(x.w, x.w, qn2);
-    }
+    const float qn2 = qn2s[lane];
     float best = -INFINITY, second = -INFINITY;
     for (int b = 0; b < nb; ++b) {
       if (!((vmask >> b) & 1u)) continue;
@@ -234,7 +263,7 @@ __global__ void __launch_bounds__(32 * SmallLayout<D, NQ>::kWarps, NQ <= 8 ? 4 :
 #pragma unroll
       for (int j = 0; j < D / 32; ++j) {
         const size_t gi = cbase + static_cast<size_t>(b) * D + lane + 32 * j;
-        const double s_new = __dadd_rn(s_old[i][j], fixed40_to_double(fixed40(p[j])));
+        const double s_new = fold_sum(s_old[i][j], fixed40(p[j]));
         a.sums[gi] = s_new;
         a.cent[gi] = centroid_value(s_new, rcp);
       }
@@ -266,7 +295,9 @@ cudaError_t launch_small_d(const SmallArgs& a, cudaStream_t st) {
 
 cudaError_t launch_update_small(const Shape& s, const __nv_bfloat16* q_new, int n_new, float* cent, double* sums,
                                 long long* counts, int* assign_out, cudaStream_t st) {
-  SmallArgs a{s.n_inst, s.G * n_new, s.nb, q_new, cent, sums, counts, assign_out};
+  int lg = 0;
+  while ((32 >> (lg + 1)) >= s.nb && lg < 3) ++lg;  // 2^lg lanes per row, 2^lg * nb <= 32
+  SmallArgs a{s.n_inst, s.G * n_new, s.nb, lg, q_new, cent, sums, counts, assign_out};
   if (a.n_inst == 0 || a.nq == 0 || a.nb == 0) return cudaSuccess;
   if (a.nq > kUpdateSmallMaxRows || a.nb > kMaxBeacons) return cudaErrorInvalidValue;
   return s.d == 128 ? launch_small_d<128>(a, st) : launch_small_d<64>(a, st);
