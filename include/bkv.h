@@ -214,6 +214,30 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
                  const void* q_recent, const int64_t* recent_pos, int32_t* kept_idx_out, float* scores_out);
 
 /*
+ * bkv_compress with a cache length of its own for every instance: in batched
+ * decoding each sequence of the batch has its own length and position
+ * (Section 5.4), and Algorithm 2 runs per sequence.  Everything is as in
+ * bkv_compress, instance by instance, except:
+ *   L           DEVICE int32 [n_layers][batch][n_kv_heads]: rows of each
+ *               instance.  An instance with L <= budget is not touched and
+ *               gets kept_idx_out[i] = i for i < L, -1 after; an instance with
+ *               budget < L is compressed to budget rows from its own L (its
+ *               softmax runs over its L keys, its window is its last
+ *               `window` rows).  A length outside 1..capacity leaves that
+ *               instance untouched with kept_idx_out all -1, and the next
+ *               bkv_sync returns BKV_EINVAL.
+ *   t_pos       HOST int64 [batch]: position of each batch row's current
+ *               decode step (its beacons are rotated there).
+ *   recent_pos  HOST int64 [batch][window]: positions of each batch row's
+ *               recent slots.
+ *   scores_out  written for j < L of the instances that are compressed.
+ * Under BKV_F_CONTINUAL_FPS only the heads of compressed instances merge
+ * (Algorithm 2's post-eviction step).
+ */
+int bkv_compress_ragged(bkv_ctx* ctx, void* K, void* V, const int32_t* L, int32_t budget, const int64_t* t_pos,
+                        const void* q_recent, const int64_t* recent_pos, int32_t* kept_idx_out, float* scores_out);
+
+/*
  * Copies the beacon state to / from caller DEVICE buffers:
  *   centroids fp32 [n_inst][n_beacons][head_dim]
  *   sums      fp64 [n_inst][n_beacons][head_dim]

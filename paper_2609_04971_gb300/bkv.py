@@ -71,6 +71,7 @@ def load_library(path: str | None = None, build: bool = True):
             "bkv_update_beacons": (ctypes.c_int, [_P, _P, ctypes.c_int32, _P]),
             "bkv_compress": (ctypes.c_int, [_P, _P, _P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, _P, _P,
                                             _P, _P]),
+            "bkv_compress_ragged": (ctypes.c_int, [_P, _P, _P, _P, ctypes.c_int32, _P, _P, _P, _P, _P]),
             "bkv_get_state": (ctypes.c_int, [_P, _P, _P, _P]),
             "bkv_set_state": (ctypes.c_int, [_P, _P, _P, _P]),
             "bkv_get_cfps_state": (ctypes.c_int, [_P, _P, _P]),
@@ -178,6 +179,20 @@ def bkv_compress(ctx, K: torch.Tensor, V: torch.Tensor, L: int, budget: int, t_p
                              int(t_pos), _ptr(q_recent, torch.bfloat16, "q_recent"), ctypes.cast(pos, _P),
                              _ptr(kept_idx_out, torch.int32, "kept_idx_out"),
                              _ptr(scores_out, torch.float32, "scores_out")), "bkv_compress", ctx)
+
+
+def bkv_compress_ragged(ctx, K: torch.Tensor, V: torch.Tensor, L: torch.Tensor, budget: int, t_pos, q_recent,
+                        recent_pos, kept_idx_out: torch.Tensor, scores_out: torch.Tensor | None = None) -> None:
+    """L: int32 device tensor, one cache length per instance; t_pos: one position per batch row;
+    recent_pos: one list of window positions per batch row (see include/bkv.h)."""
+    tp = (ctypes.c_int64 * max(1, len(t_pos)))(*[int(p) for p in t_pos])
+    flat = [int(p) for row in recent_pos for p in row]
+    rp = (ctypes.c_int64 * max(1, len(flat)))(*flat)
+    _check(_l().bkv_compress_ragged(ctx, _ptr(K, torch.bfloat16, "K"), _ptr(V, torch.bfloat16, "V"),
+                                    _ptr(L, torch.int32, "L"), int(budget), ctypes.cast(tp, _P),
+                                    _ptr(q_recent, torch.bfloat16, "q_recent"), ctypes.cast(rp, _P),
+                                    _ptr(kept_idx_out, torch.int32, "kept_idx_out"),
+                                    _ptr(scores_out, torch.float32, "scores_out")), "bkv_compress_ragged", ctx)
 
 
 def bkv_get_state(ctx, centroids=None, sums=None, counts=None) -> None:
@@ -339,6 +354,26 @@ class BeaconKV:
         if kept_out is None:
             kept_out = torch.empty(c.n_layers, c.batch, c.n_kv_heads, budget, dtype=torch.int32, device=K.device)
         bkv_compress(self.ctx, K, V, L, budget, t_pos, q_recent, recent_pos, kept_out, scores_out)
+        return kept_out
+
+    def compress_ragged(self, K, V, *, L, budget, t_pos, q_recent, recent_pos, kept_out=None, scores_out=None):
+        """Per-instance cache lengths: L is an int32 CUDA tensor [n_layers, batch, n_kv_heads]; t_pos and
+        recent_pos hold one position (one list of window positions) per batch row."""
+        c = self.cfg
+        per_head = c.n_layers * c.batch * c.n_kv_heads
+        self._expect(K, per_head * c.capacity * c.head_dim, "K")
+        self._expect(V, per_head * c.capacity * c.head_dim, "V")
+        self._expect(L, per_head, "L")
+        self._expect(q_recent, c.n_layers * c.batch * c.n_q_heads * c.window * c.head_dim, "q_recent")
+        if len(t_pos) != c.batch:
+            raise ValueError(f"t_pos has {len(t_pos)} positions; the batch is {c.batch}")
+        if len(recent_pos) != c.batch or any(len(r) != c.window for r in recent_pos):
+            raise ValueError(f"recent_pos must hold {c.batch} lists of {c.window} positions")
+        self._expect(kept_out, per_head * budget, "kept_out")
+        self._expect(scores_out, per_head * c.capacity, "scores_out")
+        if kept_out is None:
+            kept_out = torch.empty(c.n_layers, c.batch, c.n_kv_heads, budget, dtype=torch.int32, device=K.device)
+        bkv_compress_ragged(self.ctx, K, V, L, budget, t_pos, q_recent, recent_pos, kept_out, scores_out)
         return kept_out
 
     def state(self):

@@ -12,6 +12,7 @@
 #include <vector>
 
 #include "bkv.h"
+#include "bkv_device.cuh"
 #include "bkv_internal.h"
 
 using bkv::Shape;
@@ -47,6 +48,17 @@ struct bkv_ctx {
   cudaEvent_t rope_ev[kRopeSlots] = {};
   bool rope_used[kRopeSlots] = {};
   int rope_next = 0;
+  // per-instance lengths (bkv_compress_ragged): the instances a compress evicts from, and a rotary
+  // table per batch row followed by the causal gaps [batch][W] (int32), staged like `rope`
+  int* work = nullptr;            // [n_inst]
+  int* n_work = nullptr;          // [1]
+  unsigned char* rag = nullptr;   // device copy of the per-row tables and gaps
+  size_t rag_bytes = 0, rag_row = 0, rag_gaps_off = 0;  // total bytes; one row's table (double2 units); gaps offset
+  void* rag_pinned[kRopeSlots] = {};
+  void* rag_mapped[kRopeSlots] = {};
+  cudaEvent_t rag_ev[kRopeSlots] = {};
+  bool rag_used[kRopeSlots] = {};
+  int rag_next = 0;
   cudaEvent_t switch_ev = nullptr;  // orders a new stream after the previous one (bkv_set_stream)
   std::string last_error;
   // per-kernel timing
@@ -190,7 +202,12 @@ void free_all(bkv_ctx* c) {
   for (int i = 0; i < bkv_ctx::kRopeSlots; ++i) {
     if (c->rope_pinned[i]) cudaFreeHost(c->rope_pinned[i]);
     if (c->rope_ev[i]) cudaEventDestroy(c->rope_ev[i]);
+    if (c->rag_pinned[i]) cudaFreeHost(c->rag_pinned[i]);
+    if (c->rag_ev[i]) cudaEventDestroy(c->rag_ev[i]);
   }
+  cudaFree(c->work);
+  cudaFree(c->n_work);
+  cudaFree(c->rag);
   if (c->switch_ev) cudaEventDestroy(c->switch_ev);
 }
 
@@ -236,7 +253,13 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
   s.cap = cfg->capacity;
   s.n_obs = s.G * s.W + s.nb;
   s.n_obs_pad = (s.n_obs + 15) / 16 * 16;
+  s.batch = cfg->batch;
+  s.n_kv = cfg->n_kv_heads;
   c->stream = static_cast<cudaStream_t>(stream);
+  // per-row rotary tables ([W + 1][d / 2] fp64 pairs, then fp32 pairs) and causal gaps of a ragged compress
+  c->rag_row = static_cast<size_t>(s.W + 1) * (s.d / 2) * 3 / 2;  // double2 units (a multiple of 2: 16-byte rows)
+  c->rag_gaps_off = sizeof(double2) * c->rag_row * static_cast<size_t>(s.batch);
+  c->rag_bytes = c->rag_gaps_off + (sizeof(int32_t) * static_cast<size_t>(s.batch) * (s.W > 0 ? s.W : 1) + 15) / 16 * 16;
   cudaGetDevice(&c->device);
 
   const size_t ni = static_cast<size_t>(s.n_inst);
@@ -251,6 +274,8 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
       (e = dmalloc(&c->valid, ni * 4)) != cudaSuccess ||
       (e = dmalloc(&c->rscore, ni * s.cap)) != cudaSuccess ||
       (e = dmalloc(&c->rope, static_cast<size_t>(s.W + 1) * (s.d / 2) * 3 / 2 + 1)) != cudaSuccess ||
+      (e = dmalloc(&c->work, ni)) != cudaSuccess || (e = dmalloc(&c->n_work, 1)) != cudaSuccess ||
+      (e = dmalloc(&c->rag, c->rag_bytes)) != cudaSuccess ||
       (e = dmalloc(&c->err, 1)) != cudaSuccess) {
     const int code = (e == cudaErrorMemoryAllocation) ? BKV_ENOMEM : BKV_ECUDA;
     cudaGetLastError();
@@ -271,7 +296,10 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
   for (int i = 0; i < bkv_ctx::kRopeSlots; ++i) {
     if ((e = cudaMallocHost(reinterpret_cast<void**>(&c->rope_pinned[i]), rope_bytes)) != cudaSuccess ||
         (e = cudaHostGetDevicePointer(&c->rope_mapped[i], c->rope_pinned[i], 0)) != cudaSuccess ||
-        (e = cudaEventCreateWithFlags(&c->rope_ev[i], cudaEventDisableTiming)) != cudaSuccess) {
+        (e = cudaEventCreateWithFlags(&c->rope_ev[i], cudaEventDisableTiming)) != cudaSuccess ||
+        (e = cudaMallocHost(&c->rag_pinned[i], c->rag_bytes)) != cudaSuccess ||
+        (e = cudaHostGetDevicePointer(&c->rag_mapped[i], c->rag_pinned[i], 0)) != cudaSuccess ||
+        (e = cudaEventCreateWithFlags(&c->rag_ev[i], cudaEventDisableTiming)) != cudaSuccess) {
       const int code = (e == cudaErrorMemoryAllocation) ? BKV_ENOMEM : BKV_ECUDA;
       cudaGetLastError();
       free_all(c);
@@ -529,6 +557,151 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
   return BKV_OK;
 }
 
+int bkv_compress_ragged(bkv_ctx* ctx, void* K, void* V, const int32_t* L, int32_t budget, const int64_t* t_pos,
+                        const void* q_recent, const int64_t* recent_pos, int32_t* kept_idx_out, float* scores_out) {
+  if (!ctx) return BKV_EINVAL;
+  const Shape& s = ctx->shape;
+  if (!K || !V || !kept_idx_out || !L) return fail(ctx, BKV_EINVAL, "K, V, L and kept_idx_out must be non-NULL");
+  if (!aligned16(K) || !aligned16(V)) return fail(ctx, BKV_EINVAL, "K and V must be 16-byte aligned");
+  if ((reinterpret_cast<uintptr_t>(kept_idx_out) | reinterpret_cast<uintptr_t>(L)) & 3u)
+    return fail(ctx, BKV_EINVAL, "L and kept_idx_out must be 4-byte aligned");
+  if (scores_out && (reinterpret_cast<uintptr_t>(scores_out) & 3u))
+    return fail(ctx, BKV_EINVAL, "scores_out must be 4-byte aligned");
+  if (budget < 1 || budget < s.n_prefix + s.W)
+    return fail(ctx, BKV_EINVAL, "budget = %d must be >= max(1, n_prefix + window = %d)", budget, s.n_prefix + s.W);
+  if (1LL * s.n_inst * budget >= (1LL << 31)) return fail(ctx, BKV_EINVAL, "budget too large");
+  if (!t_pos) return fail(ctx, BKV_EINVAL, "t_pos (host, one per batch row) is required");
+  if (s.W > 0 && (!q_recent || !aligned16(q_recent) || !recent_pos))
+    return fail(ctx, BKV_EINVAL, "q_recent (16-byte aligned) and recent_pos are required when window > 0");
+  if (s.nb > 0 && !ctx->state_ready) return fail(ctx, BKV_ESTATE, "compress before bkv_init_beacons / bkv_set_state");
+  cudaError_t e;
+  if (budget >= s.cap) {  // no instance can hold more rows than the budget: nothing is evicted anywhere
+    ProfScope ps(ctx, BKV_K_KEEP_ALL);
+    e = bkv::launch_ragged_plan(s, L, budget, ctx->work, ctx->n_work, kept_idx_out, ctx->err, ctx->stream);
+    return e == cudaSuccess ? BKV_OK : cuda_fail(ctx, e, "ragged plan launch");
+  }
+
+  // per batch row: the rotary table (slot w < W at recent_pos[b][w], slot W at t_pos[b]), then the
+  // causal gaps t_pos[b] - recent_pos[b][w], clamped to [0, capacity + 1]
+  const int h = s.d / 2;
+  const double theta = ctx->cfg.rope_theta;
+  const int rotate = theta != 0.0;
+  {
+    const int rs = ctx->rag_next;
+    ctx->rag_next = (rs + 1) % bkv_ctx::kRopeSlots;
+    if (ctx->rag_used[rs] && (e = cudaEventSynchronize(ctx->rag_ev[rs])) != cudaSuccess)
+      return cuda_fail(ctx, e, "ragged staging wait");
+    unsigned char* host = static_cast<unsigned char*>(ctx->rag_pinned[rs]);
+    const size_t n = static_cast<size_t>(s.W + 1) * h;
+    for (int b = 0; b < s.batch; ++b) {
+      double2* tab = reinterpret_cast<double2*>(host) + static_cast<size_t>(b) * ctx->rag_row;
+      float2* tab32 = reinterpret_cast<float2*>(tab + n);
+      for (int slot = 0; rotate && slot <= s.W; ++slot) {
+        const double pos = static_cast<double>(slot < s.W ? recent_pos[static_cast<size_t>(b) * s.W + slot] : t_pos[b]);
+        for (int i = 0; i < h; ++i) {
+          const double inv_freq = std::pow(theta, -static_cast<double>(2 * i) / static_cast<double>(s.d));
+          const double ang = pos * inv_freq;
+          const double c = std::cos(ang), sn = std::sin(ang);
+          tab[static_cast<size_t>(slot) * h + i] = make_double2(c, sn);
+          tab32[static_cast<size_t>(slot) * h + i] = make_float2(static_cast<float>(c), static_cast<float>(sn));
+        }
+      }
+      int32_t* gaps = reinterpret_cast<int32_t*>(host + ctx->rag_gaps_off) + static_cast<size_t>(b) * s.W;
+      for (int w = 0; w < s.W; ++w) {
+        const int64_t rp = recent_pos[static_cast<size_t>(b) * s.W + w];
+        const int64_t g = rp >= t_pos[b] ? 0 : static_cast<int64_t>(static_cast<uint64_t>(t_pos[b]) - static_cast<uint64_t>(rp));
+        gaps[w] = static_cast<int32_t>(g > s.cap + 1LL || g < 0 ? s.cap + 1LL : g);
+      }
+    }
+    {
+      ProfScope ps(ctx, BKV_K_ROPE);
+      e = bkv::launch_rope_stage(ctx->rag_mapped[rs], ctx->rag, ctx->rag_bytes, ctx->stream);
+    }
+    if (e == cudaSuccess) e = cudaEventRecord(ctx->rag_ev[rs], ctx->stream);
+    ctx->rag_used[rs] = true;
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "ragged table upload");
+  }
+  {
+    ProfScope ps(ctx, BKV_K_KEEP_ALL);
+    e = bkv::launch_ragged_plan(s, L, budget, ctx->work, ctx->n_work, kept_idx_out, ctx->err, ctx->stream);
+  }
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "ragged plan launch");
+  bkv::CfpsArgs ca{};
+  if (ctx->cfps) {  // this compress's beacons: FPS of each head's buffer, into cent / counts
+    ca.H = ctx->n_heads;
+    ca.b_min = ctx->b_min;
+    ca.b_max = ctx->b_max;
+    ca.buf = ctx->cbuf;
+    ca.size = ctx->csize;
+    ca.bcn = ctx->cent;
+    ca.bcnt = ctx->counts;
+    ca.mode = bkv::kCfpsBeacons;
+    ProfScope ps(ctx, BKV_K_CFPS);
+    e = bkv::launch_cfps(s.d, ca, ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "continual FPS beacon launch");
+  }
+  const double2* rope_rows = reinterpret_cast<const double2*>(ctx->rag);
+  {
+    ProfScope ps(ctx, BKV_K_QOBS);
+    e = bkv::launch_qobs_ragged(s, static_cast<const __nv_bfloat16*>(q_recent), ctx->cent, ctx->counts, rope_rows,
+                                ctx->rag_row, rotate, ctx->work, ctx->n_work, ctx->qobs, ctx->valid, ctx->stream);
+  }
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "qobs launch");
+
+  CUtensorMap kmap, kmap32;
+  int rc = encode_rows(ctx, &kmap, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 128);
+  if (rc != BKV_OK) return rc;
+  rc = encode_rows(ctx, &kmap32, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 32);
+  if (rc != BKV_OK) return rc;
+  bkv::ScoreArgs sa;
+  sa.L = s.cap;  // the plan is made for the longest possible cache
+  sa.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(s.d)));
+  sa.valid = ctx->valid;
+  sa.mean = (ctx->cfg.flags & BKV_F_MEAN_AGG) != 0;
+  sa.causal = (ctx->cfg.flags & BKV_F_CAUSAL_WINDOW) != 0 && s.W > 0;
+  sa.r_out = ctx->rscore;
+  sa.err = ctx->err;
+  sa.Ls = L;
+  sa.work = ctx->work;
+  sa.n_work = ctx->n_work;
+  sa.gaps = sa.causal ? reinterpret_cast<const int*>(ctx->rag + ctx->rag_gaps_off) : nullptr;
+  for (int col0 = 0; col0 < s.n_obs_pad; col0 += bkv::kScoreMaxCols) {
+    CUtensorMap qmap;
+    sa.col0 = col0;
+    sa.n_cols = std::min(bkv::kScoreMaxCols, s.n_obs_pad - col0);
+    sa.combine = col0 > 0;
+    sa.scores_out = col0 + sa.n_cols == s.n_obs_pad ? scores_out : nullptr;
+    rc = encode_rows(ctx, &qmap, ctx->qobs, static_cast<uint64_t>(s.n_inst) * s.n_obs_pad, s.d,
+                     static_cast<uint32_t>(sa.n_cols));
+    if (rc != BKV_OK) return rc;
+    {
+      ProfScope ps(ctx, BKV_K_SCORE);
+      e = bkv::launch_score(s, kmap, kmap32, qmap, sa, ctx->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "score launch");
+  }
+  {
+    ProfScope ps(ctx, BKV_K_SELECT_GATHER);
+    e = bkv::launch_select_gather_ragged(s, ctx->rscore, L, ctx->work, ctx->n_work, budget,
+                                         static_cast<__nv_bfloat16*>(K), static_cast<__nv_bfloat16*>(V), kept_idx_out,
+                                         ctx->stream);
+  }
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "select_gather launch");
+  if (ctx->cfps) {  // after the eviction, in the instances evicted from: buffer = FPS of (beacons, window)
+    ca.mode = bkv::kCfpsMerge;
+    ca.q = static_cast<const __nv_bfloat16*>(q_recent);
+    ca.n_q = s.W;
+    ca.Ls = L;
+    ca.budget = budget;
+    ca.cap = s.cap;
+    ca.group = s.G;
+    ProfScope ps(ctx, BKV_K_CFPS);
+    e = bkv::launch_cfps(s.d, ca, ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "continual FPS merge launch");
+  }
+  return BKV_OK;
+}
+
 int bkv_get_state(bkv_ctx* ctx, float* centroids, double* sums, int64_t* counts) {
   if (!ctx) return BKV_EINVAL;
   if (ctx->cfps) return fail(ctx, BKV_EINVAL, "a continual FPS context has no centroid state");
@@ -635,6 +808,8 @@ int bkv_sync(bkv_ctx* ctx) {
     return cuda_fail(ctx, e, "error word read");
   if (h != 0) {
     cudaMemset(ctx->err, 0, sizeof(int));
+    if (h == bkv::kDevBadLength)
+      return fail(ctx, BKV_EINVAL, "a per-instance cache length was outside 1..capacity; that instance was left untouched");
     return fail(ctx, BKV_ETIMEOUT, "device wait expired (code %d)", h);
   }
   return BKV_OK;

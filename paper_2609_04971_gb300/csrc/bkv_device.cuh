@@ -19,6 +19,7 @@ enum DevErr : int {
   kDevTimeoutDrain = 4,
   kDevTimeoutCluster = 5,
   kDevTimeoutSelftest = 6,
+  kDevBadLength = 7,  // a per-instance cache length outside 1..capacity (bkv_compress_ragged)
 };
 
 // Every spin-wait gives up after this long and reports a timeout.

@@ -20,6 +20,8 @@ struct Shape {
   int cap;         // rows per instance in K / V
   int n_obs;       // G * W + nb scoring queries
   int n_obs_pad;   // n_obs rounded up to 16
+  int batch;       // batch rows: instance e belongs to batch row (e / n_kv) % batch
+  int n_kv;        // KV heads
 };
 
 constexpr int kMaxBeacons = 32;
@@ -41,6 +43,10 @@ struct CfpsArgs {
   int* size;                // [H] rows in use
   float* bcn;               // [H][b_min][d] beacons of a compress (fp32 copies of bf16 queries)
   long long* bcnt;          // [H][b_min] 1 for a beacon, 0 for an empty slot
+  // merge after a per-instance-length compress: only heads of instances with budget < Ls[h / group]
+  // <= cap were evicted from and merge; the others keep their buffers
+  const int* Ls = nullptr;
+  int budget = 0, cap = 0, group = 1;
 };
 cudaError_t launch_cfps(int d, const CfpsArgs& a, cudaStream_t st);
 // Buffers seeded with b_min fp32 rows per head (FPS picks of the prompt), size b_min.
@@ -71,6 +77,19 @@ cudaError_t launch_update_small(const Shape& s, const __nv_bfloat16* q_new, int 
 cudaError_t launch_rope_stage(const void* src, void* dst, size_t bytes, cudaStream_t st);
 cudaError_t launch_qobs(const Shape& s, const __nv_bfloat16* q_recent, const float* cent, const long long* counts,
                         const double2* rope, int rotate, __nv_bfloat16* qobs, uint32_t* valid, cudaStream_t st);
+// Per-instance cache lengths (bkv_compress_ragged): the same build for the instances work[0 .. *n_work)
+// only, batch row b taking its own rotary table at rope + b * rope_row (double2 units).
+cudaError_t launch_qobs_ragged(const Shape& s, const __nv_bfloat16* q_recent, const float* cent,
+                               const long long* counts, const double2* rope, size_t rope_row, int rotate,
+                               const int* work, const int* n_work, __nv_bfloat16* qobs, uint32_t* valid,
+                               cudaStream_t st);
+
+// ---- per-instance cache lengths (k_ragged.cu)
+// Instances whose length Ls[e] exceeds `budget` are listed in index order in work[0 .. *n_work); every
+// other instance gets kept = 0 .. L - 1 and -1 after (its K and V are not touched).  A length outside
+// 1..cap records kDevBadLength in err and leaves that instance's kept row at -1.
+cudaError_t launch_ragged_plan(const Shape& s, const int* Ls, int budget, int* work, int* n_work, int* kept, int* err,
+                               cudaStream_t st);
 
 struct ScoreArgs {
   int L = 0;
@@ -86,6 +105,13 @@ struct ScoreArgs {
   float* r_out = nullptr;          // [n_inst][cap] log2-domain scores (log2 of the aggregated weight)
   float* scores_out = nullptr;     // [n_inst][cap] probabilities, or nullptr
   int* err = nullptr;              // device error word
+  // per-instance lengths (bkv_compress_ragged): the instances work[0 .. *n_work), instance e with
+  // Ls[e] rows; L above is then the longest possible (it sizes the plan).  Causal form: gaps[b][w] is
+  // t_pos - recent_pos[w] of batch row b, clamped to [0, cap + 1] (0: the slot sees every window row).
+  const int* Ls = nullptr;
+  const int* work = nullptr;
+  const int* n_work = nullptr;
+  const int* gaps = nullptr;
 };
 // Causal mask inside the recent window: recent slot w sits at recent_pos[w] and window row j
 // (L - W <= j < L) at t_pos - (L - 1 - j), so slot w sees window row j only if
@@ -123,6 +149,10 @@ cudaError_t launch_score_causal_mean(const Shape& s, const CUtensorMap& kmap, co
 
 cudaError_t launch_select_gather(const Shape& s, const float* r, int L, int budget, __nv_bfloat16* K,
                                  __nv_bfloat16* V, int* kept, cudaStream_t st);
+// Per-instance lengths: the instances work[0 .. *n_work), instance e with Ls[e] rows (at most cap).
+cudaError_t launch_select_gather_ragged(const Shape& s, const float* r, const int* Ls, const int* work,
+                                        const int* n_work, int budget, __nv_bfloat16* K, __nv_bfloat16* V, int* kept,
+                                        cudaStream_t st);
 
 cudaError_t launch_keep_all(const Shape& s, int L, int budget, int* kept, cudaStream_t st);
 

@@ -159,6 +159,8 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
   s.cap = cfg->capacity;
   s.n_obs = s.G * s.W + s.nb;
   s.n_obs_pad = (s.n_obs + 15) / 16 * 16;
+  s.batch = cfg->batch;
+  s.n_kv = cfg->n_kv_heads;
   if (s.n_obs < 1 || s.n_obs > bkv::kMaxObs) return bad("G * window + n_beacons must be in 1..128");
 
   // ---- call arguments (same rules as bkv_compress)

@@ -280,6 +280,10 @@ __global__ void __launch_bounds__(32 * kHeadsPerCta, R == 16 ? 2 : 1) cfps_kerne
   const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.x * kHeadsPerCta + wid;
   if (h >= a.H) return;  // whole warp
+  if (MODE == kCfpsMerge && a.Ls) {  // per-instance lengths: no eviction in this instance, nothing to merge
+    const int L = a.Ls[h / a.group];
+    if (L <= a.budget || L > a.cap) return;
+  }
   WarpSmem<D, R>& w = reinterpret_cast<WarpSmem<D, R>*>(smem_raw)[wid];
   __nv_bfloat16* buf = a.buf + static_cast<size_t>(h) * a.b_max * D;
   float* bcn = a.bcn + static_cast<size_t>(h) * a.b_min * D;

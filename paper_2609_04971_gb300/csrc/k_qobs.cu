@@ -51,15 +51,24 @@ __device__ __forceinline__ __nv_bfloat16 rot_fast(float xa, float xb, float c32,
   return rot_exact(xa, xb, c.x, c.y, plus);
 }
 
+// work / n_work (per-instance lengths): block w builds instance work[w] when w < *n_work; rope_row: the
+// distance between two batch rows' rotary tables (0: one table for every instance).
 __global__ void __launch_bounds__(kQobsThreads) qobs_kernel(Shape s, const __nv_bfloat16* __restrict__ q_recent,
                                                              const float* __restrict__ cent,
                                                              const long long* __restrict__ counts,
-                                                             const double2* __restrict__ rope, int rotate,
+                                                             const double2* __restrict__ rope_all, size_t rope_row,
+                                                             int rotate, const int* __restrict__ work,
+                                                             const int* __restrict__ n_work,
                                                              __nv_bfloat16* __restrict__ qobs,
                                                              uint32_t* __restrict__ valid) {
-  const int e = blockIdx.x;
+  int e = blockIdx.x;
+  if (work) {
+    if (e >= *n_work) return;  // whole block
+    e = work[e];
+  }
   const int d = s.d, h = d / 2, h4 = h / 4;
   const int GW = s.G * s.W;
+  const double2* rope = rope_all + (rope_row ? static_cast<size_t>((e / s.n_kv) % s.batch) * rope_row : 0);
   const float2* rope32 = reinterpret_cast<const float2*>(rope + static_cast<size_t>(s.W + 1) * h);
   __nv_bfloat16* out = qobs + static_cast<size_t>(e) * s.n_obs_pad * d;
   for (int idx = threadIdx.x; idx < s.n_obs_pad * h4; idx += blockDim.x) {
@@ -133,7 +142,17 @@ cudaError_t launch_rope_stage(const void* src, void* dst, size_t bytes, cudaStre
 
 cudaError_t launch_qobs(const Shape& s, const __nv_bfloat16* q_recent, const float* cent, const long long* counts,
                         const double2* rope, int rotate, __nv_bfloat16* qobs, uint32_t* valid, cudaStream_t st) {
-  qobs_kernel<<<s.n_inst, kQobsThreads, 0, st>>>(s, q_recent, cent, counts, rope, rotate, qobs, valid);
+  qobs_kernel<<<s.n_inst, kQobsThreads, 0, st>>>(s, q_recent, cent, counts, rope, 0, rotate, nullptr, nullptr, qobs,
+                                                 valid);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_qobs_ragged(const Shape& s, const __nv_bfloat16* q_recent, const float* cent,
+                               const long long* counts, const double2* rope, size_t rope_row, int rotate,
+                               const int* work, const int* n_work, __nv_bfloat16* qobs, uint32_t* valid,
+                               cudaStream_t st) {
+  qobs_kernel<<<s.n_inst, kQobsThreads, 0, st>>>(s, q_recent, cent, counts, rope, rope_row, rotate, work, n_work,
+                                                 qobs, valid);
   return cudaGetLastError();
 }
 

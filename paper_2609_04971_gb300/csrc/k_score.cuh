@@ -113,6 +113,29 @@ struct Plan {
   int csize, slots, stream;
 };
 
+// This CTA's share of one instance of L keys: keys [k0, k1), T tiles, the first R of them resident
+// in the ring and n_str streaming.  The producer, the MMA issuer and the epilogue all derive it from
+// the same L, so they agree on every instance's job list.
+struct Geom {
+  int k0, k1, T, R, n_str;
+};
+
+__device__ __forceinline__ Geom inst_geom(int L, int crank, int csize, int slots) {
+  Geom g;
+  const int U = (L + 31) / 32;  // 32-key units of the cache
+  g.k0 = (crank * U / csize) * 32;
+  g.k1 = min(L, ((crank + 1) * U / csize) * 32);
+  g.T = (g.k1 - g.k0 + kTile - 1) / kTile;
+  g.R = g.T < slots ? g.T : slots;
+  g.n_str = g.T - g.R;
+  return g;
+}
+
+// Instance of work item w and its number of keys: the compact list of a per-instance-length
+// compress, or every instance with the launch's L.
+__device__ __forceinline__ int item_inst(const ScoreArgs& a, int w) { return a.work ? a.work[w] : w; }
+__device__ __forceinline__ int inst_len(const ScoreArgs& a, int e) { return a.Ls ? a.Ls[e] : a.L; }
+
 // Wait used while draining after an abort: ignores the abort flag.
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* err) {
   int never = 0;
@@ -323,7 +346,7 @@ __global__ void __launch_bounds__(kScThreads, 1)
   __shared__ int abort_sh;
   __shared__ __align__(16) float lse2_sh[128];
   __shared__ int vcount_sh[4];  // valid queries per 32-column group of the instance (mean aggregation)
-  __shared__ int thr_sh[CAUSAL ? 128 : 1];  // causal form: last visible window row of each column
+  __shared__ int thr_sh[CAUSAL ? 2 : 1][CAUSAL ? 128 : 1];  // causal form: last visible window row per column
   __shared__ float wred_m[kEpiWarps][64], wred_s[kEpiWarps][64];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -331,13 +354,8 @@ __global__ void __launch_bounds__(kScThreads, 1)
   const int crank = csize > 1 ? static_cast<int>(cluster_ctarank()) : 0;
   const int cluster_id = blockIdx.x / csize;
   const int n_clusters = gridDim.x / csize;
-  const int n_my = cluster_id < s.n_inst ? (s.n_inst - cluster_id + n_clusters - 1) / n_clusters : 0;
-  const int U = (a.L + 31) / 32;                     // 32-key units of the cache
-  const int k0 = (crank * U / csize) * 32;           // this CTA's keys: [k0, k1)
-  const int k1 = min(a.L, ((crank + 1) * U / csize) * 32);
-  const int T = (k1 - k0 + kTile - 1) / kTile;       // tiles this CTA owns in every instance
-  const int R = T < plan.slots ? T : plan.slots;     // resident tiles
-  const int n_str = T - R;                           // streaming tiles (plan.stream only)
+  const int n_items = a.work ? *a.n_work : s.n_inst;  // instances to compress
+  const int n_my = cluster_id < n_items ? (n_items - cluster_id + n_clusters - 1) / n_clusters : 0;
   const int ring = plan.slots;                       // resident slots, used in cyclic order
   const int str_slot = ring;                         // pass-1 streaming slots; +2, +3: pass-2 slots
   const uint32_t qbox = static_cast<uint32_t>(a.n_cols) * 128;  // one 64-column box of this launch's queries (N rows)
@@ -370,9 +388,9 @@ __global__ void __launch_bounds__(kScThreads, 1)
     fence_mbar_init();
   }
   if constexpr (CAUSAL) {
-    if (threadIdx.x < 128) {
+    if (threadIdx.x < 128 && !a.gaps) {  // one call-wide table; with per-instance lengths see the epilogue
       const int c = col0 + threadIdx.x;  // Q_obs row: recent slot c % W of head c / W, or a beacon / padding
-      thr_sh[threadIdx.x] = c < s.G * s.W ? a.thr[c % s.W] : 0x7fffffff;
+      thr_sh[0][threadIdx.x] = c < s.G * s.W ? a.thr[c % s.W] : 0x7fffffff;
     }
   }
   if (warp == 1) {
@@ -399,7 +417,9 @@ __global__ void __launch_bounds__(kScThreads, 1)
       bool ok = true;
       int q_issued = 0;
       for (int i = 0; ok && i < n_my; ++i) {
-        const int e = cluster_id + i * n_clusters;
+        const int e = item_inst(a, cluster_id + i * n_clusters);
+        const Geom gm = inst_geom(inst_len(a, e), crank, csize, ring);
+        const int k0 = gm.k0, k1 = gm.k1, T = gm.T, R = gm.R, n_str = gm.n_str;
         const int qb = i & 1;
         if (i >= 2 && !mbar_wait(&qempty_bar[qb], ((i >> 1) - 1) & 1, abort_flag, a.err, kDevTimeoutProducer)) {
           ok = false;
@@ -451,6 +471,9 @@ __global__ void __launch_bounds__(kScThreads, 1)
       int rs = 0, ru = 0;                        // next ring slot and its use count
       bool ok = true;
       for (int i = 0; ok && i < n_my; ++i) {
+        const int e = item_inst(a, cluster_id + i * n_clusters);
+        const Geom gm = inst_geom(inst_len(a, e), crank, csize, ring);
+        const int T = gm.T, R = gm.R, n_str = gm.n_str;
         if (!mbar_wait(&qfull_bar[i & 1], (i >> 1) & 1, abort_flag, a.err, kDevTimeoutMma)) break;
         for (int j = 0; j < T + n_str; ++j) {
           const int st = g % n_stages;
@@ -517,14 +540,36 @@ __global__ void __launch_bounds__(kScThreads, 1)
     // its column (Q_obs row col0 + te); the four words that threads 0, 32, 64
     // and 96 read are all of the instance's words in some order (their total
     // is the valid count of the mean form).
-    uint32_t vnext = (te < 128 && n_my > 0)
-                         ? ld_nc_u32(&a.valid[cluster_id * 4 + (COMBINE ? ((col0 >> 5) + (te >> 5)) & 3 : te >> 5)])
-                         : 0u;
+    const int vw = COMBINE ? ((col0 >> 5) + (te >> 5)) & 3 : te >> 5;  // this thread's valid word
+    int e_next = n_my > 0 ? item_inst(a, cluster_id) : 0;
+    uint32_t vnext = (te < 128 && n_my > 0) ? ld_nc_u32(&a.valid[e_next * 4 + vw]) : 0u;
     for (int i = 0; i < n_my; ++i) {
-      const int e = cluster_id + i * n_clusters;
+      const int e = e_next;
       const uint32_t vword = vnext;
-      if (te < 128 && i + 1 < n_my)
-        vnext = ld_nc_u32(&a.valid[(e + n_clusters) * 4 + (COMBINE ? ((col0 >> 5) + (te >> 5)) & 3 : te >> 5)]);
+      if (i + 1 < n_my) {
+        e_next = item_inst(a, cluster_id + (i + 1) * n_clusters);
+        if (te < 128) vnext = ld_nc_u32(&a.valid[e_next * 4 + vw]);
+      }
+      const int L_e = inst_len(a, e);
+      const Geom gm = inst_geom(L_e, crank, csize, ring);
+      const int k0 = gm.k0, k1 = gm.k1, T = gm.T, R = gm.R;
+      const int win0 = a.gaps ? L_e - s.W : a.win0;  // first window row
+      const int* thr = thr_sh[0];
+      if constexpr (CAUSAL) {
+        if (a.gaps) {  // per-instance lengths: this instance's table, in the buffer of its parity
+          thr = thr_sh[i & 1];
+          if (te < 128) {
+            const int c = col0 + te;
+            int t = 0x7fffffff;
+            if (c < s.G * s.W) {
+              const int g = a.gaps[((e / s.n_kv) % s.batch) * s.W + c % s.W];
+              t = g == 0 ? L_e : (g > L_e ? -1 : L_e - 1 - g);
+            }
+            thr_sh[i & 1][te] = t;
+          }
+          named_barrier(1, 32 * kEpiWarps);  // the table is written before pass 1 reads it
+        }
+      }
       float m[NQ], sm[NQ];
 #pragma unroll
       for (int c = 0; c < NQ; ++c) {
@@ -574,14 +619,14 @@ __global__ void __launch_bounds__(kScThreads, 1)
         // logit exceeds it by more than 64, so the terms stay below 2^64 and
         // the common step is one FFMA, one ex2 and one add per column.
         const int tile0 = k0 + j * kTile;
-        if (have && CAUSAL && tile0 + kTile > a.win0) {
+        if (have && CAUSAL && tile0 + kTile > win0) {
           // a tile with window rows: the careful path, without the masked (row, column) terms
           const int key = tile0 + key_row;
           if (key < k1) {
-            const bool in_win = key >= a.win0;
+            const bool in_win = key >= win0;
 #pragma unroll
             for (int c = 0; c < NQ; ++c) {
-              if (in_win && key > thr_sh[half * NQ + c]) continue;
+              if (in_win && key > thr[half * NQ + c]) continue;
               const float t = fmaf(v[c], sc, -m[c]);
               if (t > 64.f) {
                 const float y = v[c] * sc;
@@ -675,8 +720,8 @@ __global__ void __launch_bounds__(kScThreads, 1)
         float r = -INFINITY;
         const int key = k0 + j * kTile + key_row;
         if (resident_ok)
-          r = (CAUSAL && k0 + j * kTile + kTile > a.win0)
-                  ? tile_agg_causal<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m, key, a.win0, thr_sh)
+          r = (CAUSAL && k0 + j * kTile + kTile > win0)
+                  ? tile_agg_causal<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m, key, win0, thr)
                   : tile_agg<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m);
         tc_fence_before();
         __syncwarp();
@@ -696,8 +741,8 @@ __global__ void __launch_bounds__(kScThreads, 1)
         const int key = k0 + j * kTile + key_row;
         if (have) {
           tc_fence_after();
-          r = (CAUSAL && k0 + j * kTile + kTile > a.win0)
-                  ? tile_agg_causal<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m, key, a.win0, thr_sh)
+          r = (CAUSAL && k0 + j * kTile + kTile > win0)
+                  ? tile_agg_causal<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m, key, win0, thr)
                   : tile_agg<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m);
         }
         tc_fence_before();
@@ -726,39 +771,89 @@ __global__ void __launch_bounds__(kScThreads, 1)
   if (csize > 1) cluster_sync_all();  // no CTA leaves while a peer may still access its shared memory
 }
 
-// Cluster size and tensor-memory placement: the fewest CTAs per instance
-// whose tiles all fit the slot ring, with at least kSlack spare slots where
-// eight CTAs allow it; when not even eight CTAs hold an instance, eight CTAs
-// with streaming slots.  Slot barriers exist for kMaxSlots slots, and tensor
-// memory holds kTmemCols / n_cols of them (at least 8: a launch has n_cols <= 64).
-constexpr int kSlack = 1;
+// Cluster size and tensor-memory placement.  sms[c] (c = 1..kMaxCluster) is how many SMs clusters
+// of c CTAs keep busy at once (0: not available).  Among the sizes whose tiles all fit the slot ring,
+// the one keeping the most SMs busy wins (ties: more spare slots, then fewer CTAs); one spare slot
+// lets the next instance's first tile land while an instance finishes.  When no size fits, the size
+// keeping the most SMs busy streams its extra tiles through four slots after the ring.  Slot
+// barriers exist for kMaxSlots slots, and tensor memory holds kTmemCols / n_cols of them (at least 8:
+// a launch has n_cols <= 64).
+constexpr int kMaxCluster = 16;  // 9 and more need the non-portable cluster-size attribute
+constexpr int kMaxDevicesScore = 64;
 
-Plan plan_score(int L, int n_cols) {
+Plan plan_score(int L, int n_cols, const int* sms) {
   const int U = (L + 31) / 32;
   int cap = static_cast<int>(kTmemCols) / n_cols;
   if (cap > kMaxSlots) cap = kMaxSlots;
-  const int cmax = U < 8 ? U : 8;  // every CTA owns at least one 32-key unit
-  for (int slack = kSlack; slack >= 0; --slack)
-    for (int c = 1; c <= cmax; ++c) {
-      const int tiles = ((U + c - 1) / c + 3) / 4;  // tiles of the CTA with the most units
-      if (tiles + slack <= cap) return Plan{c, cap, 0};
+  const int cmax = U < kMaxCluster ? U : kMaxCluster;  // every CTA owns at least one 32-key unit
+  int best = 0, best_sms = 0, best_slack = -1;
+  for (int c = 1; c <= cmax; ++c) {
+    const int tiles = ((U + c - 1) / c + 3) / 4;  // tiles of the CTA with the most units
+    const int slack = cap - tiles;
+    if (slack < 0 || sms[c] <= 0) continue;
+    const int sl = slack > 0 ? 1 : 0;
+    if (sms[c] > best_sms || (sms[c] == best_sms && sl > best_slack)) {
+      best = c;
+      best_sms = sms[c];
+      best_slack = sl;
     }
-  return Plan{cmax, cap - 4, 1};
+  }
+  if (best > 0) return Plan{best, cap, 0};
+  int sc = 1;
+  for (int c = 2; c <= cmax; ++c)
+    if (sms[c] > sms[sc]) sc = c;
+  return Plan{sc, cap - 4, 1};
 }
 
 template <int D, int NQ, bool MEAN, bool CAUSAL, bool COMBINE>
 cudaError_t launch_score_dq(const Shape& s, const CUtensorMap& kmap, const CUtensorMap& kmap32,
                             const CUtensorMap& qmap, const ScoreArgs& a, cudaStream_t st) {
   using C = ScoreCfg<D>;
-  const Plan plan = plan_score(a.L, 2 * NQ);
-  const size_t smem = C::smem_bytes(2 * NQ, plan.csize);
-  const int n_stages = C::stages(2 * NQ, plan.csize);
-  cudaError_t err = cudaFuncSetAttribute(score_kernel<D, NQ, MEAN, CAUSAL, COMBINE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-  if (err != cudaSuccess) return err;
+  auto kern = score_kernel<D, NQ, MEAN, CAUSAL, COMBINE>;
   int dev = 0, sms = 0, max_clusters = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  // SMs that clusters of each size keep busy, queried once per device for this kernel (the shared
+  // memory of a cluster's CTAs grows with its size by a few bytes only, so the largest is used)
+  static int busy[kMaxDevicesScore][kMaxCluster + 1] = {};
+  cudaError_t err = cudaSuccess;
+  if (dev < kMaxDevicesScore && busy[dev][0] == 0) {
+    const size_t smem_q = C::smem_bytes(2 * NQ, kMaxCluster);
+    if ((err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem_q))) !=
+            cudaSuccess ||
+        (err = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) != cudaSuccess)
+      return err;
+    for (int c = 1; c <= kMaxCluster; ++c) {
+      cudaLaunchConfig_t q = {};
+      q.blockDim = dim3(kScThreads);
+      q.dynamicSmemBytes = smem_q;
+      q.gridDim = dim3(static_cast<unsigned>(c * sms));
+      cudaLaunchAttribute qa[1];
+      qa[0].id = cudaLaunchAttributeClusterDimension;
+      qa[0].val.clusterDim.x = static_cast<unsigned>(c);
+      qa[0].val.clusterDim.y = 1;
+      qa[0].val.clusterDim.z = 1;
+      q.attrs = qa;
+      q.numAttrs = 1;
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, kern, &q) != cudaSuccess) {
+        cudaGetLastError();
+        n = c <= 8 ? sms / c : 0;
+      }
+      busy[dev][c] = n * c;
+    }
+    busy[dev][0] = 1;
+  }
+  int fallback[kMaxCluster + 1] = {};
+  for (int c = 1; c <= 8; ++c) fallback[c] = (sms / c) * c;
+  const Plan plan = plan_score(a.L, 2 * NQ, dev < kMaxDevicesScore ? busy[dev] : fallback);
+  const size_t smem = C::smem_bytes(2 * NQ, plan.csize);
+  const int n_stages = C::stages(2 * NQ, plan.csize);
+  err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (err != cudaSuccess) return err;
+  if (plan.csize > 8 && (err = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) !=
+                            cudaSuccess)
+    return err;
   cudaLaunchConfig_t cfg = {};
   cfg.blockDim = dim3(kScThreads);
   cfg.dynamicSmemBytes = smem;

@@ -45,10 +45,14 @@ __device__ __forceinline__ void block_count_scan(bool flag, int* wsum, int& excl
   __syncthreads();
 }
 
+// work / n_work (per-instance lengths): block w compresses instance work[w], with Ls[work[w]] rows,
+// when w < *n_work; otherwise every block compresses its own instance from L rows.
 template <int D>
 __global__ void __launch_bounds__(kSgThreads) select_gather_kernel(Shape s, const float* __restrict__ r, int L,
                                                                     int budget, __nv_bfloat16* K, __nv_bfloat16* V,
-                                                                    int* kept) {
+                                                                    int* kept, const int* __restrict__ Ls,
+                                                                    const int* __restrict__ work,
+                                                                    const int* __restrict__ n_work) {
   extern __shared__ __align__(16) uint32_t keys[];  // [L]
   __shared__ uint32_t hist[kSgWarps][256];
   __shared__ uint32_t tot[256];
@@ -56,7 +60,13 @@ __global__ void __launch_bounds__(kSgThreads) select_gather_kernel(Shape s, cons
   __shared__ uint32_t sh_prefix, sh_k;
   __shared__ int sh_first_evicted;
 
-  const int e = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  int e = blockIdx.x;
+  if (work) {
+    if (e >= *n_work) return;  // whole block
+    e = work[e];
+    L = Ls[e];
+  }
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int c_lo = s.n_prefix, c_hi = L - s.W;
   const int k_sel = budget - s.n_prefix - s.W;
   const float* r_e = r + static_cast<size_t>(e) * s.cap;
@@ -205,7 +215,19 @@ cudaError_t launch_sg_d(const Shape& s, const float* r, int L, int budget, __nv_
   cudaError_t err = cudaFuncSetAttribute(select_gather_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
   if (err != cudaSuccess) return err;
-  select_gather_kernel<D><<<s.n_inst, kSgThreads, smem, st>>>(s, r, L, budget, K, V, kept);
+  select_gather_kernel<D><<<s.n_inst, kSgThreads, smem, st>>>(s, r, L, budget, K, V, kept, nullptr, nullptr, nullptr);
+  return cudaGetLastError();
+}
+
+// L_max sizes the shared-memory key array (every instance has at most that many rows).
+template <int D>
+cudaError_t launch_sg_ragged_d(const Shape& s, const float* r, const int* Ls, const int* work, const int* n_work,
+                               int L_max, int budget, __nv_bfloat16* K, __nv_bfloat16* V, int* kept, cudaStream_t st) {
+  const size_t smem = sizeof(uint32_t) * static_cast<size_t>(L_max);
+  cudaError_t err = cudaFuncSetAttribute(select_gather_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+  if (err != cudaSuccess) return err;
+  select_gather_kernel<D><<<s.n_inst, kSgThreads, smem, st>>>(s, r, L_max, budget, K, V, kept, Ls, work, n_work);
   return cudaGetLastError();
 }
 
@@ -215,6 +237,13 @@ cudaError_t launch_select_gather(const Shape& s, const float* r, int L, int budg
                                  __nv_bfloat16* V, int* kept, cudaStream_t st) {
   return s.d == 128 ? launch_sg_d<128>(s, r, L, budget, K, V, kept, st)
                     : launch_sg_d<64>(s, r, L, budget, K, V, kept, st);
+}
+
+cudaError_t launch_select_gather_ragged(const Shape& s, const float* r, const int* Ls, const int* work,
+                                        const int* n_work, int budget, __nv_bfloat16* K, __nv_bfloat16* V, int* kept,
+                                        cudaStream_t st) {
+  return s.d == 128 ? launch_sg_ragged_d<128>(s, r, Ls, work, n_work, s.cap, budget, K, V, kept, st)
+                    : launch_sg_ragged_d<64>(s, r, Ls, work, n_work, s.cap, budget, K, V, kept, st);
 }
 
 cudaError_t launch_keep_all(const Shape& s, int L, int budget, int* kept, cudaStream_t st) {
