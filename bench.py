@@ -31,6 +31,7 @@ plain fp64 restatement of the method) on the host cores instead.
 from __future__ import annotations
 
 import argparse
+import ctypes
 import hashlib
 import json
 import os
@@ -435,8 +436,6 @@ def step_bench(args, wl, job, cfps: bool, steps: int, warmup: int, with_e2e: boo
         prepare(i)
         step(i)
     bk.sync()
-    bkv.bkv_profile_read(bk.ctx)
-    bkv.bkv_profile_enable(bk.ctx, True)
 
     sampler = ClockSampler(job.gpu_index)
     sampler.start()
@@ -452,6 +451,14 @@ def step_bench(args, wl, job, cfps: bool, steps: int, warmup: int, with_e2e: boo
     job.barrier()
     clocks = sampler.stop()
     bk.sync()
+    # per-kernel times: the library brackets each launch with events (which take device time of
+    # their own), so they come from further steps after the timed ones, not from the timed steps
+    prof_steps = min(steps, 20)
+    bkv.bkv_profile_read(bk.ctx)
+    bkv.bkv_profile_enable(bk.ctx, True)
+    for i in range(prof_steps):
+        prepare(warmup + steps + i)
+        step(warmup + steps + i)
     prof = bkv.bkv_profile_read(bk.ctx)
     bkv.bkv_profile_enable(bk.ctx, False)
     step_ms = [a.elapsed_time(b) for a, b in ev]
@@ -471,11 +478,11 @@ def step_bench(args, wl, job, cfps: bool, steps: int, warmup: int, with_e2e: boo
     if cfps:  # three launches per step: buffer update, beacon selection, merge; accounted per step
         ms, n = prof.get("cfps", (0.0, 0))
         b = cfps_bytes(wl)
-        per = ms / steps
+        per = ms / prof_steps
         kernels["cfps"] = {"ms_per_step": per, "launches": n, "alg_bytes_per_step": b,
                            "achieved_gbs": b / (per * 1e-3) / 1e9, "frac_of_hbm": b / (per * 1e-3) / 1e9 / hbm_gbs,
                            "note": "per step: update (n_new queries per head) + beacon FPS + post-eviction merge"}
-    kernels.update(kernel_table(prof, alg_bytes, steps, hbm_gbs))
+    kernels.update(kernel_table(prof, alg_bytes, prof_steps, hbm_gbs))
     ms, n = prof.get("rope_stage", (0.0, 0))
     if n:  # the rotary table of a compress, 24 (W + 1) d / 2 bytes copied from pinned host memory
         kernels["rope_stage"] = {"ms_per_launch": ms / n, "launches": n}
@@ -493,7 +500,7 @@ def step_bench(args, wl, job, cfps: bool, steps: int, warmup: int, with_e2e: boo
         step_bytes = wl.compress_bytes() + cfps_bytes(wl)
         step_flops = wl.compress_flops()
         step_roof_s = max(step_bytes / (hbm_gbs * 1e9), step_flops / (bf16_tflops * 1e12))
-    launches = sum(n for _, n in prof.values())
+    launches = sum(n for _, n in prof.values()) * steps // prof_steps  # the same launches in every step
 
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps,
@@ -503,7 +510,8 @@ def step_bench(args, wl, job, cfps: bool, steps: int, warmup: int, with_e2e: boo
         "roofline": roofline,
         "step_roofline": {"alg_bytes": step_bytes, "alg_flops": step_flops,
                           "roofline_ms": step_roof_s * 1e3, "frac": step_roof_s * 1e3 / ms_per_step},
-        "kernels": kernels, "gpu_launches": launches, "clocks": clocks,
+        "kernels": kernels, "kernels_note": f"per-launch times from {prof_steps} profiled steps after the timed ones",
+        "gpu_launches": launches, "clocks": clocks,
         "step_ms_p10_p50_p90": [float(x) for x in
                                 (sorted(step_ms)[len(step_ms) // 10], statistics.median(step_ms),
                                  sorted(step_ms)[(9 * len(step_ms)) // 10])],
@@ -557,9 +565,10 @@ def trace_bench(args, wl, job, cfps: bool, steps: int) -> dict:
     the buffers while L <= B_max - n_recent, the beacons are then fixed (the library selects them from
     the unchanged buffer at the eviction), and the last n_recent queries are kept with their positions
     for the eviction and the merge that follows it.  The timed quantity is the compression overhead of
-    the whole trace: the device time of every bkv_update_beacons and bkv_compress call, each bracketed
-    by CUDA events on the library's stream.  The model's own work between them (appending the K / V
-    row, building the recent-query block) runs outside the events.  Queries and K / V rows cycle through
+    the whole trace: the device time of every bkv_update_beacons and bkv_compress call, measured with
+    CUDA events on the library's stream (one pair around each compress, one around the back-to-back
+    updates of each period between compresses).  The model's own work (appending the K / V rows,
+    building the recent-query block) runs outside the events.  Queries and K / V rows cycle through
     TRACE_POOL pre-generated decode steps (drifting clusters within the pool), so that host-side input
     generation does not pace the trace."""
     import collections
@@ -612,15 +621,26 @@ def trace_bench(args, wl, job, cfps: bool, steps: int) -> dict:
     bk.init_beacons(q_init)
     bk.sync()
     bkv.bkv_profile_read(bk.ctx)
-    bkv.bkv_profile_enable(bk.ctx, True)
 
-    drain = 256  # events are read back (host-side, outside the timed brackets) every `drain` steps
-    ev_u = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(drain)]
-    ev_c = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-            for _ in range(len(sched))]
-    upd_ms, n_upd = 0.0, 0
+    # The trace runs in periods that end at each compress (and at the last step).  A period's K / V
+    # rows are appended with one copy per tensor and its recent-query history is kept on the host;
+    # neither depends on the beacon updates, so the period's updates are then enqueued back to back
+    # (the C ABI called directly, no per-call Python checks) between one pair of events: the events
+    # measure the device time of the updates, not the host's pace.  The compress that ends a period
+    # follows its updates on the stream, as in a decode loop.
+    lib = bkv._l()
+    qptr = [ctypes.c_void_p(q_pool[j].data_ptr()) for j in range(pool)]
+
+    def update_call(j):
+        rc = lib.bkv_update_beacons(bk.ctx, qptr[j], 1, None)
+        if rc != bkv.BKV_OK:
+            raise bkv.BkvError(rc, "bkv_update_beacons", bkv.bkv_last_error(bk.ctx))
+
+    ends = sorted(set(sched) | ({steps - 1} if steps else set()))
+    ev_u, ev_c = [], []
+    n_upd = 0
     hist = collections.deque(maxlen=W)   # (query [nl, B, Hq, d], absolute position) of the latest steps
-    L, pos, c = wl.prefill, wl.prefill, 0
+    L, pos, s0 = wl.prefill, wl.prefill, 0
     compress_at = set(sched)
     prof = {name: (0.0, 0) for name in bkv.KERNEL_NAMES}
 
@@ -629,37 +649,41 @@ def trace_bench(args, wl, job, cfps: bool, steps: int) -> dict:
     job.barrier()
     torch.cuda.synchronize()
     wall0 = time.perf_counter()
-    pending = 0  # update events recorded since the last drain
-    for s in range(steps):
-        j = s % pool
-        if not cfps or phases[s] == "obs":
-            e0, e1 = ev_u[pending]
-            e0.record()
-            bk.update(q_pool[j])
-            e1.record()
-            pending += 1
-        K[:, :, :, L].copy_(k_pool[j])
-        V[:, :, :, L].copy_(v_pool[j])
-        hist.append((q_pool[j, :, :, :, 0], pos))
-        L += 1
-        pos += 1
-        if s in compress_at:
+    for period, s_end in enumerate(ends):
+        idx = [s % pool for s in range(s0, s_end + 1)]
+        n = len(idx)
+        K[:, :, :, L:L + n].copy_(k_pool[idx].permute(1, 2, 3, 0, 4))
+        V[:, :, :, L:L + n].copy_(v_pool[idx].permute(1, 2, 3, 0, 4))
+        for s in range(s0, s_end + 1):
+            hist.append((q_pool[s % pool, :, :, :, 0], pos))
+            pos += 1
+        L += n
+        upd = [s % pool for s in range(s0, s_end + 1) if not cfps or phases[s] == "obs"]
+        if upd:
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            for j in upd:
+                update_call(j)
+            b.record()
+            ev_u.append((a, b))
+            n_upd += len(upd)
+        if s_end in compress_at:
             q_recent = torch.stack([h[0] for h in hist], dim=3)
-            a, b = ev_c[c]
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            # the library's per-launch events only around the compress kernels (milliseconds each);
+            # the updates run without them, timed as a period by ev_u
+            bkv.bkv_profile_enable(bk.ctx, True)
             a.record()
             bk.compress(K, V, L=L, budget=budget, t_pos=pos - 1, q_recent=q_recent,
                         recent_pos=[h[1] for h in hist], kept_out=kept)
             b.record()
-            c += 1
+            bkv.bkv_profile_enable(bk.ctx, False)
+            ev_c.append((a, b))
             L = budget
-        if pending == drain or s == steps - 1:
-            if pending:
-                ev_u[pending - 1][1].synchronize()
-                upd_ms += sum(x.elapsed_time(y) for x, y in ev_u[:pending])
-                n_upd += pending
-                pending = 0
-            for name, (ms, n) in bkv.bkv_profile_read(bk.ctx).items():  # recycles the library's events
-                prof[name] = (prof[name][0] + ms, prof[name][1] + n)
+        s0 = s_end + 1
+        if period % 16 == 15 or s_end == steps - 1:  # fold the library's launch timings (recycles its events)
+            for name, (ms, cnt) in bkv.bkv_profile_read(bk.ctx).items():
+                prof[name] = (prof[name][0] + ms, prof[name][1] + cnt)
     torch.cuda.synchronize()
     wall_s = time.perf_counter() - wall0
     job.barrier()
@@ -667,6 +691,10 @@ def trace_bench(args, wl, job, cfps: bool, steps: int) -> dict:
     bk.sync()
     bkv.bkv_profile_enable(bk.ctx, False)
     bk.close()
+    upd_ms = sum(x.elapsed_time(y) for x, y in ev_u)
+    if n_upd:  # the updates' device time, from the period events (no per-launch events around them)
+        name = "cfps" if cfps else "update"
+        prof[name] = (prof[name][0] + upd_ms, prof[name][1] + n_upd)
     cmp_ms = [x.elapsed_time(y) for x, y in ev_c]
     total_ms = max_over_ranks(upd_ms + sum(cmp_ms), world, dev)
 
