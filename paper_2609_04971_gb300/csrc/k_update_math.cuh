@@ -74,6 +74,27 @@ __device__ __forceinline__ long long fixed40(const Parts& p) {
   return h + m + l;
 }
 
+// Float <-> int conversions run on a slow unit of this part, so the small cases below use the
+// magic-number route instead: for an integer-valued float x with |x| <= 2^22, x + 1.5 * 2^23 holds the
+// integer in its low mantissa bits (the sum stays in [2^23, 2^24], where every integer is exact),
+// and for an integer |i| <= 2^22 the reverse subtraction gives float(i) exactly.
+__device__ __forceinline__ int magic_f2i(float x) {  // x integer-valued, |x| <= 2^22
+  return __float_as_int(__fadd_rn(x, 12582912.f)) - 0x4B400000;
+}
+__device__ __forceinline__ float magic_i2f(int i) {  // |i| <= 2^22, exact
+  return __fadd_rn(__int_as_float(0x4B400000 + i), -12582912.f);
+}
+
+// fixed40 for part sums of at most 32 values (a few queries per beacon, the decode-step kernel): each
+// scaled part is an integer of magnitude at most 2^22 (|x| < 2^14 for the high part, 2^-4 for the
+// middle one, 2^-21 for the low one), so the magic-number conversions are exact and equal fixed40's.
+__device__ __forceinline__ long long fixed40_few(const Parts& p) {
+  const long long h = static_cast<long long>(magic_f2i(p.h * 8.0f)) << 37;
+  const long long m = static_cast<long long>(magic_f2i(p.m * 1048576.0f)) << 20;
+  const long long l = static_cast<long long>(magic_f2i(p.l * 274877906944.0f)) << 2;
+  return h + m + l;
+}
+
 // Splits the bf16 value x (exact in fp32) into the three parts and adds them.
 __device__ __forceinline__ void parts_add(Parts& p, float x) {
   const float xh = __fadd_rn(__fadd_rn(x, 1572864.f), -1572864.f);  // multiple of 2^-3 (1.5 * 2^20 magic)
@@ -175,12 +196,11 @@ __device__ __forceinline__ double fold_sum_fp64(double s, long long acc) {
 // 1 / n for a count n >= 1 as a double-float: the correctly rounded fp32 reciprocal of n
 // refined by one Newton-Raphson step r' = r + r (1 - n r), the residual formed exactly.
 __device__ __forceinline__ DF count_reciprocal(long long n) {
-  // 64-bit integer <-> float conversions run on the slow fp64 unit of this part: counts below 2^31
-  // (all practical ones) take the 32-bit forms, which give the same values
-  const bool small = n < (1LL << 31);
-  const float nf = small ? __int2float_rn(static_cast<int>(n)) : static_cast<float>(n);  // exact below 2^24
-  const long long nfi = small ? static_cast<long long>(__float2int_rn(nf)) : static_cast<long long>(nf);
-  const float nl = small ? __int2float_rn(static_cast<int>(n - nfi)) : static_cast<float>(n - nfi);
+  // conversions run on a slow unit of this part: counts up to 2^22 (all practical ones) are exact floats
+  // by the magic-number route (nl = 0), larger ones take the conversion instructions, with equal values
+  const bool small = n <= (1LL << 22);
+  const float nf = small ? magic_i2f(static_cast<int>(n)) : static_cast<float>(n);  // exact below 2^24
+  const float nl = small ? 0.f : static_cast<float>(n - static_cast<long long>(nf));
   const float r = __frcp_rn(nf);
   const float p = __fmul_rn(nf, r);
   const float pe = __fmaf_rn(nl, r, __fmaf_rn(nf, r, -p));     // n r - p
@@ -206,9 +226,14 @@ __device__ __forceinline__ float centroid_value(double s, DF rcp) {
   const unsigned long long m = (bits & ((1ull << 52) - 1)) | (1ull << 52);  // 53-bit significand
   const unsigned long long m_hi = (m + (1ull << 28) - 1 + ((m >> 29) & 1)) >> 29;  // m / 2^29, nearest even
   const long long rem = static_cast<long long>(m) - static_cast<long long>(m_hi << 29);  // |rem| <= 2^28
-  // 32-bit conversions (m_hi <= 2^24 and |rem| <= 2^28 fit; 64-bit ones run on the slow fp64 unit)
-  float hi = __fmul_rn(__uint2float_rn(static_cast<uint32_t>(m_hi)), pow2f(e - 1046));  // exact: m_hi <= 2^24
-  float lo = __fmul_rn(__int2float_rn(static_cast<int>(rem)), pow2f(e - 1075));  // rem rounded to fp32
+  // no conversion instructions (a slow unit on this part): m_hi is in [2^23, 2^24], whose float has the
+  // bit pattern m_hi + 0x4A800000; rem (|rem| <= 2^28) is rounded to fp32 as the fp32 sum of its exact
+  // high part (rem with its low 6 bits cleared) and its exact low 6 bits: one rounding, as a conversion
+  const float mh = __int_as_float(static_cast<int>(m_hi) + 0x4A800000);
+  const int rem_i = static_cast<int>(rem);
+  const float rem_f = __fadd_rn(__fmul_rn(magic_i2f(rem_i >> 6), 64.f), magic_i2f(rem_i & 63));
+  float hi = __fmul_rn(mh, pow2f(e - 1046));  // exact: m_hi <= 2^24
+  float lo = __fmul_rn(rem_f, pow2f(e - 1075));
   if (bits >> 63) {
     hi = -hi;
     lo = -lo;

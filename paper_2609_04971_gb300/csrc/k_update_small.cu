@@ -19,7 +19,10 @@
 //     differ by at most 1e-4 |q| (or a norm is extreme) the query is re-decided
 //     exactly, with the same double-float arithmetic and the same centroid
 //     norm data as the batched kernel (built only when a call needs it), so
-//     both kernels take the same decisions;
+//     both kernels take the same decisions.  Only beacons screened within
+//     2e-4 |q| of the best enter the exact comparison: the screening error is
+//     far below 5e-5 |q|, so the exact maximum (and any exact tie with it)
+//     lies among them;
 //   sums: per touched beacon, the rows assigned to it are added as the same
 //     three exact fp32 parts, turned into round(sum * 2^40), added once to the
 //     fp64 running sum (fold_sum: exact integer addition and one rounding, no
@@ -167,6 +170,7 @@ __global__ void __launch_bounds__(32 * SmallLayout<D, NQ>::kWarps, NQ <= 8 ? 4 :
   // ---- lane r: decision for query r against the centroids at call start
   int dec = -1;
   bool need_exact = false;
+  uint32_t cand = 0;  // candidate beacons of an exact re-decision (lane r: query r)
   if (lane < nq) {
     const float qn2 = qn2s[lane];
     float best = -INFINITY, second = -INFINITY;
@@ -181,15 +185,28 @@ __global__ void __launch_bounds__(32 * SmallLayout<D, NQ>::kWarps, NQ <= 8 ? 4 :
         second = p;
       }
     }
-    need_exact =
-        dec >= 0 && (degenerate || !(qn2 > 1e-30f && qn2 < 1e30f) || !(best - second > kMarginRel * sqrtf(qn2)));
+    const bool wild = degenerate || !(qn2 > 1e-30f && qn2 < 1e30f);
+    need_exact = dec >= 0 && (wild || !(best - second > kMarginRel * sqrtf(qn2)));
+    // Candidates for the exact decision: a screened value is within kMarginRel |q| / 2 of the exact
+    // one, so only beacons screened within 2 kMarginRel |q| of the best can have the largest exact
+    // value (or tie with it); with an extreme norm every valid beacon is a candidate.
+    if (need_exact) {
+      if (wild) {
+        cand = vmask;
+      } else {
+        const float floor_v = best - 2.f * kMarginRel * sqrtf(qn2);
+        for (int b = 0; b < nb; ++b)
+          if (((vmask >> b) & 1u) && sc[lane * SP + b] >= floor_v) cand |= 1u << b;
+      }
+    }
   }
 
   // ---- close calls: exact re-decisions, with the batched kernel's centroid norm data
   const uint32_t need = __ballot_sync(0xffffffffu, need_exact);
+  const uint32_t cand_any = __reduce_or_sync(0xffffffffu, cand);  // beacons whose norm data is needed
   if (need) {
     for (int b = 0; b < nb; ++b) {
-      if (!((vmask >> b) & 1u)) continue;  // warp-uniform
+      if (!((cand_any >> b) & 1u)) continue;  // warp-uniform
       float n2b = 0.f;
       DF n2d{0.f, 0.f};
 #pragma unroll
@@ -210,12 +227,13 @@ __global__ void __launch_bounds__(32 * SmallLayout<D, NQ>::kWarps, NQ <= 8 ? 4 :
     __syncwarp();
     for (uint32_t m = need; m; m &= m - 1) {
       const int r = __ffs(m) - 1;
+      const uint32_t cand_r = __shfl_sync(0xffffffffu, cand, r);
       float x[D / 32];
 #pragma unroll
       for (int j = 0; j < D / 32; ++j) x[j] = qs[r * P + lane + 32 * j];
       const int d = exact_decision<D>(
           x, nb, [&](int b, int col) { return a.cent[cbase + static_cast<size_t>(b) * D + col]; },
-          [&](int b) { return ((vmask >> b) & 1u) != 0; }, cninv);
+          [&](int b) { return ((cand_r >> b) & 1u) != 0; }, cninv);
       if (lane == r) dec = d;
     }
   }
@@ -263,7 +281,7 @@ __global__ void __launch_bounds__(32 * SmallLayout<D, NQ>::kWarps, NQ <= 8 ? 4 :
 #pragma unroll
       for (int j = 0; j < D / 32; ++j) {
         const size_t gi = cbase + static_cast<size_t>(b) * D + lane + 32 * j;
-        const double s_new = fold_sum(s_old[i][j], fixed40(p[j]));
+        const double s_new = fold_sum(s_old[i][j], fixed40_few(p[j]));
         a.sums[gi] = s_new;
         a.cent[gi] = centroid_value(s_new, rcp);
       }

@@ -8,7 +8,9 @@
 //           sum, formed on the host from the exact integer s * 2^40 + acc;
 //   off     s off the 2^-40 grid, at or beyond 2^22, subnormal or zero (the fp64 route):
 //           bit-identical.
-// fold_sum_fp64 (the batched kernel's form) must equal fold_sum bit for bit on every input.
+// fold_sum_fp64 (the batched kernel's form) must equal fold_sum bit for bit on every input;
+// fixed40_few must equal fixed40 on sums of up to 32 values; centroid_value must be within one fp32
+// ulp of s / n.
 // Prints one line per class and exits non-zero on any mismatch.  Test code only.
 #include <cmath>
 #include <cstdint>
@@ -26,6 +28,23 @@ __global__ void fold_kernel(const double* s, const long long* acc, double* got, 
   got[i] = bkv::fold_sum(s[i], acc[i]);
   got64[i] = bkv::fold_sum_fp64(s[i], acc[i]);
   want[i] = acc[i] == 0 ? s[i] : __dadd_rn(s[i], bkv::fixed40_to_double(acc[i]));
+}
+
+// fixed40_few (magic-number conversions) against fixed40 (conversion instructions) on the part sums
+// of up to 32 bf16-exact values, and centroid_value against the exactly computed quotient.
+__global__ void parts_kernel(const float* x, int rows, int n, long long* few, long long* ref) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  bkv::Parts p{0.f, 0.f, 0.f};
+  for (int r = 0; r < rows; ++r) bkv::parts_add(p, x[static_cast<size_t>(i) * rows + r]);
+  few[i] = bkv::fixed40_few(p);
+  ref[i] = bkv::fixed40(p);
+}
+
+__global__ void centroid_kernel(const double* s, const long long* cnt, float* got, int n) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  got[i] = bkv::centroid_value(s[i], bkv::count_reciprocal(cnt[i]));
 }
 
 uint64_t rng_state = 0x9e3779b97f4a7c15ull;
@@ -158,6 +177,74 @@ int main() {
   for (int i = 0; i < n; ++i) forms_differ += to_bits(got[i]) != to_bits(got64[i]);
   std::printf("fold_sum_fp64 differs from fold_sum: %lld of %d\n", forms_differ, n);
   fail |= forms_differ != 0;
+  // ---- fixed40_few against fixed40: 100000 sets of up to 32 values, |x| < 2^14, bf16-exact
+  {
+    const int sets = 100000, rows = 32;
+    std::vector<float> xs(static_cast<size_t>(sets) * rows);
+    for (int i = 0; i < sets; ++i)
+      for (int r = 0; r < rows; ++r) {
+        const int e = -34 + static_cast<int>(next() % 48);                    // 2^-34 .. 2^13
+        const float m = static_cast<float>(128 + (next() % 128)) / 128.f;   // 8 significant bits
+        float v = std::ldexp(m, e);
+        if (next() & 1) v = -v;
+        if (i % 7 == 0) v = (r % 2 ? 1.f : -1.f) * std::ldexp(255.f / 128.f, 13);  // extremes, alternating
+        if (i % 11 == 0) v = std::ldexp(255.f / 128.f, 13);                         // all at the maximum
+        xs[static_cast<size_t>(i) * rows + r] = v;
+      }
+    float* dx;
+    long long *dfew, *dref;
+    cudaMalloc(&dx, sizeof(float) * xs.size());
+    cudaMalloc(&dfew, sizeof(long long) * sets);
+    cudaMalloc(&dref, sizeof(long long) * sets);
+    cudaMemcpy(dx, xs.data(), sizeof(float) * xs.size(), cudaMemcpyHostToDevice);
+    parts_kernel<<<(sets + 255) / 256, 256>>>(dx, rows, sets, dfew, dref);
+    std::vector<long long> hf(sets), hr(sets);
+    cudaMemcpy(hf.data(), dfew, sizeof(long long) * sets, cudaMemcpyDeviceToHost);
+    cudaMemcpy(hr.data(), dref, sizeof(long long) * sets, cudaMemcpyDeviceToHost);
+    long long diff = 0;
+    for (int i = 0; i < sets; ++i) diff += hf[i] != hr[i];
+    std::printf("fixed40_few differs from fixed40: %lld of %d sets of %d values\n", diff, sets, rows);
+    fail |= diff != 0;
+    cudaFree(dx);
+    cudaFree(dfew);
+    cudaFree(dref);
+  }
+  // ---- centroid_value within one fp32 ulp of s / n (host: the fp64 quotient, then fp32)
+  {
+    const int m = 200000;
+    std::vector<double> cs(m);
+    std::vector<long long> cn(m);
+    for (int i = 0; i < m; ++i) {
+      cs[i] = grid_value(-40 + static_cast<int>(next() % 62));
+      cn[i] = 1 + static_cast<long long>(next() % (i % 3 == 0 ? 100 : (i % 3 == 1 ? 100000 : 10000000)));
+    }
+    double* dcs;
+    long long* dcn;
+    float* dcg;
+    cudaMalloc(&dcs, sizeof(double) * m);
+    cudaMalloc(&dcn, sizeof(long long) * m);
+    cudaMalloc(&dcg, sizeof(float) * m);
+    cudaMemcpy(dcs, cs.data(), sizeof(double) * m, cudaMemcpyHostToDevice);
+    cudaMemcpy(dcn, cn.data(), sizeof(long long) * m, cudaMemcpyHostToDevice);
+    centroid_kernel<<<(m + 255) / 256, 256>>>(dcs, dcn, dcg, m);
+    std::vector<float> cg(m);
+    cudaMemcpy(cg.data(), dcg, sizeof(float) * m, cudaMemcpyDeviceToHost);
+    long long off = 0, exact = 0;
+    for (int i = 0; i < m; ++i) {
+      const float ref = static_cast<float>(cs[i] / static_cast<double>(cn[i]));
+      uint32_t a, b;
+      std::memcpy(&a, &cg[i], 4);
+      std::memcpy(&b, &ref, 4);
+      const long long d = static_cast<long long>(a) - static_cast<long long>(b);
+      exact += d == 0;
+      off += d > 1 || d < -1;
+    }
+    std::printf("centroid_value: %lld of %d equal fp32(s / n), %lld more than one ulp away\n", exact, m, off);
+    fail |= off != 0;
+    cudaFree(dcs);
+    cudaFree(dcn);
+    cudaFree(dcg);
+  }
   cudaFree(dg64);
   cudaFree(ds);
   cudaFree(dg);
