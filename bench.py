@@ -69,6 +69,9 @@ def parse():
                     help="Continual FPS: beacons per query head (the buffer holds this + window queries)")
     ap.add_argument("--trace-steps", type=int, default=0,
                     help="decode steps of the long-trace mode (0: the workload's own; config 5 runs a trace)")
+    ap.add_argument("--trace-updates", choices=["seq", "per-step"], default="seq",
+                    help="trace: a period's decode-step beacon updates in one bkv_update_beacons_seq call per "
+                         "contiguous run of pooled queries, or one bkv_update_beacons call per step")
     ap.add_argument("--bmin-ratio", type=float, default=1.0,
                     help="trace mode: B_min / B_max; B_min is the workload's budget and B_max = budget / ratio "
                          "(1.0: the workload's own L, e.g. 7/8 = 0.875 as in the paper's setting)")
@@ -564,10 +567,13 @@ def trace_bench(args, wl, job, cfps: bool, steps: int) -> dict:
     updates the beacons.  With Continual FPS buffers the queries follow Algorithm 2's phases: they feed
     the buffers while L <= B_max - n_recent, the beacons are then fixed (the library selects them from
     the unchanged buffer at the eviction), and the last n_recent queries are kept with their positions
-    for the eviction and the merge that follows it.  The timed quantity is the compression overhead of
-    the whole trace: the device time of every bkv_update_beacons and bkv_compress call, measured with
-    CUDA events on the library's stream (one pair around each compress, one around the back-to-back
-    updates of each period between compresses).  The model's own work (appending the K / V rows,
+    for the eviction and the merge that follows it.  Nothing reads the beacons between two compresses,
+    so by default a period's decode-step updates go to bkv_update_beacons_seq at once (one call per run
+    of contiguous pooled queries; state and assignments bit-identical to one bkv_update_beacons call per
+    step, which --trace-updates per-step times instead).  The timed quantity is the compression
+    overhead of the whole trace: the device time of every beacon update and bkv_compress call, measured
+    with CUDA events on the library's stream (one pair around each compress, one around the updates of
+    each period between compresses).  The model's own work (appending the K / V rows,
     building the recent-query block) runs outside the events.  Queries and K / V rows cycle through
     TRACE_POOL pre-generated decode steps (drifting clusters within the pool), so that host-side input
     generation does not pace the trace."""
@@ -631,14 +637,30 @@ def trace_bench(args, wl, job, cfps: bool, steps: int) -> dict:
     lib = bkv._l()
     qptr = [ctypes.c_void_p(q_pool[j].data_ptr()) for j in range(pool)]
 
-    def update_call(j):
-        rc = lib.bkv_update_beacons(bk.ctx, qptr[j], 1, None)
+    seq_updates = args.trace_updates == "seq"
+
+    def update_call(j, n=1):
+        if seq_updates:
+            rc = lib.bkv_update_beacons_seq(bk.ctx, qptr[j], n, None)
+        else:
+            rc = lib.bkv_update_beacons(bk.ctx, qptr[j], 1, None)
         if rc != bkv.BKV_OK:
             raise bkv.BkvError(rc, "bkv_update_beacons", bkv.bkv_last_error(bk.ctx))
 
+    def runs(idx):
+        """Maximal runs of consecutive pool slots: (first slot, length)."""
+        out = []
+        for j in idx:
+            if out and out[-1][0] + out[-1][1] == j:
+                out[-1][1] += 1
+            else:
+                out.append([j, 1])
+        return out
+
     ends = sorted(set(sched) | ({steps - 1} if steps else set()))
     ev_u, ev_c = [], []
-    n_upd = 0
+    n_upd = n_upd_calls = 0
+    upd_bytes_total = 0
     hist = collections.deque(maxlen=W)   # (query [nl, B, Hq, d], absolute position) of the latest steps
     L, pos, s0 = wl.prefill, wl.prefill, 0
     compress_at = set(sched)
@@ -662,8 +684,16 @@ def trace_bench(args, wl, job, cfps: bool, steps: int) -> dict:
         if upd:
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record()
-            for j in upd:
-                update_call(j)
+            if seq_updates:
+                for j, n_run in runs(upd):
+                    update_call(j, n_run)
+                    n_upd_calls += 1
+                    upd_bytes_total += wl.update_seq_bytes(n_run)
+            else:
+                for j in upd:
+                    update_call(j)
+                n_upd_calls += len(upd)
+                upd_bytes_total += len(upd) * wl.update_bytes(1)
             b.record()
             ev_u.append((a, b))
             n_upd += len(upd)
@@ -694,29 +724,29 @@ def trace_bench(args, wl, job, cfps: bool, steps: int) -> dict:
     upd_ms = sum(x.elapsed_time(y) for x, y in ev_u)
     if n_upd:  # the updates' device time, from the period events (no per-launch events around them)
         name = "cfps" if cfps else "update"
-        prof[name] = (prof[name][0] + upd_ms, prof[name][1] + n_upd)
+        prof[name] = (prof[name][0] + upd_ms, prof[name][1] + n_upd_calls)
     cmp_ms = [x.elapsed_time(y) for x, y in ev_c]
     total_ms = max_over_ranks(upd_ms + sum(cmp_ms), world, dev)
 
     tokens = len(sched) * wl.n_inst * cap * world
     if cfps:  # lower bound: read each new query and write it into its head's buffer
-        upd_bytes = 2 * wl.n_layers * wl.batch * wl.n_q_heads * d * 2
-    else:
-        upd_bytes = wl.update_bytes(1)
-    trace_bytes = len(sched) * wl.compress_bytes() + n_upd * upd_bytes
+        upd_bytes_total = n_upd * 2 * wl.n_layers * wl.batch * wl.n_q_heads * d * 2
+    trace_bytes = len(sched) * wl.compress_bytes() + upd_bytes_total
     trace_flops = len(sched) * wl.compress_flops() + (0 if cfps else n_upd * wl.update_flops(1))
     roof_ms = 1e3 * max(trace_bytes / (hbm_gbs * 1e9), trace_flops / (bf16_tflops * 1e12))
     per_launch_bytes = {"qobs": wl.n_inst * wl.group * W * d * 2, "score": wl.n_inst * cap * d * 2,
                         "select_gather": wl.n_inst * (budget * d * 2 * 4 + budget * 4)}
-    if not cfps:
-        per_launch_bytes["update"] = upd_bytes
     kernels = {}
     for name, (ms, n) in prof.items():
         if not n:
             continue
         k = {"ms_per_launch": ms / n, "launches": n, "ms_total": ms}
-        if name in per_launch_bytes:
-            bl = per_launch_bytes[name] * (len(sched) if name != "update" else n_upd) / n
+        if name == "update" and not cfps:
+            bl = upd_bytes_total / n
+            k.update(alg_bytes_per_launch=bl, achieved_gbs=bl / (ms / n * 1e-3) / 1e9,
+                     frac_of_hbm=bl / (ms / n * 1e-3) / 1e9 / hbm_gbs)
+        elif name in per_launch_bytes:
+            bl = per_launch_bytes[name] * len(sched) / n
             k.update(alg_bytes_per_launch=bl, achieved_gbs=bl / (ms / n * 1e-3) / 1e9,
                      frac_of_hbm=bl / (ms / n * 1e-3) / 1e9 / hbm_gbs)
         kernels[name] = k
@@ -734,16 +764,20 @@ def trace_bench(args, wl, job, cfps: bool, steps: int) -> dict:
         "warmup": args.warmup, "ms_per_step": total_ms / steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": dict(config_block(wl, world), beacon_mode=args.beacons if cfps else "centroid",
-                       decode_steps=steps, compresses=len(sched), beacon_updates=n_upd, b_max=cap, b_min=budget,
+                       decode_steps=steps, compresses=len(sched), beacon_updates=n_upd,
+                       update_calls=n_upd_calls, update_form=args.trace_updates, b_max=cap, b_min=budget,
                        query_pool_steps=pool, l2="K/V working set 10 GB > L2; no flush between decode steps"),
         "roofline": roofline,
         "step_roofline": {"alg_bytes": trace_bytes, "alg_flops": trace_flops, "roofline_ms": roof_ms,
                           "frac": roof_ms / total_ms,
                           "note": "whole trace: every compress plus every beacon update"
+                                  + ("; a seq call reads the centroids once and writes the touched ones once"
+                                     if seq_updates and not cfps else "")
                                   + ("; Continual FPS updates counted as query read + buffer append only"
                                      if cfps else "")},
         "trace": {"overhead_s": total_ms / 1e3, "overhead_us_per_decode_step": 1e3 * total_ms / steps,
-                  "update_us_per_call": 1e3 * upd_ms / max(n_upd, 1),
+                  "update_us_per_decode_step": 1e3 * upd_ms / max(n_upd, 1),
+                  "update_us_per_call": 1e3 * upd_ms / max(n_upd_calls, 1),
                   "compress_ms_mean": statistics.mean(cmp_ms) if cmp_ms else 0.0,
                   "wall_s": wall_s},
         "kernels": kernels, "gpu_launches": sum(n for _, n in prof.values()), "clocks": clocks,

@@ -183,6 +183,25 @@ int bkv_init_beacons(bkv_ctx* ctx, const void* q_init, int32_t n_init);
 int bkv_update_beacons(bkv_ctx* ctx, const void* q_new, int32_t n_new, int32_t* assign_out);
 
 /*
+ * A run of decode steps in one call: step t brings one query per query head
+ * (Algorithm 2's decode branch, one generated token), and the steps are
+ * applied in order, each against the centroids the steps before it left.
+ * The state afterwards and every assignment are bit-identical to those of
+ * n_steps calls of bkv_update_beacons(q_steps + t * step, n_new = 1), under
+ * every flag.  Nothing reads the beacons between two compressions, so a
+ * decode loop may hold a period's queries and hand them over at once; the
+ * state is then read from and written back to device memory once per call
+ * instead of once per step.  The paper has no such call: it is a batching of
+ * Algorithm 2's per-token updates.
+ *   q_steps     bf16 [n_steps][n_layers][batch][n_q_heads][head_dim], pre-RoPE
+ *               (step-major: each step is the q_new of a one-query call).
+ *   assign_out  int32 [n_steps][n_layers][batch][n_q_heads] or NULL.
+ * Same element limits as bkv_update_beacons, per step.  n_steps == 0 is a
+ * no-op.  BKV_ESTATE as bkv_update_beacons.
+ */
+int bkv_update_beacons_seq(bkv_ctx* ctx, const void* q_steps, int32_t n_steps, int32_t* assign_out);
+
+/*
  * One compression of every instance's cache from L rows to `budget` rows.
  * Observation queries (Section 4.3): for each instance, the recent queries of
  * its G query heads, query (h, w) rotated to position recent_pos[w], and its
@@ -238,18 +257,25 @@ int bkv_compress_ragged(bkv_ctx* ctx, void* K, void* V, const int32_t* L, int32_
                         const void* q_recent, const int64_t* recent_pos, int32_t* kept_idx_out, float* scores_out);
 
 /*
- * Copies the beacon state to / from caller DEVICE buffers:
+ * Copies the beacon state to / from caller buffers (checkpoint / resume):
  *   centroids fp32 [n_inst][n_beacons][head_dim]
  *   sums      fp64 [n_inst][n_beacons][head_dim]
  *   counts    int64 [n_inst][n_beacons]
- * Any pointer may be NULL to skip that array (get only).  bkv_set_state
- * needs all three and marks the state as initialised (checkpoint / resume).
+ * Each pointer may be device memory or host memory (pinned or pageable): the
+ * direction of each copy is taken from the pointer (unified addressing).  The
+ * copies are ordered on the context's stream; host results of bkv_get_state
+ * are valid once the stream has been synchronised (bkv_sync), and host
+ * sources of bkv_set_state may be reused when the call returns (a copy from
+ * pageable memory is staged before the call returns).  Any pointer may be
+ * NULL to skip that array (get only).  bkv_set_state needs all three and
+ * marks the state as initialised.
  */
 int bkv_get_state(bkv_ctx* ctx, float* centroids, double* sums, int64_t* counts);
 int bkv_set_state(bkv_ctx* ctx, const float* centroids, const double* sums, const int64_t* counts);
 
 /*
- * Continual FPS contexts: copies the buffers to / from caller DEVICE memory.
+ * Continual FPS contexts: copies the buffers to / from caller memory (device
+ * or host, as for bkv_get_state).
  *   buffers  bf16 [n_layers][batch][n_q_heads][n_beacons + window][head_dim];
  *            rows [0, size) of each head are in use, in buffer order.
  *   sizes    int32 [n_layers][batch][n_q_heads], each in 0..n_beacons + window - 1.

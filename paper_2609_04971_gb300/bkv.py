@@ -69,6 +69,7 @@ def load_library(path: str | None = None, build: bool = True):
             "bkv_set_stream": (ctypes.c_int, [_P, _P]),
             "bkv_init_beacons": (ctypes.c_int, [_P, _P, ctypes.c_int32]),
             "bkv_update_beacons": (ctypes.c_int, [_P, _P, ctypes.c_int32, _P]),
+            "bkv_update_beacons_seq": (ctypes.c_int, [_P, _P, ctypes.c_int32, _P]),
             "bkv_compress": (ctypes.c_int, [_P, _P, _P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, _P, _P,
                                             _P, _P]),
             "bkv_compress_ragged": (ctypes.c_int, [_P, _P, _P, _P, ctypes.c_int32, _P, _P, _P, _P, _P]),
@@ -107,6 +108,17 @@ def _ptr(t: torch.Tensor | None, dtype: torch.dtype, name: str, device=None):
         raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
     if not t.is_cuda:
         raise TypeError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _ptr_any(t: torch.Tensor | None, dtype: torch.dtype, name: str):
+    """Pointer of a CUDA or host tensor (the state copies take their direction from the pointer)."""
+    if t is None:
+        return None
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
     if not t.is_contiguous():
         raise ValueError(f"{name} must be contiguous")
     return ctypes.c_void_p(t.data_ptr())
@@ -171,6 +183,11 @@ def bkv_update_beacons(ctx, q_new: torch.Tensor, n_new: int, assign_out: torch.T
                                    _ptr(assign_out, torch.int32, "assign_out")), "bkv_update_beacons", ctx)
 
 
+def bkv_update_beacons_seq(ctx, q_steps: torch.Tensor, n_steps: int, assign_out: torch.Tensor | None = None) -> None:
+    _check(_l().bkv_update_beacons_seq(ctx, _ptr(q_steps, torch.bfloat16, "q_steps"), int(n_steps),
+                                       _ptr(assign_out, torch.int32, "assign_out")), "bkv_update_beacons_seq", ctx)
+
+
 def bkv_compress(ctx, K: torch.Tensor, V: torch.Tensor, L: int, budget: int, t_pos: int,
                  q_recent: torch.Tensor | None, recent_pos, kept_idx_out: torch.Tensor,
                  scores_out: torch.Tensor | None = None) -> None:
@@ -196,23 +213,26 @@ def bkv_compress_ragged(ctx, K: torch.Tensor, V: torch.Tensor, L: torch.Tensor, 
 
 
 def bkv_get_state(ctx, centroids=None, sums=None, counts=None) -> None:
-    _check(_l().bkv_get_state(ctx, _ptr(centroids, torch.float32, "centroids"), _ptr(sums, torch.float64, "sums"),
-                              _ptr(counts, torch.int64, "counts")), "bkv_get_state", ctx)
+    """Tensors may live on the device or the host; host results are valid after bkv_sync."""
+    _check(_l().bkv_get_state(ctx, _ptr_any(centroids, torch.float32, "centroids"),
+                              _ptr_any(sums, torch.float64, "sums"), _ptr_any(counts, torch.int64, "counts")),
+           "bkv_get_state", ctx)
 
 
 def bkv_set_state(ctx, centroids, sums, counts) -> None:
-    _check(_l().bkv_set_state(ctx, _ptr(centroids, torch.float32, "centroids"), _ptr(sums, torch.float64, "sums"),
-                              _ptr(counts, torch.int64, "counts")), "bkv_set_state", ctx)
+    _check(_l().bkv_set_state(ctx, _ptr_any(centroids, torch.float32, "centroids"),
+                              _ptr_any(sums, torch.float64, "sums"), _ptr_any(counts, torch.int64, "counts")),
+           "bkv_set_state", ctx)
 
 
 def bkv_get_cfps_state(ctx, buffers=None, sizes=None) -> None:
-    _check(_l().bkv_get_cfps_state(ctx, _ptr(buffers, torch.bfloat16, "buffers"), _ptr(sizes, torch.int32, "sizes")),
-           "bkv_get_cfps_state", ctx)
+    _check(_l().bkv_get_cfps_state(ctx, _ptr_any(buffers, torch.bfloat16, "buffers"),
+                                   _ptr_any(sizes, torch.int32, "sizes")), "bkv_get_cfps_state", ctx)
 
 
 def bkv_set_cfps_state(ctx, buffers, sizes) -> None:
-    _check(_l().bkv_set_cfps_state(ctx, _ptr(buffers, torch.bfloat16, "buffers"), _ptr(sizes, torch.int32, "sizes")),
-           "bkv_set_cfps_state", ctx)
+    _check(_l().bkv_set_cfps_state(ctx, _ptr_any(buffers, torch.bfloat16, "buffers"),
+                                   _ptr_any(sizes, torch.int32, "sizes")), "bkv_set_cfps_state", ctx)
 
 
 def bkv_sync(ctx) -> None:
@@ -340,6 +360,17 @@ class BeaconKV:
         c = self.cfg
         self._expect(assign_out, c.n_layers * c.batch * c.n_q_heads * n_new, "assign_out")
         bkv_update_beacons(self.ctx, q_new, n_new, assign_out)
+
+    def update_seq(self, q_steps: torch.Tensor, assign_out: torch.Tensor | None = None):
+        """Decode steps in order: q_steps is [n_steps, n_layers, batch, n_q_heads, head_dim]."""
+        c = self.cfg
+        per_step = c.n_layers * c.batch * c.n_q_heads
+        if q_steps.dim() < 2 or q_steps.shape[-1] != c.head_dim or q_steps.numel() % (per_step * c.head_dim):
+            raise ValueError(f"q_steps must be [n_steps, n_layers, batch, n_q_heads, head_dim = {c.head_dim}], "
+                             f"got {tuple(q_steps.shape)}")
+        n_steps = q_steps.numel() // (per_step * c.head_dim)
+        self._expect(assign_out, per_step * n_steps, "assign_out")
+        bkv_update_beacons_seq(self.ctx, q_steps, n_steps, assign_out)
 
     def compress(self, K, V, *, L, budget, t_pos, q_recent, recent_pos, kept_out=None, scores_out=None):
         c = self.cfg

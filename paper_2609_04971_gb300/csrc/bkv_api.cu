@@ -435,6 +435,34 @@ int bkv_update_beacons(bkv_ctx* ctx, const void* q_new, int32_t n_new, int32_t* 
   return BKV_OK;
 }
 
+int bkv_update_beacons_seq(bkv_ctx* ctx, const void* q_steps, int32_t n_steps, int32_t* assign_out) {
+  if (!ctx) return BKV_EINVAL;
+  const Shape& s = ctx->shape;
+  if (n_steps < 0) return fail(ctx, BKV_EINVAL, "n_steps must be >= 0");
+  if (n_steps == 0) return BKV_OK;
+  if (!q_steps || !aligned16(q_steps)) return fail(ctx, BKV_EINVAL, "q_steps must be a non-NULL 16-byte aligned pointer");
+  if (assign_out && (reinterpret_cast<uintptr_t>(assign_out) & 3u))
+    return fail(ctx, BKV_EINVAL, "assign_out must be 4-byte aligned");
+  const size_t per_step = static_cast<size_t>(s.n_inst) * s.G;  // queries (and assignments) of one step
+  if (1LL * s.n_inst * s.G * n_steps >= (1LL << 31)) return fail(ctx, BKV_EINVAL, "n_steps too large");
+  if (s.nb > 0 && !ctx->state_ready) return fail(ctx, BKV_ESTATE, "update before bkv_init_beacons / bkv_set_state");
+  if (s.nb > 0 && !ctx->cfps && s.G <= bkv::kUpdateSmallMaxRows) {
+    ProfScope ps(ctx, BKV_K_UPDATE);
+    cudaError_t e = bkv::launch_update_seq(s, static_cast<const __nv_bfloat16*>(q_steps), n_steps, ctx->cent,
+                                           ctx->sums, ctx->counts, assign_out, ctx->stream);
+    if (e == cudaSuccess) return BKV_OK;
+    if (e != cudaErrorInvalidValue) return cuda_fail(ctx, e, "update launch");
+    cudaGetLastError();  // the state does not fit in shared memory: step by step below
+  }
+  // step by step: no beacons, Continual FPS buffers, or more query heads per group than one warp takes
+  const char* q = static_cast<const char*>(q_steps);
+  for (int32_t t = 0; t < n_steps; ++t) {
+    const int rc = bkv_update_beacons(ctx, q + t * per_step * s.d * 2, 1, assign_out ? assign_out + t * per_step : nullptr);
+    if (rc != BKV_OK) return rc;
+  }
+  return BKV_OK;
+}
+
 int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int64_t t_pos, const void* q_recent,
                  const int64_t* recent_pos, int32_t* kept_idx_out, float* scores_out) {
   if (!ctx) return BKV_EINVAL;
@@ -708,13 +736,13 @@ int bkv_get_state(bkv_ctx* ctx, float* centroids, double* sums, int64_t* counts)
   const Shape& s = ctx->shape;
   const size_t n = static_cast<size_t>(s.n_inst) * s.nb;
   cudaError_t e = cudaSuccess;
-  if (centroids && (e = cudaMemcpyAsync(centroids, ctx->cent, sizeof(float) * n * s.d, cudaMemcpyDeviceToDevice,
+  if (centroids && (e = cudaMemcpyAsync(centroids, ctx->cent, sizeof(float) * n * s.d, cudaMemcpyDefault,
                                         ctx->stream)) != cudaSuccess)
     return cuda_fail(ctx, e, "get_state centroids");
-  if (sums && (e = cudaMemcpyAsync(sums, ctx->sums, sizeof(double) * n * s.d, cudaMemcpyDeviceToDevice,
+  if (sums && (e = cudaMemcpyAsync(sums, ctx->sums, sizeof(double) * n * s.d, cudaMemcpyDefault,
                                    ctx->stream)) != cudaSuccess)
     return cuda_fail(ctx, e, "get_state sums");
-  if (counts && (e = cudaMemcpyAsync(counts, ctx->counts, sizeof(int64_t) * n, cudaMemcpyDeviceToDevice,
+  if (counts && (e = cudaMemcpyAsync(counts, ctx->counts, sizeof(int64_t) * n, cudaMemcpyDefault,
                                      ctx->stream)) != cudaSuccess)
     return cuda_fail(ctx, e, "get_state counts");
   return BKV_OK;
@@ -727,11 +755,11 @@ int bkv_set_state(bkv_ctx* ctx, const float* centroids, const double* sums, cons
   if (!centroids || !sums || !counts) return fail(ctx, BKV_EINVAL, "set_state needs all three arrays");
   const size_t n = static_cast<size_t>(s.n_inst) * s.nb;
   cudaError_t e;
-  if ((e = cudaMemcpyAsync(ctx->cent, centroids, sizeof(float) * n * s.d, cudaMemcpyDeviceToDevice, ctx->stream)) !=
+  if ((e = cudaMemcpyAsync(ctx->cent, centroids, sizeof(float) * n * s.d, cudaMemcpyDefault, ctx->stream)) !=
           cudaSuccess ||
-      (e = cudaMemcpyAsync(ctx->sums, sums, sizeof(double) * n * s.d, cudaMemcpyDeviceToDevice, ctx->stream)) !=
+      (e = cudaMemcpyAsync(ctx->sums, sums, sizeof(double) * n * s.d, cudaMemcpyDefault, ctx->stream)) !=
           cudaSuccess ||
-      (e = cudaMemcpyAsync(ctx->counts, counts, sizeof(int64_t) * n, cudaMemcpyDeviceToDevice, ctx->stream)) !=
+      (e = cudaMemcpyAsync(ctx->counts, counts, sizeof(int64_t) * n, cudaMemcpyDefault, ctx->stream)) !=
           cudaSuccess)
     return cuda_fail(ctx, e, "set_state copy");
   ctx->state_ready = true;
@@ -744,9 +772,9 @@ int bkv_get_cfps_state(bkv_ctx* ctx, void* buffers, int32_t* sizes) {
   const size_t nh = static_cast<size_t>(ctx->n_heads);
   cudaError_t e = cudaSuccess;
   if (buffers && (e = cudaMemcpyAsync(buffers, ctx->cbuf, sizeof(__nv_bfloat16) * nh * ctx->b_max * ctx->shape.d,
-                                      cudaMemcpyDeviceToDevice, ctx->stream)) != cudaSuccess)
+                                      cudaMemcpyDefault, ctx->stream)) != cudaSuccess)
     return cuda_fail(ctx, e, "get_cfps_state buffers");
-  if (sizes && (e = cudaMemcpyAsync(sizes, ctx->csize, sizeof(int32_t) * nh, cudaMemcpyDeviceToDevice, ctx->stream)) !=
+  if (sizes && (e = cudaMemcpyAsync(sizes, ctx->csize, sizeof(int32_t) * nh, cudaMemcpyDefault, ctx->stream)) !=
                    cudaSuccess)
     return cuda_fail(ctx, e, "get_cfps_state sizes");
   return BKV_OK;
@@ -759,8 +787,8 @@ int bkv_set_cfps_state(bkv_ctx* ctx, const void* buffers, const int32_t* sizes) 
   const size_t nh = static_cast<size_t>(ctx->n_heads);
   cudaError_t e;
   if ((e = cudaMemcpyAsync(ctx->cbuf, buffers, sizeof(__nv_bfloat16) * nh * ctx->b_max * ctx->shape.d,
-                           cudaMemcpyDeviceToDevice, ctx->stream)) != cudaSuccess ||
-      (e = cudaMemcpyAsync(ctx->csize, sizes, sizeof(int32_t) * nh, cudaMemcpyDeviceToDevice, ctx->stream)) !=
+                           cudaMemcpyDefault, ctx->stream)) != cudaSuccess ||
+      (e = cudaMemcpyAsync(ctx->csize, sizes, sizeof(int32_t) * nh, cudaMemcpyDefault, ctx->stream)) !=
           cudaSuccess)
     return cuda_fail(ctx, e, "set_cfps_state");
   ctx->state_ready = true;

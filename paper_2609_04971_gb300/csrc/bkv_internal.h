@@ -67,6 +67,12 @@ cudaError_t launch_update(const Shape& s, const CUtensorMap& qmap, int box_rows,
 constexpr int kUpdateSmallMaxRows = 32;
 cudaError_t launch_update_small(const Shape& s, const __nv_bfloat16* q_new, int n_new, float* cent, double* sums,
                                 long long* counts, int* assign_out, cudaStream_t st);
+// n_steps decode steps of one query per query head, applied in order (k_update_seq.cu): the result of
+// one launch_update_small(n_new = 1) per step, bit for bit.  q_steps: [n_steps][n_inst * G][d];
+// assign_out: [n_steps][n_inst * G] or nullptr.  cudaErrorInvalidValue when G > kUpdateSmallMaxRows or
+// one instance's state does not fit in shared memory (the caller then goes step by step).
+cudaError_t launch_update_seq(const Shape& s, const __nv_bfloat16* q_steps, int n_steps, float* cent, double* sums,
+                              long long* counts, int* assign_out, cudaStream_t st);
 
 // ---- compression (k_qobs.cu, k_score.cu, k_select_gather.cu)
 // rope: [W + 1][d / 2] fp64 (cos, sin) pairs, immediately followed by the same

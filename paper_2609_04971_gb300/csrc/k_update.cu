@@ -342,6 +342,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
         have = __all_sync(0xffffffffu, have);
         float best = -INFINITY, second = -INFINITY, qn2 = 0.f;
         int bi = -1;
+        bool any_valid = false;  // a valid beacon (screened values that are all NaN leave bi at -1)
         if (have) {
           tc_fence_after();
           const uint32_t d = tmem + ab * acc_cols + lane_addr;
@@ -365,6 +366,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
             for (int u = 0; u < 8; ++u) {
               const int b = c0 + u;
               if (b < nb && bvalid[pb][b]) {
+                any_valid = true;
                 const float dot = __uint_as_float(h[u]) + __uint_as_float(l[u]);
                 if (dot > best) {
                   second = best;
@@ -384,7 +386,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
         // ---- decision; close calls go to the exact list; counts per beacon by ballot
         int my_b = -1, my_pos = 0;
         if (have && n < rows) {
-          if (bi >= 0 && (degenerate[pb] || !(qn2 > 1e-30f && qn2 < 1e30f) ||
+          if (any_valid && (degenerate[pb] || !(qn2 > 1e-30f && qn2 < 1e30f) ||
                           !(best - second > kMarginRel * sqrtf(qn2)))) {
             refine_t[ob][atomicAdd(&n_refine[ob], 1)] = n;
           } else {

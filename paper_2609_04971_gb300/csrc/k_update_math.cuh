@@ -95,6 +95,33 @@ __device__ __forceinline__ long long fixed40_few(const Parts& p) {
   return h + m + l;
 }
 
+// fixed40_one below 2^-31 in magnitude (e < 96): x * 2^38 = M / 2^(96 - e) rounded to nearest
+// even, times 4 (0 once the shift reaches 9).  Out of line: rare, and kept off the common path.
+__device__ __noinline__ long long fixed40_one_tiny(int M, int e) {
+  const int sh = 96 - e;
+  if (sh >= 9) return 0;
+  int q = M >> sh;
+  const int rem = M & ((1 << sh) - 1), half = 1 << (sh - 1);
+  if (rem > half || (rem == half && (q & 1))) ++q;
+  return static_cast<long long>(q) << 2;
+}
+
+// round(x * 2^40) of one bf16-exact value x (|x| < 2^14), from integer operations on its bits: what
+// fixed40 gives for the part sums of x alone (exact for |x| >= 2^-31; below, x * 2^38 rounded to the
+// nearest even integer, times 4, as the low part's conversion does).
+__device__ __forceinline__ long long fixed40_one(float x) {
+  const uint32_t b = __float_as_uint(x);
+  const int e = static_cast<int>((b >> 23) & 0xffu);
+  const int M = static_cast<int>(((b >> 16) & 0x7fu) | 0x80u);  // the 8-bit significand
+  long long F;
+  if (e >= 96) {
+    F = static_cast<long long>(M) << (e - 94);  // x * 2^40 = M * 2^(e - 94), exact
+  } else {
+    F = e == 0 ? 0 : fixed40_one_tiny(M, e);  // zero or a subnormal rounds to 0 on the 2^-38 grid
+  }
+  return (b >> 31) ? -F : F;
+}
+
 // Splits the bf16 value x (exact in fp32) into the three parts and adds them.
 __device__ __forceinline__ void parts_add(Parts& p, float x) {
   const float xh = __fadd_rn(__fadd_rn(x, 1572864.f), -1572864.f);  // multiple of 2^-3 (1.5 * 2^20 magic)
@@ -108,12 +135,15 @@ __device__ __forceinline__ void parts_add(Parts& p, float x) {
 // 1 / |c| of a centroid from its double-float sum of squares n2d (fp32 value n2),
 // and whether |c|^2 is far from fp32 over- and underflow (`plain`); outside that
 // range the same quantity is taken in fp64.
-__device__ __forceinline__ DF centroid_inv_norm(DF n2d, float n2, bool& plain) {
-  plain = n2 > 1e-30f && n2 < 1e30f;
-  if (plain) return df_rsqrt(n2d);
+__device__ __noinline__ DF centroid_inv_norm_wide(DF n2d) {
   const double inv = __drcp_rn(sqrt(static_cast<double>(n2d.hi) + static_cast<double>(n2d.lo)));
   const float inv_hi = __double2float_rn(inv);
   return DF{inv_hi, __double2float_rn(inv - static_cast<double>(inv_hi))};
+}
+
+__device__ __forceinline__ DF centroid_inv_norm(DF n2d, float n2, bool& plain) {
+  plain = n2 > 1e-30f && n2 < 1e30f;
+  return plain ? df_rsqrt(n2d) : centroid_inv_norm_wide(n2d);
 }
 
 // The fold of a call's exact sum into the running state.  acc * 2^-40 as a double: one
@@ -146,6 +176,9 @@ __device__ __forceinline__ double fixed40_round(long long t) {
   const unsigned long long e = static_cast<unsigned long long>(msb - 40 + 1023);
   return __longlong_as_double(static_cast<long long>(sign | (e << 52) | (mant & ((1ull << 52) - 1ull))));
 }
+
+// fold_sum's fp64 route, out of line (rare: sums off the 2^-40 grid or at 2^22 and above).
+__device__ __noinline__ double fold_sum_wide(double s, long long acc) { return __dadd_rn(s, fixed40_to_double(acc)); }
 
 // s + acc * 2^-40 rounded to the nearest double (ties to even), the running sum after a call
 // whose exact sum is acc (fixed point, 40 fractional bits).  fp64 arithmetic is slow on this
@@ -181,7 +214,7 @@ __device__ __forceinline__ double fold_sum(double s, long long acc) {
       return t == 0 ? 0.0 : fixed40_round(t);
     }
   }
-  return __dadd_rn(s, fixed40_to_double(acc));
+  return fold_sum_wide(s, acc);
 }
 
 // fold_sum for warps that have the fp64 pipe to themselves: below 2^53, acc * 2^-40 is exact in
@@ -193,14 +226,25 @@ __device__ __forceinline__ double fold_sum_fp64(double s, long long acc) {
   return fold_sum(s, acc);
 }
 
+// n > 2^22 as nf + nl: nf = fp32(n), nl = fp32(n - nf).  Out of line: the 64-bit conversions run on
+// a slow unit of this part, and inlined they would be executed for every count.
+__device__ __noinline__ float2 count_split_large(long long n) {
+  const float nf = static_cast<float>(n);
+  return make_float2(nf, static_cast<float>(n - static_cast<long long>(nf)));
+}
+
 // 1 / n for a count n >= 1 as a double-float: the correctly rounded fp32 reciprocal of n
 // refined by one Newton-Raphson step r' = r + r (1 - n r), the residual formed exactly.
 __device__ __forceinline__ DF count_reciprocal(long long n) {
-  // conversions run on a slow unit of this part: counts up to 2^22 (all practical ones) are exact floats
-  // by the magic-number route (nl = 0), larger ones take the conversion instructions, with equal values
-  const bool small = n <= (1LL << 22);
-  const float nf = small ? magic_i2f(static_cast<int>(n)) : static_cast<float>(n);  // exact below 2^24
-  const float nl = small ? 0.f : static_cast<float>(n - static_cast<long long>(nf));
+  // counts up to 2^22 (all practical ones) are exact floats by the magic-number route (nl = 0)
+  float nf, nl = 0.f;
+  if (n <= (1LL << 22)) {
+    nf = magic_i2f(static_cast<int>(n));
+  } else {
+    const float2 v = count_split_large(n);
+    nf = v.x;
+    nl = v.y;
+  }
   const float r = __frcp_rn(nf);
   const float p = __fmul_rn(nf, r);
   const float pe = __fmaf_rn(nl, r, __fmaf_rn(nf, r, -p));     // n r - p
@@ -218,11 +262,16 @@ __device__ __forceinline__ float pow2f(int k) { return __uint_as_float(static_ca
 // rounded to fp32) by integer operations on its bits, multiplied by rcp as double-floats and
 // rounded once to fp32; within one fp32 ulp of fp32(s / n).  |s| outside [2^-70, 2^100]
 // (and zero) takes the fp64 route.
+// centroid_value outside [2^-70, 2^100] (and at zero), in fp64; out of line so that its fp64
+// instructions are never executed for the common case.
+__device__ __noinline__ float centroid_value_wide(double s, DF rcp) {
+  return __double2float_rn(__dmul_rn(s, __dadd_rn(static_cast<double>(rcp.hi), static_cast<double>(rcp.lo))));
+}
+
 __device__ __forceinline__ float centroid_value(double s, DF rcp) {
   const unsigned long long bits = static_cast<unsigned long long>(__double_as_longlong(s));
   const int e = static_cast<int>((bits >> 52) & 0x7ff);
-  if (e < 1023 - 70 || e > 1023 + 100)
-    return __double2float_rn(__dmul_rn(s, __dadd_rn(static_cast<double>(rcp.hi), static_cast<double>(rcp.lo))));
+  if (e < 1023 - 70 || e > 1023 + 100) return centroid_value_wide(s, rcp);
   const unsigned long long m = (bits & ((1ull << 52) - 1)) | (1ull << 52);  // 53-bit significand
   const unsigned long long m_hi = (m + (1ull << 28) - 1 + ((m >> 29) & 1)) >> 29;  // m / 2^29, nearest even
   const long long rem = static_cast<long long>(m) - static_cast<long long>(m_hi << 29);  // |rem| <= 2^28

@@ -9,8 +9,9 @@
 // gives each centroid row R = 32 / nb lanes (nb rounded up to a power of two):
 //   screening: the R lanes of beacon b stream its row from HBM once, in
 //     interleaved 16-byte chunks (adjacent lanes read adjacent chunks), and
-//     form its squared norm and its dot with every query, added over the R
-//     lanes at the end; the screened value of (query r, beacon b) is
+//     form its squared norm and its dot with every query (packed fp32
+//     multiply-adds, two columns per instruction), added over the R lanes at
+//     the end; the screened value of (query r, beacon b) is
 //     dot * rsqrtf(|c_b|^2), whose error is far below 1e-4 |q|.  The
 //     centroids are never held in shared memory, so every instance of a
 //     decode step fits in one wave;
@@ -70,6 +71,20 @@ struct SmallLayout {
 // prefetched into L2 first).
 constexpr int kFoldChunk = 2;
 
+// Packed fp32 (two columns per instruction, low word first): d = a * b + c.
+__device__ __forceinline__ unsigned long long fma2(unsigned long long a, unsigned long long b, unsigned long long c) {
+  unsigned long long d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ unsigned long long pack2(float lo, float hi) {
+  return static_cast<unsigned long long>(__float_as_uint(lo)) |
+         (static_cast<unsigned long long>(__float_as_uint(hi)) << 32);
+}
+__device__ __forceinline__ float sum2(unsigned long long v) {
+  return __uint_as_float(static_cast<uint32_t>(v)) + __uint_as_float(static_cast<uint32_t>(v >> 32));
+}
+
 template <int D, int NQ>
 __global__ void __launch_bounds__(32 * SmallLayout<D, NQ>::kWarps, NQ <= 8 ? 4 : 2)
     update_small_kernel(SmallArgs a) {
@@ -125,28 +140,30 @@ __global__ void __launch_bounds__(32 * SmallLayout<D, NQ>::kWarps, NQ <= 8 ? 4 :
   const int row = lane >> lg_r, part = lane & (R - 1);
   const bool has_row = row < nb;
   const float4* crow = reinterpret_cast<const float4*>(a.cent + cbase + static_cast<size_t>(has_row ? row : 0) * D);
-  float acc[NQ];
+  // packed fp32 accumulators: even columns in the low word, odd ones in the high word
+  unsigned long long acc2[NQ];
 #pragma unroll
-  for (int r = 0; r < NQ; ++r) acc[r] = 0.f;
-  float n2 = 0.f;
+  for (int r = 0; r < NQ; ++r) acc2[r] = 0ull;
+  unsigned long long n2p = 0ull;
   int nz = 0;
 #pragma unroll(NQ <= 4 ? 4 : 2)
   for (int k = part; k < D / 4; k += R) {
     const float4 c = has_row ? crow[k] : make_float4(0.f, 0.f, 0.f, 0.f);
-    n2 = fmaf(c.x, c.x, n2);
-    n2 = fmaf(c.y, c.y, n2);
-    n2 = fmaf(c.z, c.z, n2);
-    n2 = fmaf(c.w, c.w, n2);
+    const unsigned long long c01 = pack2(c.x, c.y), c23 = pack2(c.z, c.w);
+    n2p = fma2(c01, c01, n2p);
+    n2p = fma2(c23, c23, n2p);
     nz |= (c.x != 0.f) | (c.y != 0.f) | (c.z != 0.f) | (c.w != 0.f);
 #pragma unroll
     for (int r = 0; r < NQ; ++r) {
-      const float4 x = *reinterpret_cast<const float4*>(qs + r * P + 4 * k);  // R distinct addresses per warp
-      acc[r] = fmaf(x.x, c.x, acc[r]);
-      acc[r] = fmaf(x.y, c.y, acc[r]);
-      acc[r] = fmaf(x.z, c.z, acc[r]);
-      acc[r] = fmaf(x.w, c.w, acc[r]);
+      const ulonglong2 x = *reinterpret_cast<const ulonglong2*>(qs + r * P + 4 * k);  // R distinct addresses
+      acc2[r] = fma2(x.x, c01, acc2[r]);
+      acc2[r] = fma2(x.y, c23, acc2[r]);
     }
   }
+  float acc[NQ];
+#pragma unroll
+  for (int r = 0; r < NQ; ++r) acc[r] = sum2(acc2[r]);
+  float n2 = sum2(n2p);
   for (int o = 1; o < R; o <<= 1) {
     n2 += __shfl_xor_sync(0xffffffffu, n2, o);
     nz |= __shfl_xor_sync(0xffffffffu, nz, o);
@@ -186,7 +203,8 @@ __global__ void __launch_bounds__(32 * SmallLayout<D, NQ>::kWarps, NQ <= 8 ? 4 :
       }
     }
     const bool wild = degenerate || !(qn2 > 1e-30f && qn2 < 1e30f);
-    need_exact = dec >= 0 && (wild || !(best - second > kMarginRel * sqrtf(qn2)));
+    // with a valid beacon but no screened best (every value NaN: an extreme norm), best - second is NaN
+    need_exact = vmask != 0u && (wild || !(best - second > kMarginRel * sqrtf(qn2)));
     // Candidates for the exact decision: a screened value is within kMarginRel |q| / 2 of the exact
     // one, so only beacons screened within 2 kMarginRel |q| of the best can have the largest exact
     // value (or tie with it); with an extreme norm every valid beacon is a candidate.
@@ -268,20 +286,29 @@ __global__ void __launch_bounds__(32 * SmallLayout<D, NQ>::kWarps, NQ <= 8 ? 4 :
       if (i >= nbk) break;  // warp-uniform
       const int b = bs[i];
       const uint32_t rows = __ballot_sync(0xffffffffu, lane < nq && dec == b);
-      Parts p[D / 32];
+      long long acc[D / 32];
+      if (__popc(rows) == 1) {  // one query (the common case): its fixed-point value directly
+        const int r = __ffs(rows) - 1;
 #pragma unroll
-      for (int j = 0; j < D / 32; ++j) p[j] = Parts{0.f, 0.f, 0.f};
-      for (uint32_t m = rows; m; m &= m - 1) {
-        const int r = __ffs(m) - 1;
+        for (int j = 0; j < D / 32; ++j) acc[j] = fixed40_one(qs[r * P + lane + 32 * j]);
+      } else {
+        Parts p[D / 32];
 #pragma unroll
-        for (int j = 0; j < D / 32; ++j) parts_add(p[j], qs[r * P + lane + 32 * j]);
+        for (int j = 0; j < D / 32; ++j) p[j] = Parts{0.f, 0.f, 0.f};
+        for (uint32_t m = rows; m; m &= m - 1) {
+          const int r = __ffs(m) - 1;
+#pragma unroll
+          for (int j = 0; j < D / 32; ++j) parts_add(p[j], qs[r * P + lane + 32 * j]);
+        }
+#pragma unroll
+        for (int j = 0; j < D / 32; ++j) acc[j] = fixed40_few(p[j]);
       }
       const long long cnt = __shfl_sync(0xffffffffu, cnt_lane, b) + __popc(rows);
       const DF rcp = count_reciprocal(cnt);
 #pragma unroll
       for (int j = 0; j < D / 32; ++j) {
         const size_t gi = cbase + static_cast<size_t>(b) * D + lane + 32 * j;
-        const double s_new = fold_sum(s_old[i][j], fixed40_few(p[j]));
+        const double s_new = fold_sum(s_old[i][j], acc[j]);
         a.sums[gi] = s_new;
         a.cent[gi] = centroid_value(s_new, rcp);
       }

@@ -88,6 +88,14 @@ class Workload:
         per = nq * d * 2 + self.n_beacons * d * 4 + min(nq, self.n_beacons) * d * 4
         return per * self.n_inst
 
+    def update_seq_bytes(self, n_steps: int) -> int:
+        """Algorithmic HBM bytes of n_steps decode steps (one query per query head each) applied in one
+        call: every step's queries, the centroids read once, the touched centroids written once."""
+        d = self.head_dim
+        nq = self.group * n_steps
+        per = nq * d * 2 + self.n_beacons * d * 4 + min(nq, self.n_beacons) * d * 4
+        return per * self.n_inst
+
     def compress_flops(self) -> int:
         return 2 * self.n_obs * self.L * self.head_dim * self.n_inst
 

@@ -9,8 +9,8 @@
 //   off     s off the 2^-40 grid, at or beyond 2^22, subnormal or zero (the fp64 route):
 //           bit-identical.
 // fold_sum_fp64 (the batched kernel's form) must equal fold_sum bit for bit on every input;
-// fixed40_few must equal fixed40 on sums of up to 32 values; centroid_value must be within one fp32
-// ulp of s / n.
+// fixed40_few must equal fixed40 on sums of up to 32 values, fixed40_one on single values of every
+// exponent; centroid_value must be within one fp32 ulp of s / n.
 // Prints one line per class and exits non-zero on any mismatch.  Test code only.
 #include <cmath>
 #include <cstdint>
@@ -38,6 +38,16 @@ __global__ void parts_kernel(const float* x, int rows, int n, long long* few, lo
   bkv::Parts p{0.f, 0.f, 0.f};
   for (int r = 0; r < rows; ++r) bkv::parts_add(p, x[static_cast<size_t>(i) * rows + r]);
   few[i] = bkv::fixed40_few(p);
+  ref[i] = bkv::fixed40(p);
+}
+
+// fixed40_one (integer operations on the bits) against fixed40 of the parts of one value
+__global__ void one_kernel(const float* x, int n, long long* one, long long* ref) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  bkv::Parts p{0.f, 0.f, 0.f};
+  bkv::parts_add(p, x[i]);
+  one[i] = bkv::fixed40_one(x[i]);
   ref[i] = bkv::fixed40(p);
 }
 
@@ -208,6 +218,39 @@ int main() {
     cudaFree(dx);
     cudaFree(dfew);
     cudaFree(dref);
+  }
+  // ---- fixed40_one against fixed40 on single bf16-exact values of every exponent (2^-140 .. 2^13)
+  {
+    std::vector<float> xs;
+    for (int e = -140; e <= 13; ++e)
+      for (int k = 0; k < 128; ++k) {
+        const float v = std::ldexp(static_cast<float>(128 + k) / 128.f, e);
+        xs.push_back(v);
+        xs.push_back(-v);
+      }
+    xs.push_back(0.f);
+    xs.push_back(-0.f);
+    const int n1 = static_cast<int>(xs.size());
+    float* dx;
+    long long *d1, *dr;
+    cudaMalloc(&dx, sizeof(float) * n1);
+    cudaMalloc(&d1, sizeof(long long) * n1);
+    cudaMalloc(&dr, sizeof(long long) * n1);
+    cudaMemcpy(dx, xs.data(), sizeof(float) * n1, cudaMemcpyHostToDevice);
+    one_kernel<<<(n1 + 255) / 256, 256>>>(dx, n1, d1, dr);
+    std::vector<long long> h1(n1), hr(n1);
+    cudaMemcpy(h1.data(), d1, sizeof(long long) * n1, cudaMemcpyDeviceToHost);
+    cudaMemcpy(hr.data(), dr, sizeof(long long) * n1, cudaMemcpyDeviceToHost);
+    long long diff = 0;
+    for (int i = 0; i < n1; ++i) {
+      if (h1[i] != hr[i] && diff < 3) std::printf("  x = %g: one %lld, parts %lld\n", xs[i], h1[i], hr[i]);
+      diff += h1[i] != hr[i];
+    }
+    std::printf("fixed40_one differs from fixed40 of one value: %lld of %d\n", diff, n1);
+    fail |= diff != 0;
+    cudaFree(dx);
+    cudaFree(d1);
+    cudaFree(dr);
   }
   // ---- centroid_value within one fp32 ulp of s / n (host: the fp64 quotient, then fp32)
   {

@@ -80,3 +80,37 @@ def test_rejected_arguments_leave_everything_untouched():
         assert bool((k_h[:, -wl.window:] == torch.arange(wl.L - wl.window, wl.L, dtype=torch.int32)).all())
     finally:
         bk.close()
+
+
+def test_state_round_trip_through_host_memory():
+    """bkv_get_state / bkv_set_state take host buffers as well as device ones: a state saved to pageable
+    and pinned host tensors and restored into a second context gives, after the same update, the same
+    state as the original context."""
+    from paper_2609_04971_gb300 import bkv, synth
+    from paper_2609_04971_gb300.workloads import QWEN3_4B
+    wl = QWEN3_4B.scaled(name="state_host", n_layers=1, batch=2)
+    dev = torch.device("cuda")
+    inp = synth.step_inputs(wl, 57, dev)
+    a, b = bkv.BeaconKV.for_workload(wl), bkv.BeaconKV.for_workload(wl)
+    try:
+        a.init_beacons(inp["q_init"])
+        a.update(inp["q_new"][..., :64, :].contiguous())
+        shape = (wl.n_inst, wl.n_beacons)
+        host = [torch.empty(shape + (wl.head_dim,), dtype=torch.float32),
+                torch.empty(shape + (wl.head_dim,), dtype=torch.float64, pin_memory=True),
+                torch.empty(shape, dtype=torch.int64)]
+        bkv.bkv_get_state(a.ctx, *host)
+        a.sync()
+        dev_state = a.state()
+        torch.cuda.synchronize()
+        for h, d in zip(host, dev_state):
+            assert torch.equal(h, d.cpu())
+        bkv.bkv_set_state(b.ctx, *host)
+        rest = inp["q_new"][..., 64:, :].contiguous()
+        a.update(rest)
+        b.update(rest)
+        for x, y in zip(a.state(), b.state()):
+            assert torch.equal(x, y)
+    finally:
+        a.close()
+        b.close()
