@@ -36,21 +36,22 @@
 //     does: where its margin test passes, the screened best is the exact
 //     maximum, and otherwise both take the exact argmax;
 //   fold: after a second barrier, each lane folds its own column of every
-//     touched beacon.  While a warp's running sums are multiples of 2^-40
-//     below 2^13 in magnitude (what a sum of bf16 queries of 2^-31 or more
-//     is), each is held exactly as three fp32 parts h + m + l (h a multiple
-//     of 2^-3, |m| <= 2^-4 a multiple of 2^-20, |l| <= 2^-21 a multiple of
-//     2^-40); a query element splits exactly into the same three parts, so a
-//     step adds its rows with fp32 additions that are all exact and carries
-//     between the parts: the exact total, which fold_sum also reaches (no
-//     rounding below 2^13).  The few-query kernel rounds elements below 2^-31
-//     (their sum over a beacon's rows, to a multiple of 2^-38); a step with
-//     such an element sums each beacon's rows first and rounds likewise.  A
-//     warp whose columns leave that range (a sum reaching 2^13, or one that
-//     never was on the grid) keeps doubles and folds with fold_sum.
-//     Centroids are formed at the end, for the touched beacons, from their
-//     final sums and counts (centroid_value's arithmetic, without forming the
-//     double).
+//     touched beacon.  While a warp's running sums are below 2^18 in
+//     magnitude and on the 2^-40 grid (what sums of bf16 queries of 2^-31 or
+//     more are), each is held exactly as three fp32 parts h + m + l (h a
+//     multiple of 2^-3, |m| <= 2^-4 a multiple of 2^-20, |l| <= 2^-21 a
+//     multiple of 2^-40); a query element splits exactly into the same three
+//     parts, so a step adds its rows with fp32 additions that are all exact
+//     and carries between the parts.  That exact total is fold_sum's result
+//     below 2^13; from 2^13 on fold_sum rounds it to its double's grid, and so
+//     does the fold (the low part rounded).  The few-query kernel rounds
+//     elements below 2^-31 (their sum over a beacon's rows, to a multiple of
+//     2^-38); a step with such an element sums each beacon's rows first and
+//     rounds likewise.  A warp whose columns leave that range (a sum reaching
+//     2^18, or one that never was on the grid) keeps doubles and folds with
+//     fold_sum.  Centroids are formed at the end, for the touched beacons,
+//     from their final sums and counts (centroid_value's arithmetic, without
+//     forming the double).
 #include "bkv_device.cuh"
 #include "bkv_internal.h"
 #include "k_update_math.cuh"
@@ -123,13 +124,13 @@ __device__ __forceinline__ float key_value(uint32_t k) {
   return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
 }
 
-// s as the integer s * 2^40 when s is +0 or a multiple of 2^-40 with |s| < 2^13 (then |S| < 2^53).
+// s as the integer s * 2^40 when s is +0 or a multiple of 2^-40 with |s| < 2^18 (then |S| < 2^58).
 __device__ __forceinline__ bool to_fixed(double s, long long& f) {
   const unsigned long long bits = static_cast<unsigned long long>(__double_as_longlong(s));
   const int e = static_cast<int>((bits >> 52) & 0x7ff);
   f = 0;
   if (bits == 0ull) return true;
-  if (e == 0 || e >= 1023 + 13) return false;  // -0, subnormal, or |s| >= 2^13
+  if (e == 0 || e >= 1023 + 18) return false;  // -0, subnormal, or |s| >= 2^18
   const unsigned long long m = (bits & ((1ull << 52) - 1ull)) | (1ull << 52);
   const int sh = e - 1035;  // s * 2^40 = m * 2^(e - 1075 + 40)
   unsigned long long v;
@@ -144,16 +145,18 @@ __device__ __forceinline__ bool to_fixed(double s, long long& f) {
   return true;
 }
 
-// The double S * 2^-40 for |S| < 2^53 (exact; +0 for S = 0): fold_sum's result for that total.
+// The double S * 2^-40 (+0 for S = 0): fold_sum's result for that total (exact when S has at most 53
+// significant bits).
 __device__ __forceinline__ double from_fixed(long long S) { return S == 0 ? 0.0 : fixed40_round(S); }
 
-// centroid_value(S * 2^-40, rcp) for |S| < 2^53, without forming the double: for S = a * 2^-40
-// with a = |S| and p its leading bit, the double's 53-bit significand is a << (52 - p) and its
-// exponent field 983 + p, so centroid_value's split gives hi = m_hi * 2^(p - 63) and lo = rem * 2^(p - 92).
+// centroid_value(S * 2^-40, rcp) for an S of at most 53 significant bits (|S| < 2^63), without forming
+// the double: for a = |S| with leading bit p, the double's 53-bit significand is a shifted to bit 52
+// and its exponent field 983 + p, so centroid_value's split gives hi = m_hi * 2^(p - 63) and
+// lo = rem * 2^(p - 92).
 __device__ __forceinline__ float centroid_fixed(long long S, DF rcp) {
   const unsigned long long a = static_cast<unsigned long long>(S < 0 ? -S : S) | (S == 0 ? 1ull : 0ull);
   const int p = 63 - __clzll(static_cast<long long>(a));
-  const unsigned long long m = a << (52 - p);
+  const unsigned long long m = p >= 52 ? a >> ((p - 52) & 63) : a << ((52 - p) & 63);
   const unsigned long long m_hi = (m + (1ull << 28) - 1 + ((m >> 29) & 1)) >> 29;
   const int rem_i = static_cast<int>(static_cast<long long>(m) - static_cast<long long>(m_hi << 29));
   const float mh = __int_as_float(static_cast<int>(m_hi) + 0x4A800000);
@@ -204,7 +207,7 @@ __device__ __noinline__ long long parts_fixed_wide(float h, float m, float l) {
          static_cast<long long>(magic_f2i(l * 1099511627776.f));
 }
 
-// Carried parts of S * 2^-40 for |S| < 2^53.
+// Carried parts of S * 2^-40 for |S| < 2^58.
 __device__ __forceinline__ void fixed_parts(long long S, float& h, float& m, float& l) {
   const long long hq = (S + (1ll << 36)) >> 37;
   const long long rem = S - (hq << 37);
@@ -213,6 +216,25 @@ __device__ __forceinline__ void fixed_parts(long long S, float& h, float& m, flo
   h = magic_i2f(static_cast<int>(hq)) * 0.125f;
   m = magic_i2f(static_cast<int>(mq)) * 9.5367431640625e-07f;          // 2^-20
   l = magic_i2f(static_cast<int>(lq)) * 9.094947017729282e-13f;        // 2^-40
+}
+
+// floor(log2 |h + m + l|) of carried parts with a nonzero total, from the exact integer.
+__device__ __noinline__ int parts_exponent(float h, float m, float l) {
+  const long long S = parts_fixed(h, m, l);
+  return 23 - __clzll(S < 0 ? -S : S);  // (63 - clz) - 40
+}
+
+// From 2^13 on, a double's grid is coarser than 2^-40, and fold_sum rounds each step's exact total to
+// it (to nearest, ties to even).  For carried parts of a total s with |s| < 2^18 (sv: s to within
+// 2^-22 relative) that is the low part rounded to a multiple of 2^(e - 52), e = floor(log2 |s|): h and
+// m are multiples of 2^-20, so they do not change, and the total's last kept bit is l's.  e is read
+// from sv unless sv lies within 2^-19 relative of a power of two, where it is taken exactly.
+__device__ __forceinline__ void round_to_double(float h, float m, float& l, float sv) {
+  const uint32_t bits = __float_as_uint(sv);
+  int e = static_cast<int>((bits >> 23) & 0xffu) - 127;
+  const uint32_t man = bits & 0x7fffffu;
+  if (e >= 12 && (man < 16u || man > 0x7fffefu)) e = parts_exponent(h, m, l);
+  if (e >= 13) l = magic_i2f(magic_f2i(l * pow2f(52 - e))) * pow2f(e - 52);
 }
 
 // Shared-memory views of one CTA's instance.
@@ -513,7 +535,7 @@ __global__ void __launch_bounds__(D, (NQ <= 8 ? 5 : 3) * 128 / D) update_seq_ker
         const int decr = lane < nq ? dec_sh[lane] : -1;  // lane r: query r's beacon
         const uint32_t touched = __reduce_or_sync(0xffffffffu, decr >= 0 ? (1u << decr) : 0u);
         touched_all |= touched;
-        bool out = false;  // a sum reaching 2^13 in parts form
+        bool out = false;  // a sum reaching 2^18 in parts form
         int tiny = 0;
 #pragma unroll
         for (int r = 0; r < NQ; ++r) {
@@ -531,11 +553,12 @@ __global__ void __launch_bounds__(D, (NQ <= 8 ? 5 : 3) * 128 / D) update_seq_ker
               split3(Q_sh[r * QP + col], xh, xm, xl);
               float h = __fadd_rn(Ph[i], xh), mm = __fadd_rn(Pm[i], xm), l = __fadd_rn(Pl[i], xl);
               carry3(h, mm, l);
+              const float sv = __fadd_rn(__fadd_rn(h, mm), l);  // the sum within 2^-22 relative; 0 iff it is 0
+              if (__any_sync(0xffffffffu, fabsf(sv) >= 8191.f)) round_to_double(h, mm, l, sv);
               Ph[i] = h;
               Pm[i] = mm;
               Pl[i] = l;
-              out |= fabsf(h) > 8191.f;
-              const float sv = __fadd_rn(__fadd_rn(h, mm), l);  // the sum within 2^-23 relative; 0 iff it is 0
+              out |= fabsf(sv) >= 262143.f;
               C_sh[b * CP + col] = sv;
               nzbits = (nzbits & ~(1u << b)) | ((sv != 0.f ? 1u : 0u) << b);  // the centroid is 0 iff the sum is
               if (lane == b) ++cnt_add;
@@ -565,11 +588,12 @@ __global__ void __launch_bounds__(D, (NQ <= 8 ? 5 : 3) * 128 / D) update_seq_ker
               ls = __fadd_rn(ls, -lc);
               float h = __fadd_rn(Ph[i], hs), mm = __fadd_rn(Pm[i], ms), l = __fadd_rn(Pl[i], ls);
               carry3(h, mm, l);
+              c = __fadd_rn(__fadd_rn(h, mm), l);
+              if (__any_sync(0xffffffffu, fabsf(c) >= 8191.f)) round_to_double(h, mm, l, c);
               Ph[i] = h;
               Pm[i] = mm;
               Pl[i] = l;
-              out |= fabsf(h) > 8191.f;
-              c = __fadd_rn(__fadd_rn(h, mm), l);
+              out |= fabsf(c) >= 262143.f;
               C_sh[b * CP + col] = c;
             } else {
               const double s_new = fold_sum(get_d(i), fixed40_few(Parts{hs, ms, ls}));
@@ -581,8 +605,8 @@ __global__ void __launch_bounds__(D, (NQ <= 8 ? 5 : 3) * 128 / D) update_seq_ker
           }
         }
         if (fixed && __any_sync(0xffffffffu, out)) {
-          // a sum reached 2^13: this warp's columns go to fp64 form for good.  The parts hold the exact
-          // totals; fold_sum rounds each once, as fixed40_round does (exact for the untouched ones)
+          // a sum reached 2^18: this warp's columns go to fp64 form for good.  The parts hold the
+          // running sums exactly (each on its double's grid)
           for (int b = 0; b < nb; ++b) {
             const int i = b * D + col;
             put_d(i, from_fixed(parts_fixed_wide(Ph[i], Pm[i], Pl[i])));

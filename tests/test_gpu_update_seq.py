@@ -180,3 +180,47 @@ def test_seq_rejects_bad_arguments():
         bkv.bkv_update_beacons_seq(bk.ctx, q, 0)  # no-op, even before any state
     finally:
         bk.close()
+
+
+def _large_state(wl, seed, base, spread):
+    """Sums far from zero (|s| around `base`, on the 2^-40 grid), counts in the thousands, centroids
+    fp32(s / n): the running sums cross 2^13, 2^14, ... (the double's grid coarsens) over the steps."""
+    n_inst, nb, d = wl.n_inst, wl.n_beacons, wl.head_dim
+    g = torch.Generator().manual_seed(seed)
+    counts = torch.randint(2000, 6000, (n_inst, nb), generator=g, dtype=torch.int64)
+    sign = torch.where(torch.rand(n_inst, nb, d, generator=g) < 0.5, -1.0, 1.0).double()
+    mag = base + spread * torch.rand(n_inst, nb, d, generator=g, dtype=torch.float64)
+    sums = torch.round(sign * mag * 2.0 ** 20) / 2.0 ** 20  # multiples of 2^-20
+    cent = (sums / counts.unsqueeze(-1).double()).float()
+    return cent, sums, counts
+
+
+@pytest.mark.parametrize("case", ["cross_2p13", "near_binades", "past_2p18"])
+def test_seq_large_running_sums(case):
+    """Running sums past 2^13, where fold_sum rounds every step's total to the double's grid: the seq
+    kernel's exact parts must round alike; sums starting just below powers of two (the binade read
+    exactly); sums that reach 2^18 (the warp's columns go to fp64 form mid-call)."""
+    wl = QWEN3_8B_TRACE.scaled(name="large", n_layers=1, batch=2, n_q_heads=16, n_kv_heads=4, n_beacons=8,
+                               n_clusters=8)
+    base, spread = {"cross_2p13": (7000.0, 3000.0), "near_binades": (0.0, 0.0),
+                    "past_2p18": (260000.0, 3000.0)}[case]
+    cent, sums, counts = _large_state(wl, 40, base, spread)
+    if case == "near_binades":  # each element a few 2^-20 steps below 2^k, k = 13 .. 17
+        g = torch.Generator().manual_seed(41)
+        k = torch.randint(13, 18, sums.shape, generator=g)
+        below = torch.randint(1, 64, sums.shape, generator=g).double() * 2.0 ** -20
+        sgn = torch.where(torch.rand(sums.shape, generator=g) < 0.5, -1.0, 1.0).double()
+        sums = sgn * (2.0 ** k.double() - below)
+        cent = (sums / counts.unsqueeze(-1).double()).float()
+    steps = 60
+    n_inst, G, d = wl.n_inst, wl.group, wl.head_dim
+    g = torch.Generator().manual_seed(42)
+    pick = torch.randint(0, wl.n_beacons, (steps, n_inst, G), generator=g)
+    direction = torch.sign(cent)  # queries along the centroids' signs: the sums keep growing in magnitude
+    q = torch.stack([torch.stack([direction[e, pick[t, e]] for e in range(n_inst)]) for t in range(steps)])
+    scale = 2.0 ** -10 if case == "near_binades" else 3.0
+    noise = torch.randn(q.shape, generator=g) * (0.25 * scale)
+    q = (q * scale + noise).to(torch.bfloat16)
+    q = q.view(steps, wl.n_layers, wl.batch, wl.n_q_heads, d).cuda().contiguous()
+    a = _compare(wl, q, state=(cent.cuda(), sums.cuda(), counts.cuda()))
+    assert (a >= 0).all()
