@@ -298,10 +298,10 @@ __device__ __forceinline__ float centroid_value(double s, DF rcp) {
 // the valid beacon maximising (q . c_b) * (1 / |c_b|) in double-float arithmetic (exact
 // products, TwoSum accumulation, then a butterfly over the lanes), ties to the lower
 // beacon; -1 for a zero query or when no beacon is valid.  cent_at(b, col) reads centroid
-// b; valid(b) is warp-uniform.
-template <int D, typename CentAt, typename Valid>
+// b; valid(b) is warp-uniform; cninv[b] is 1 / |c_b| (a pointer, or any type with that operator).
+template <int D, typename CentAt, typename Valid, typename CnInv>
 __device__ __forceinline__ int exact_decision(const float (&x)[D / 32], int nb, CentAt cent_at, Valid valid,
-                                              const DF* cninv) {
+                                              const CnInv& cninv) {
   const int lane = threadIdx.x & 31;
   int nz = 0;
 #pragma unroll

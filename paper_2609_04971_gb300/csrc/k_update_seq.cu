@@ -71,11 +71,13 @@ struct SeqArgs {
 
 // Shared memory of one CTA (one instance), byte offsets.
 struct SeqLayout {
-  size_t s, c, q, dots, norms, nzf, mode, qn2, dec, cninv, rcp, total;
+  size_t s, c, q, dots, norms, nzf, mode, qn2, dec, total;
 };
 
 __host__ __device__ inline SeqLayout seq_layout(int D, int NQ, int nb, int R) {
   const int W = D / 32;
+  int nbp = 1;
+  while (nbp < nb) nbp <<= 1;
   SeqLayout L;
   size_t o = 0;
   L.s = o;  // float [3][nb][D]: the parts h, m, l of each running sum (fp64 form: its bits in h and m)
@@ -84,8 +86,8 @@ __host__ __device__ inline SeqLayout seq_layout(int D, int NQ, int nb, int R) {
   o += 4ull * nb * (D + 4 * R);
   L.q = o;  // float [NQ][D + 4]: the step's queries
   o += 4ull * NQ * (D + 4);
-  L.dots = o;  // float [W][NQ][32]: partial dots
-  o += 4ull * W * NQ * 32;
+  L.dots = o;  // float [W][NQ][nbp]: partial dots (nbp: nb rounded up to a power of two)
+  o += 4ull * W * NQ * nbp;
   L.norms = o;  // float [W][32]: partial squared norms of the screening rows
   o += 4ull * W * 32;
   L.nzf = o;  // uint32 [W]: bit b set when centroid b has a nonzero element among the warp's columns
@@ -96,11 +98,6 @@ __host__ __device__ inline SeqLayout seq_layout(int D, int NQ, int nb, int R) {
   o += 4ull * W * NQ;
   L.dec = o;  // int [NQ]: the step's decisions
   o += 4ull * NQ;
-  o = (o + 15) / 16 * 16;
-  L.cninv = o;  // DF [W][kMaxBeacons]: 1 / |c_b| for exact re-decisions, per warp
-  o += 8ull * W * kMaxBeacons;
-  L.rcp = o;  // DF [W][kMaxBeacons]: 1 / count of touched candidates, per warp
-  o += 8ull * W * kMaxBeacons;
   L.total = (o + 15) / 16 * 16;
   return L;
 }
@@ -237,6 +234,15 @@ __device__ __forceinline__ void round_to_double(float h, float m, float& l, floa
   if (e >= 13) l = magic_i2f(magic_f2i(l * pow2f(52 - e))) * pow2f(e - 52);
 }
 
+// Per-beacon double-float values held by the lanes of a warp (lane b: beacon b); [b] reads beacon b's
+// (b warp-uniform, every lane calling).
+struct LaneDF {
+  DF v;
+  __device__ __forceinline__ DF operator[](int b) const {
+    return DF{__shfl_sync(0xffffffffu, v.hi, b), __shfl_sync(0xffffffffu, v.lo, b)};
+  }
+};
+
 // Shared-memory views of one CTA's instance.
 struct SeqShared {
   float *Ph, *Pm, *Pl;  // parts of the running sums, [nb][D] each (fp64 form: bits in Ph and Pm)
@@ -249,25 +255,21 @@ struct SeqShared {
 // The exact centroid of (beacon b, column c) as the few-query kernel holds it after the steps so far:
 // the loaded centroid until b is touched, then centroid_value of its running sum (rcp: 1 / count).
 template <int D>
-__device__ __forceinline__ float seq_exact_c(const SeqShared& sh, uint32_t touched_all, const DF* rcp, int b, int c) {
+__device__ __forceinline__ float seq_exact_c(const SeqShared& sh, uint32_t touched_all, const LaneDF& rcp, int b, int c) {
   if (!((touched_all >> b) & 1u)) return sh.C[b * sh.CP + c];
   const int i = b * D + c;
-  if (sh.mode[c >> 5]) return centroid_fixed(parts_fixed(sh.Ph[i], sh.Pm[i], sh.Pl[i]), rcp[b]);
-  return centroid_value(__hiloint2double(__float_as_int(sh.Pm[i]), __float_as_int(sh.Ph[i])), rcp[b]);
+  const DF rb = rcp[b];
+  if (sh.mode[c >> 5]) return centroid_fixed(parts_fixed(sh.Ph[i], sh.Pm[i], sh.Pl[i]), rb);
+  return centroid_value(__hiloint2double(__float_as_int(sh.Pm[i]), __float_as_int(sh.Ph[i])), rb);
 }
 
 // Exact re-decision of query r among the candidate beacons (warp-wide; lane b holds beacon b's count):
 // the few-query kernel's double-float arithmetic on whole rows of exact centroids.  Out of line: rare.
 template <int D>
 __device__ __noinline__ int seq_exact(const SeqShared& sh, int r, uint32_t cand, int nb, uint32_t touched_all,
-                                      long long cnt, DF* rcp, DF* cninv) {
+                                      long long cnt) {
   const int lane = threadIdx.x & 31;
-  for (uint32_t m = cand & touched_all; m; m &= m - 1) {
-    const int b = __ffs(m) - 1;
-    const DF rb = count_reciprocal(__shfl_sync(0xffffffffu, cnt, b));
-    if (lane == 0) rcp[b] = rb;
-  }
-  __syncwarp();
+  LaneDF rcp{count_reciprocal(cnt > 0 ? cnt : 1)}, cninv{DF{0.f, 0.f}};  // lane b: beacon b's 1 / count
   for (uint32_t m = cand; m; m &= m - 1) {
     const int b = __ffs(m) - 1;
     float n2b = 0.f;
@@ -285,16 +287,14 @@ __device__ __noinline__ int seq_exact(const SeqShared& sh, int r, uint32_t cand,
       n2d = df_add(n2d, DF{__shfl_xor_sync(0xffffffffu, n2d.hi, o), __shfl_xor_sync(0xffffffffu, n2d.lo, o)});
     bool plain = true;
     const DF inv_df = centroid_inv_norm(n2d, n2b, plain);
-    if (lane == 0) cninv[b] = inv_df;
+    if (lane == b) cninv.v = inv_df;
   }
-  __syncwarp();
   float x[D / 32];
 #pragma unroll
   for (int j = 0; j < D / 32; ++j) x[j] = sh.Q[r * (D + 4) + lane + 32 * j];
   const int d = exact_decision<D>(
       x, nb, [&](int b, int c) { return seq_exact_c<D>(sh, touched_all, rcp, b, c); },
       [&](int b) { return ((cand >> b) & 1u) != 0; }, cninv);
-  __syncwarp();
   return d;
 }
 
@@ -334,7 +334,7 @@ __device__ __forceinline__ void seq_screen(const float* crow, const float* qw, f
 }
 
 template <int D, int NQ>
-__global__ void __launch_bounds__(D, (NQ <= 8 ? 5 : 3) * 128 / D) update_seq_kernel(SeqArgs a) {
+__global__ void __launch_bounds__(D, (NQ <= 8 ? 6 : 3) * 128 / D) update_seq_kernel(SeqArgs a) {
   constexpr int W = D / 32;  // warps per CTA; warp w owns columns [32 w, 32 w + 32)
   constexpr int QP = D + 4;  // query row pitch (floats)
   constexpr int QU = NQ / 4; // 8-byte query loads per lane and step: NQ rows x 32 columns per warp
@@ -347,6 +347,8 @@ __global__ void __launch_bounds__(D, (NQ <= 8 ? 5 : 3) * 128 / D) update_seq_ker
   const bool has_row = row < nb;
   const int CP = D + (4 << lg_r);  // screening row pitch (floats): R lanes' 16-byte reads conflict-free
   const int col = 32 * w + lane;   // this lane's column in the fold
+  int nbp = 1;                     // nb rounded up to a power of two: the partial dots' row pitch
+  while (nbp < nb) nbp <<= 1;
   const SeqLayout lay = seq_layout(D, NQ, nb, 1 << lg_r);
   SeqShared sh;
   sh.Ph = reinterpret_cast<float*>(seq_sh + lay.s);
@@ -366,8 +368,6 @@ __global__ void __launch_bounds__(D, (NQ <= 8 ? 5 : 3) * 128 / D) update_seq_ker
   uint32_t* nzw = reinterpret_cast<uint32_t*>(seq_sh + lay.nzf);  // [W]: the warps' nonzero masks
   float* qn2p = reinterpret_cast<float*>(seq_sh + lay.qn2);
   int* dec_sh = reinterpret_cast<int*>(seq_sh + lay.dec);
-  DF* cninv = reinterpret_cast<DF*>(seq_sh + lay.cninv) + w * kMaxBeacons;
-  DF* rcpx = reinterpret_cast<DF*>(seq_sh + lay.rcp) + w * kMaxBeacons;
   const size_t step_elems = static_cast<size_t>(a.n_inst) * nq * D;  // one step's query block
   // a running sum in fp64 form: its bits in the h and m slots
   auto get_d = [&](int i) { return __hiloint2double(__float_as_int(Pm[i]), __float_as_int(Ph[i])); };
@@ -475,7 +475,7 @@ __global__ void __launch_bounds__(D, (NQ <= 8 ? 5 : 3) * 128 / D) update_seq_ker
         }
         if ((lane & ((1 << lg_r) - 1)) == 0 && has_row) {
 #pragma unroll
-          for (int r = 0; r < NQ; ++r) dots[(w * NQ + r) * 32 + row] = acc[r];
+          for (int r = 0; r < NQ; ++r) dots[(w * NQ + r) * nbp + row] = acc[r];
           norms[w * 32 + row] = n2;
         }
         const uint32_t nzm = __reduce_or_sync(0xffffffffu, nzbits);
@@ -501,7 +501,7 @@ __global__ void __launch_bounds__(D, (NQ <= 8 ? 5 : 3) * 128 / D) update_seq_ker
 #pragma unroll
           for (int v = 0; v < W; ++v) {
             qn2 += qn2p[v * NQ + r];
-            dot += dots[(v * NQ + r) * 32 + lane];
+            dot += lane < nb ? dots[(v * NQ + r) * nbp + lane] : 0.f;
           }
           const float val = valid ? dot * inv : -INFINITY;
           const uint32_t key = order_key(val, valid);
@@ -519,7 +519,7 @@ __global__ void __launch_bounds__(D, (NQ <= 8 ? 5 : 3) * 128 / D) update_seq_ker
             // candidates: a screened value is within kMarginRel |q| / 2 of the exact one, so only beacons
             // screened within 2 kMarginRel |q| of the best can have the largest exact value
             const uint32_t cand = wild ? vmask : __ballot_sync(0xffffffffu, valid && val >= best - 2.f * margin);
-            dec = seq_exact<D>(sh, r, cand, nb, touched_all, cnt_base + cnt_add, rcpx, cninv);
+            dec = seq_exact<D>(sh, r, cand, nb, touched_all, cnt_base + cnt_add);
           }
           if (lane == 0) {
             dec_sh[r] = dec;
@@ -554,13 +554,18 @@ __global__ void __launch_bounds__(D, (NQ <= 8 ? 5 : 3) * 128 / D) update_seq_ker
               float h = __fadd_rn(Ph[i], xh), mm = __fadd_rn(Pm[i], xm), l = __fadd_rn(Pl[i], xl);
               carry3(h, mm, l);
               const float sv = __fadd_rn(__fadd_rn(h, mm), l);  // the sum within 2^-22 relative; 0 iff it is 0
-              if (__any_sync(0xffffffffu, fabsf(sv) >= 8191.f)) round_to_double(h, mm, l, sv);
+              // the centroid is 0 iff the sum is; sums from 2^13 on are rounded to their double's grid
+              if (__any_sync(0xffffffffu, fabsf(sv) >= 8191.f || sv == 0.f)) {
+                round_to_double(h, mm, l, sv);
+                out |= fabsf(sv) >= 262143.f;
+                nzbits = (nzbits & ~(1u << b)) | ((sv != 0.f ? 1u : 0u) << b);
+              } else {
+                nzbits |= 1u << b;
+              }
               Ph[i] = h;
               Pm[i] = mm;
               Pl[i] = l;
-              out |= fabsf(sv) >= 262143.f;
               C_sh[b * CP + col] = sv;
-              nzbits = (nzbits & ~(1u << b)) | ((sv != 0.f ? 1u : 0u) << b);  // the centroid is 0 iff the sum is
               if (lane == b) ++cnt_add;
             }
           }
@@ -654,6 +659,9 @@ cudaError_t launch_seq_dq(const SeqArgs& a, int sms, cudaStream_t st) {
   if (lay.total > 227 * 1024) return cudaErrorInvalidValue;
   cudaError_t e = cudaFuncSetAttribute(update_seq_kernel<D, NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(lay.total));
+  if (e == cudaSuccess)  // all of the SM's on-chip memory as shared memory: the CTAs per SM are smem-bound
+    e = cudaFuncSetAttribute(update_seq_kernel<D, NQ>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
   if (e != cudaSuccess) return e;
   int per_sm = 0;
   e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, update_seq_kernel<D, NQ>, D, lay.total);
