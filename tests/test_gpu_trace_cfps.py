@@ -1,7 +1,9 @@
 """Algorithm 2's phase machine on a decode trace, Continual FPS beacons, through the C ABI.
 
 A shortened long-decode workload (one layer, one batch row, 8 KV heads, 4 query
-heads per KV head, drifting query clusters) after a 128-token prompt:
+heads per KV head, drifting query clusters) after a 128-token prompt, at two
+B_max -> B_min settings (320 -> 256, and 320 -> 280 = 7/8 B_max with 4 leading
+rows always kept):
 
   * while the cache holds at most B_max - window rows, each step's query of
     every head joins that head's buffer (bkv_update_beacons, n_new = 1;
@@ -36,11 +38,14 @@ def _bits(t: torch.Tensor) -> np.ndarray:
     return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
 
 
-@pytest.mark.parametrize("steps,b_min,kv_min,kv_grow", [(420, 8, 256, 64)])
-def test_algorithm2_trace_every_step(steps, b_min, kv_min, kv_grow):
+@pytest.mark.parametrize("steps,b_min,kv_min,kv_grow,n_prefix", [
+    (420, 8, 256, 64, 0),
+    (420, 8, 280, 40, 4),  # B_min = 7/8 B_max (Section 4.1), with 4 leading rows always kept
+])
+def test_algorithm2_trace_every_step(steps, b_min, kv_min, kv_grow, n_prefix):
     kv_max = kv_min + kv_grow
     wl = QWEN3_8B_TRACE.scaled(name="trace_cfps_1L_b1", n_layers=1, batch=1, L=kv_max, budget=kv_min,
-                               trace_steps=steps)
+                               trace_steps=steps, n_prefix=n_prefix)
     dev = torch.device("cuda")
     lib = O.load()
     G, d, W, Hq = wl.group, wl.head_dim, wl.window, wl.n_q_heads
@@ -57,7 +62,8 @@ def test_algorithm2_trace_every_step(steps, b_min, kv_min, kv_grow):
     recent, recent_pos = [], []
 
     bk = BeaconKV(n_layers=wl.n_layers, batch=wl.batch, n_q_heads=Hq, n_kv_heads=wl.n_kv_heads, head_dim=d,
-                  n_beacons=b_min, window=W, capacity=kv_max, rope_theta=wl.rope_theta, continual_fps=True)
+                  n_beacons=b_min, window=W, capacity=kv_max, rope_theta=wl.rope_theta, n_prefix=wl.n_prefix,
+                  continual_fps=True)
 
     def state():
         buf, sizes = bk.cfps_state()
