@@ -225,13 +225,16 @@ __device__ __noinline__ int parts_exponent(float h, float m, float l) {
 // it (to nearest, ties to even).  For carried parts of a total s with |s| < 2^18 (sv: s to within
 // 2^-22 relative) that is the low part rounded to a multiple of 2^(e - 52), e = floor(log2 |s|): h and
 // m are multiples of 2^-20, so they do not change, and the total's last kept bit is l's.  e is read
-// from sv unless sv lies within 2^-19 relative of a power of two, where it is taken exactly.
+// from sv unless sv lies within 2^-19 relative of a power of two, where it is taken exactly.  The
+// rounding adds and subtracts 1.5 * 2^(e - 29), whose ulp is the grid (|l| <= 2^-21 is far below it;
+// the constant's even multiple of the grid keeps ties to even); below 2^13 it adds and subtracts 0.
 __device__ __forceinline__ void round_to_double(float h, float m, float& l, float sv) {
   const uint32_t bits = __float_as_uint(sv);
   int e = static_cast<int>((bits >> 23) & 0xffu) - 127;
   const uint32_t man = bits & 0x7fffffu;
   if (e >= 12 && (man < 16u || man > 0x7fffefu)) e = parts_exponent(h, m, l);
-  if (e >= 13) l = magic_i2f(magic_f2i(l * pow2f(52 - e))) * pow2f(e - 52);
+  const float c = e >= 13 ? __uint_as_float((static_cast<uint32_t>(e + 98) << 23) | 0x400000u) : 0.f;
+  l = __fadd_rn(__fadd_rn(l, c), -c);
 }
 
 // Per-beacon double-float values held by the lanes of a warp (lane b: beacon b); [b] reads beacon b's
