@@ -450,3 +450,45 @@ def check_cfps_compress(wl: Workload, b_min: int, buf: np.ndarray, size: np.ndar
     rel, swaps = check_compress(wl, cent, counts, q_rec, recent_pos, t_pos, K0, V0, K1, V1, kept_g, scores_g, L,
                                 budget, lib, tag=tag, mean=mean, causal=causal)
     return rel, swaps, ties
+
+
+def smoke_decode_steps(wl: Workload, steps: int, seed: int) -> str:
+    """A few decode steps (one query per query head each) on the GPU: one bkv_update_beacons call per
+    step, each checked against the oracle from the state the GPU carried forward, and the same steps in
+    one bkv_update_beacons_seq call, whose state and assignments must be bit-identical."""
+    import torch
+    from paper_2609_04971_gb300 import bkv, synth
+    lib = O.load()
+    dev = torch.device("cuda")
+    q_init = synth.queries(wl, seed, "q_init", wl.n_init, dev)
+    q = synth.queries(wl, seed, "q_decode", steps, dev)                 # [layers, batch, Hq, steps, d]
+    q_steps = q.permute(3, 0, 1, 2, 4).contiguous()                    # [steps, layers, batch, Hq, d]
+    per_step = wl.n_layers * wl.batch * wl.n_q_heads
+    outs, ties = [], 0
+    for seq in (False, True):
+        bk = bkv.BeaconKV.for_workload(wl)
+        try:
+            bk.init_beacons(q_init)
+            assign = torch.empty(steps, per_step, dtype=torch.int32, device=dev)
+            if seq:
+                bk.update_seq(q_steps, assign)
+            else:
+                state = [x.cpu().numpy() for x in bk.state()]
+                for t in range(steps):
+                    bk.update(q_steps[t].unsqueeze(-2), assign[t])
+                    new = [x.cpu().numpy() for x in bk.state()]
+                    qb = synth.to_bits(q_steps[t]).reshape(wl.n_inst, wl.group, wl.head_dim)
+                    a_g = assign[t].view(wl.n_inst, wl.group).cpu().numpy()
+                    for e in range(wl.n_inst):
+                        pre = dict(cent=state[0][e].copy(), sums=state[1][e].copy(), counts=state[2][e].copy())
+                        post = dict(cent=new[0][e], sums=new[1][e], counts=new[2][e])
+                        ties += check_update(qb[e], pre, a_g[e], post, lib, tag=f"decode step {t} instance {e}")[0]
+                    state = new
+            bk.sync()
+            c, sm, n = bk.state()
+            outs.append((assign.cpu(), c.cpu().view(torch.int32), sm.cpu().view(torch.int64), n.cpu()))
+        finally:
+            bk.close()
+    for x, y in zip(*outs):
+        assert torch.equal(x, y), "bkv_update_beacons_seq differs from one bkv_update_beacons call per step"
+    return f"{steps} steps x {wl.n_inst} instances, oracle ties {ties}, seq call bit-identical"

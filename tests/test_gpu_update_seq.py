@@ -224,3 +224,12 @@ def test_seq_large_running_sums(case):
     q = q.view(steps, wl.n_layers, wl.batch, wl.n_q_heads, d).cuda().contiguous()
     a = _compare(wl, q, state=(cent.cuda(), sums.cuda(), counts.cuda()))
     assert (a >= 0).all()
+
+
+def test_seq_and_per_step_calls_against_the_oracle():
+    """Every per-step call checked against the fp64 oracle from the GPU's carried state, and the seq call
+    bit-identical to them (the check __graft_entry__.smoke() runs)."""
+    from paper_2609_04971_gb300.workloads import TINY
+    from tests import parity as P
+    P.smoke_decode_steps(TINY, steps=12, seed=3)
+    P.smoke_decode_steps(QWEN3_8B_TRACE.scaled(name="trace_1L_b2", n_layers=1, batch=2), steps=20, seed=4)
