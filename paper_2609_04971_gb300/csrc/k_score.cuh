@@ -244,6 +244,37 @@ __device__ __forceinline__ float tile_score(uint32_t taddr, const float* lse2, f
   return fmaxf(r0, r1);
 }
 
+// The N (<= 64) columns of this thread's lane of a slot, all loaded before one wait: the slot can be
+// released before the arithmetic.
+template <int N>
+__device__ __forceinline__ void tile_load(uint32_t taddr, float (&v)[64]) {
+  static_assert(N <= 64 && N % 16 == 0, "columns in loads of 32 and 16");
+#pragma unroll
+  for (int c0 = 0; c0 < N; c0 += 32) {
+    if (c0 + 32 <= N) {
+      tmem_ld32(taddr + c0, *reinterpret_cast<float(*)[32]>(v + c0));
+    } else {
+      tmem_ld16(taddr + c0, v + c0);
+    }
+  }
+  tmem_wait_ld();
+}
+
+// tile_score on loaded columns.
+template <int N>
+__device__ __forceinline__ float tile_score_regs(const float (&v)[64], const float* lse2, float sc) {
+  float r0 = -INFINITY, r1 = -INFINITY;
+#pragma unroll
+  for (int u = 0; u < N; u += 4) {
+    const float4 l = *reinterpret_cast<const float4*>(lse2 + u);
+    r0 = fmaxf(r0, fmaf(v[u], sc, -l.x));
+    r1 = fmaxf(r1, fmaf(v[u + 1], sc, -l.y));
+    r0 = fmaxf(r0, fmaf(v[u + 2], sc, -l.z));
+    r1 = fmaxf(r1, fmaf(v[u + 3], sc, -l.w));
+  }
+  return fmaxf(r0, r1);
+}
+
 // r = log2 of inv_m times the sum over the N columns of 2^(v * sc - lse2)
 // (mean aggregation; a column with lse2 = +inf adds nothing).
 template <int N>
@@ -719,13 +750,24 @@ __global__ void __launch_bounds__(kScThreads, 1)
         const int slot = rs + j < ring ? rs + j : rs + j - ring;
         float r = -INFINITY;
         const int key = k0 + j * kTile + key_row;
-        if (resident_ok)
-          r = (CAUSAL && k0 + j * kTile + kTile > win0)
-                  ? tile_agg_causal<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m, key, win0, thr)
-                  : tile_agg<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m);
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive_cnt(&slot_free[slot], 2);  // two arrivals: this warp stands for its pair
+        const bool window_tile = CAUSAL && k0 + j * kTile + kTile > win0;  // warp-uniform
+        if (!MEAN && N <= 64 && resident_ok && !window_tile) {
+          // max form: the columns into registers, the slot released, then the arithmetic
+          float v[64];
+          tile_load<N>(tmem + slot * N + lane_addr, v);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cnt(&slot_free[slot], 2);  // two arrivals: this warp stands for its pair
+          r = tile_score_regs<N>(v, lse2_sh, sc);
+        } else {
+          if (resident_ok)
+            r = window_tile
+                    ? tile_agg_causal<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m, key, win0, thr)
+                    : tile_agg<N, MEAN>(tmem + slot * N + lane_addr, lse2_sh, sc, inv_m);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cnt(&slot_free[slot], 2);
+        }
         if (resident_ok && key < k1) {
           if constexpr (COMBINE) r = fold_split<MEAN>(r_e[key], r);
           r_e[key] = r;
