@@ -92,16 +92,21 @@ def test_seq_equals_per_step_trace_shape():
 def test_seq_in_chunks_and_without_assignments():
     q_init, q = _steps(TRACE, 64, seed=32, zero_frac=0.05)
     _compare(TRACE, q, q_init, chunks=[1, 17, 30, 16])
+    _compare(TRACE, q, q_init, chunks=[1] * 64)
     _compare(TRACE, q, q_init, with_assign=False)
 
 
-@pytest.mark.parametrize("shape", ["d64_g8_nb4", "d128_g32_nb32", "d64_g1_nb8", "d128_g2_nb3"])
+@pytest.mark.parametrize("shape", ["d64_g8_nb4", "d128_g32_nb32", "d64_g1_nb8", "d128_g2_nb3", "d128_g5_nb16",
+                                   "d64_g5_nb2", "d128_g16_nb16"])
 def test_seq_equals_per_step_shapes(shape):
     kw = {
         "d64_g8_nb4": dict(head_dim=64, n_q_heads=16, n_kv_heads=2, n_beacons=4, n_clusters=4),
         "d128_g32_nb32": dict(head_dim=128, n_q_heads=64, n_kv_heads=2, n_beacons=32, n_clusters=24, window=2),
         "d64_g1_nb8": dict(head_dim=64, n_q_heads=8, n_kv_heads=8, n_beacons=8, n_clusters=8),
         "d128_g2_nb3": dict(head_dim=128, n_q_heads=8, n_kv_heads=4, n_beacons=3, n_clusters=3),
+        "d128_g5_nb16": dict(head_dim=128, n_q_heads=40, n_kv_heads=8, n_beacons=16, n_clusters=16),  # Qwen3-14B
+        "d64_g5_nb2": dict(head_dim=64, n_q_heads=10, n_kv_heads=2, n_beacons=2, n_clusters=2),
+        "d128_g16_nb16": dict(head_dim=128, n_q_heads=32, n_kv_heads=2, n_beacons=16, n_clusters=16, window=4),
     }[shape]
     wl = QWEN3_8B_TRACE.scaled(name=shape, n_layers=2, batch=2, **kw)
     q_init, q = _steps(wl, 45, seed=33, zero_frac=0.1)
