@@ -133,6 +133,18 @@ __device__ __forceinline__ void add_fixed(long long (&s)[kCols], const unsigned 
   }
 }
 
+// *cell += v on a shared int64 cell, as two 32-bit atomic additions: the low word's carry-out is
+// decided by the value that addition found, so concurrent additions still sum exactly (a 64-bit
+// shared-memory atomic addition is a compare-and-swap loop on this part).
+__device__ __forceinline__ void shared_add_i64(long long* cell, long long v) {
+  uint32_t* w = reinterpret_cast<uint32_t*>(cell);
+  const uint32_t lo = static_cast<uint32_t>(v);
+  const uint32_t old = atomicAdd(w, lo);
+  const uint32_t carry = old + lo < old ? 1u : 0u;
+  const uint32_t hi = static_cast<uint32_t>(static_cast<unsigned long long>(v) >> 32) + carry;
+  if (hi != 0u) atomicAdd(w + 1, hi);
+}
+
 // The same split for two adjacent columns at once, on packed f32x2 values
 // (low word: the first column), with Blackwell's paired fp32 adds.
 struct Parts2 {
@@ -450,8 +462,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
             add_fixed<kCols>(sr, qs + sw128_offset(r, col0, kQBox));
 #pragma unroll
             for (int c = 0; c < kCols; ++c)
-              atomicAdd(reinterpret_cast<unsigned long long*>(&acc_i[best_b * D + c * 32 + lane]),
-                        static_cast<unsigned long long>(sr[c]));
+              shared_add_i64(&acc_i[best_b * D + c * 32 + lane], sr[c]);
           }
         }
         named_barrier(1, 32 * kScreeners);
@@ -490,8 +501,7 @@ __global__ void __launch_bounds__(kUThreads, 1)
         auto flush = [&]() {
 #pragma unroll
           for (int c = 0; c < kCols; ++c)
-            atomicAdd(reinterpret_cast<unsigned long long*>(&acc_i[cur * D + c * 32 + lane]),
-                      static_cast<unsigned long long>(fixed40(parts2_get(s[c >> 1], c & 1))));
+            shared_add_i64(&acc_i[cur * D + c * 32 + lane], fixed40(parts2_get(s[c >> 1], c & 1)));
 #pragma unroll
           for (int h = 0; h < kPairs; ++h) s[h] = Parts2{0ull, 0ull, 0ull};
         };
