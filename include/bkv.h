@@ -63,6 +63,7 @@ extern "C" {
 #define BKV_ECUDA (-3)    /* a CUDA runtime / driver call failed                 */
 #define BKV_ETIMEOUT (-4) /* a bounded device-side wait expired (kernel aborted) */
 #define BKV_ESTATE (-5)   /* call order violated (e.g. update before init)       */
+#define BKV_EBOUNDS (-6)  /* a device-side bounds check failed (checked builds)  */
 
 /* bkv_config.flags (bitwise OR). */
 #define BKV_F_NONE 0u
@@ -288,7 +289,10 @@ int bkv_set_cfps_state(bkv_ctx* ctx, const void* buffers, const int32_t* sizes);
 /*
  * Waits for the context's stream, then reads and clears the device error
  * word.  Returns BKV_OK, BKV_ETIMEOUT (a kernel gave up a bounded wait and
- * its outputs are invalid) or BKV_ECUDA.
+ * its outputs are invalid), BKV_EINVAL (a per-instance length of
+ * bkv_compress_ragged outside 1..capacity), BKV_EBOUNDS (a library built with
+ * BKV_CHECKED found an index from device data out of range, skipped that
+ * access, and the outputs are invalid) or BKV_ECUDA.
  */
 int bkv_sync(bkv_ctx* ctx);
 
@@ -304,6 +308,38 @@ int bkv_sync(bkv_ctx* ctx);
  * a NULL context or a limit out of range; BKV_ECUDA on a CUDA error.
  */
 int bkv_selftest_wait_timeout(bkv_ctx* ctx, int64_t limit_ns);
+
+/*
+ * Checked builds (diagnostic; no counterpart in the paper).  A library
+ * compiled with BKV_CHECKED defined checks every index that its kernels take
+ * from device data before using it: work-list entries and per-instance
+ * lengths of a ragged compress, the positions and source rows of the kept
+ * set in the selection and gather, and the stored Continual FPS buffer
+ * sizes.  A failing check records BKV_EBOUNDS in the device error word (see
+ * bkv_sync) and the access is skipped or redirected in range; nothing traps.
+ * The default build compiles the checks out.
+ *
+ * bkv_checked_build returns 1 for a library built with BKV_CHECKED, else 0.
+ * bkv_selftest_bounds, after a bkv_sync of earlier work, launches one kernel
+ * that makes a checked store one past the logical end of a shared-memory
+ * array twice that long (so the store stays in memory the kernel owns with
+ * or without checks) and returns what bkv_sync then reports: BKV_EBOUNDS in
+ * a checked build, BKV_OK in the default one, with the error word cleared
+ * and the context usable either way.
+ */
+int bkv_checked_build(void);
+int bkv_selftest_bounds(bkv_ctx* ctx);
+
+/*
+ * Allocation-failure hook (test diagnostic).  With nth > 0, the nth device
+ * or pinned host allocation that later bkv_create calls attempt (counted
+ * from this call, across contexts) fails as if memory ran out, without
+ * allocating: that bkv_create releases what it had allocated, leaves *out
+ * NULL and returns BKV_ENOMEM.  The hook disarms itself after that one
+ * failure; nth = 0 disarms it.  Not thread-safe with concurrent bkv_create
+ * calls.  Returns BKV_OK, or BKV_EINVAL for nth < 0.
+ */
+int bkv_debug_fail_alloc(int32_t nth);
 
 /*
  * Per-kernel timing (tracing).  While enabled, every kernel launch made by
@@ -346,7 +382,8 @@ int bkv_profile_read(bkv_ctx* ctx, double* ms, int64_t* launches, int32_t n_kern
  * 16) bytes plus the rotary table, each part rounded up to 256 bytes - is
  * rejected with BKV_EINVAL and a message.
  *   dev_status  device int32 or NULL: cleared by the call, set non-zero if a
- *               kernel's bounded wait expires (outputs are then invalid).
+ *               kernel's bounded wait expires or, in a checked build, a
+ *               device-side bounds check fails (outputs are then invalid).
  *   err_msg     host buffer of err_len bytes or NULL: reason of a failure.
  * The rotary table (rope_theta != 0) reaches the device inside the
  * parameters of small kernels on `stream`, 16 KB per launch: no copy from

@@ -22,6 +22,7 @@ BKV_ENOMEM = -2
 BKV_ECUDA = -3
 BKV_ETIMEOUT = -4
 BKV_ESTATE = -5
+BKV_EBOUNDS = -6
 
 KERNEL_NAMES = ("fps_init", "update", "qobs", "score", "select_gather", "keep_all", "cfps", "rope_stage")
 
@@ -54,12 +55,15 @@ _P = ctypes.c_void_p
 
 
 def load_library(path: str | None = None, build: bool = True):
-    """Load libbkv.so (building it in-tree first if it is missing or stale)."""
+    """Load libbkv.so (building it in-tree first if it is missing or stale).  With the environment
+    variable BKV_CHECKED=1 the process uses the bounds-checked flavour libbkv_checked.so instead."""
     global _lib
     with _lock:
         if _lib is not None and path is None:
             return _lib
-        p = path or (_build.build() if build else _build.LIB_PATH)
+        checked = os.environ.get("BKV_CHECKED") == "1"
+        default = _build.LIB_PATH_CHECKED if checked else _build.LIB_PATH
+        p = path or (_build.build(checked=checked) if build else default)
         if not os.path.exists(p):
             raise RuntimeError(f"libbkv.so not found at {p}; run __graft_entry__.build()")
         lib = ctypes.CDLL(p)
@@ -79,6 +83,9 @@ def load_library(path: str | None = None, build: bool = True):
             "bkv_set_cfps_state": (ctypes.c_int, [_P, _P, _P]),
             "bkv_sync": (ctypes.c_int, [_P]),
             "bkv_selftest_wait_timeout": (ctypes.c_int, [_P, ctypes.c_int64]),
+            "bkv_selftest_bounds": (ctypes.c_int, [_P]),
+            "bkv_checked_build": (ctypes.c_int, []),
+            "bkv_debug_fail_alloc": (ctypes.c_int, [ctypes.c_int32]),
             "bkv_compress_static": (ctypes.c_int, [ctypes.POINTER(BkvConfig), _P, _P, _P, _P, ctypes.c_int32,
                                                    ctypes.c_int32, ctypes.c_int64, _P, _P, _P, _P, _P, _P,
                                                    ctypes.c_char_p, ctypes.c_size_t]),
@@ -247,6 +254,24 @@ def bkv_selftest_wait_timeout(ctx, limit_ns: int) -> int:
     if rc not in (BKV_OK, BKV_ETIMEOUT):
         _check(rc, "bkv_selftest_wait_timeout", ctx)
     return rc
+
+
+def bkv_selftest_bounds(ctx) -> int:
+    """Runs one checked out-of-range store (see include/bkv.h) and returns the status code bkv_sync
+    reports for it: BKV_EBOUNDS in a checked build, BKV_OK otherwise; raises on other errors."""
+    rc = _l().bkv_selftest_bounds(ctx)
+    if rc not in (BKV_OK, BKV_EBOUNDS):
+        _check(rc, "bkv_selftest_bounds", ctx)
+    return rc
+
+
+def bkv_checked_build() -> bool:
+    return bool(_l().bkv_checked_build())
+
+
+def bkv_debug_fail_alloc(nth: int) -> None:
+    """Arms (nth > 0) or disarms (0) the allocation-failure hook of bkv_create (include/bkv.h)."""
+    _check(_l().bkv_debug_fail_alloc(int(nth)), "bkv_debug_fail_alloc")
 
 
 def bkv_profile_enable(ctx, on: bool = True) -> None:

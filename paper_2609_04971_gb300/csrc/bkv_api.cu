@@ -3,6 +3,7 @@
 // the rotary table, and kernel launches on the context's stream.
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -176,9 +177,29 @@ int validate_config(const bkv_config* cfg, std::string& why) {
   return BKV_OK;
 }
 
+// Allocation-failure hook (bkv_debug_fail_alloc): once armed with n > 0, the n-th device or pinned
+// host allocation that bkv_create attempts reports cudaErrorMemoryAllocation without allocating,
+// and the hook disarms itself.
+std::atomic<int> g_fail_nth{0};
+std::atomic<int> g_alloc_seen{0};
+
+bool fail_this_alloc() {
+  const int nth = g_fail_nth.load();
+  if (nth <= 0 || g_alloc_seen.fetch_add(1) + 1 != nth) return false;
+  g_fail_nth.store(0);
+  return true;
+}
+
 template <typename T>
 cudaError_t dmalloc(T** p, size_t n) {
+  if (fail_this_alloc()) return cudaErrorMemoryAllocation;
   return cudaMalloc(reinterpret_cast<void**>(p), sizeof(T) * (n ? n : 1));
+}
+
+template <typename T>
+cudaError_t hmalloc(T** p, size_t bytes) {
+  if (fail_this_alloc()) return cudaErrorMemoryAllocation;
+  return cudaMallocHost(reinterpret_cast<void**>(p), bytes);
 }
 
 void free_all(bkv_ctx* c) {
@@ -215,6 +236,13 @@ void free_all(bkv_ctx* c) {
 
 extern "C" {
 
+int bkv_debug_fail_alloc(int32_t nth) {
+  if (nth < 0) return BKV_EINVAL;
+  g_alloc_seen.store(0);
+  g_fail_nth.store(nth);
+  return BKV_OK;
+}
+
 const char* bkv_version(void) { return "bkv 0.1.0 (sm_103a, tcgen05)"; }
 
 const char* bkv_strerror(int code) {
@@ -225,6 +253,7 @@ const char* bkv_strerror(int code) {
     case BKV_ECUDA: return "CUDA error";
     case BKV_ETIMEOUT: return "device wait timed out; outputs are invalid";
     case BKV_ESTATE: return "beacon state not initialised";
+    case BKV_EBOUNDS: return "device-side bounds check failed (checked build); outputs are invalid";
     default: return "unknown error";
   }
 }
@@ -294,10 +323,10 @@ int bkv_create(const bkv_config* cfg, void* stream, bkv_ctx** out) {
   }
   const size_t rope_bytes = sizeof(double2) * (static_cast<size_t>(s.W + 1) * (s.d / 2) * 3 / 2 + 1);
   for (int i = 0; i < bkv_ctx::kRopeSlots; ++i) {
-    if ((e = cudaMallocHost(reinterpret_cast<void**>(&c->rope_pinned[i]), rope_bytes)) != cudaSuccess ||
+    if ((e = hmalloc(&c->rope_pinned[i], rope_bytes)) != cudaSuccess ||
         (e = cudaHostGetDevicePointer(&c->rope_mapped[i], c->rope_pinned[i], 0)) != cudaSuccess ||
         (e = cudaEventCreateWithFlags(&c->rope_ev[i], cudaEventDisableTiming)) != cudaSuccess ||
-        (e = cudaMallocHost(&c->rag_pinned[i], c->rag_bytes)) != cudaSuccess ||
+        (e = hmalloc(&c->rag_pinned[i], c->rag_bytes)) != cudaSuccess ||
         (e = cudaHostGetDevicePointer(&c->rag_mapped[i], c->rag_pinned[i], 0)) != cudaSuccess ||
         (e = cudaEventCreateWithFlags(&c->rag_ev[i], cudaEventDisableTiming)) != cudaSuccess) {
       const int code = (e == cudaErrorMemoryAllocation) ? BKV_ENOMEM : BKV_ECUDA;
@@ -410,6 +439,7 @@ int bkv_update_beacons(bkv_ctx* ctx, const void* q_new, int32_t n_new, int32_t* 
     ca.size = ctx->csize;
     ca.bcn = ctx->cent;
     ca.bcnt = ctx->counts;
+    ca.err = ctx->err;
     ProfScope ps(ctx, BKV_K_CFPS);
     cudaError_t e = bkv::launch_cfps(s.d, ca, ctx->stream);
     return e == cudaSuccess ? BKV_OK : cuda_fail(ctx, e, "continual FPS update launch");
@@ -527,6 +557,7 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
     ca.size = ctx->csize;
     ca.bcn = ctx->cent;
     ca.bcnt = ctx->counts;
+    ca.err = ctx->err;
     ca.mode = bkv::kCfpsBeacons;
     ProfScope ps(ctx, BKV_K_CFPS);
     e = bkv::launch_cfps(s.d, ca, ctx->stream);
@@ -535,7 +566,7 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
   {
     ProfScope ps(ctx, BKV_K_QOBS);
     e = bkv::launch_qobs(s, static_cast<const __nv_bfloat16*>(q_recent), ctx->cent, ctx->counts, ctx->rope, rotate,
-                         ctx->qobs, ctx->valid, ctx->stream);
+                         ctx->qobs, ctx->valid, ctx->err, ctx->stream);
   }
   if (e != cudaSuccess) return cuda_fail(ctx, e, "qobs launch");
 
@@ -571,7 +602,7 @@ int bkv_compress(bkv_ctx* ctx, void* K, void* V, int32_t L, int32_t budget, int6
   {
     ProfScope ps(ctx, BKV_K_SELECT_GATHER);
     e = bkv::launch_select_gather(s, ctx->rscore, L, budget, static_cast<__nv_bfloat16*>(K),
-                                  static_cast<__nv_bfloat16*>(V), kept_idx_out, ctx->stream);
+                                  static_cast<__nv_bfloat16*>(V), kept_idx_out, ctx->err, ctx->stream);
   }
   if (e != cudaSuccess) return cuda_fail(ctx, e, "select_gather launch");
   if (ctx->cfps) {  // after the eviction: buffer = FPS of (beacons, then the window queries)
@@ -663,6 +694,7 @@ int bkv_compress_ragged(bkv_ctx* ctx, void* K, void* V, const int32_t* L, int32_
     ca.size = ctx->csize;
     ca.bcn = ctx->cent;
     ca.bcnt = ctx->counts;
+    ca.err = ctx->err;
     ca.mode = bkv::kCfpsBeacons;
     ProfScope ps(ctx, BKV_K_CFPS);
     e = bkv::launch_cfps(s.d, ca, ctx->stream);
@@ -672,7 +704,8 @@ int bkv_compress_ragged(bkv_ctx* ctx, void* K, void* V, const int32_t* L, int32_
   {
     ProfScope ps(ctx, BKV_K_QOBS);
     e = bkv::launch_qobs_ragged(s, static_cast<const __nv_bfloat16*>(q_recent), ctx->cent, ctx->counts, rope_rows,
-                                ctx->rag_row, rotate, ctx->work, ctx->n_work, ctx->qobs, ctx->valid, ctx->stream);
+                                ctx->rag_row, rotate, ctx->work, ctx->n_work, ctx->qobs, ctx->valid, ctx->err,
+                                ctx->stream);
   }
   if (e != cudaSuccess) return cuda_fail(ctx, e, "qobs launch");
 
@@ -712,7 +745,7 @@ int bkv_compress_ragged(bkv_ctx* ctx, void* K, void* V, const int32_t* L, int32_
     ProfScope ps(ctx, BKV_K_SELECT_GATHER);
     e = bkv::launch_select_gather_ragged(s, ctx->rscore, L, ctx->work, ctx->n_work, budget,
                                          static_cast<__nv_bfloat16*>(K), static_cast<__nv_bfloat16*>(V), kept_idx_out,
-                                         ctx->stream);
+                                         ctx->err, ctx->stream);
   }
   if (e != cudaSuccess) return cuda_fail(ctx, e, "select_gather launch");
   if (ctx->cfps) {  // after the eviction, in the instances evicted from: buffer = FPS of (beacons, window)
@@ -827,6 +860,23 @@ int bkv_selftest_wait_timeout(bkv_ctx* ctx, int64_t limit_ns) {
   return bkv_sync(ctx);
 }
 
+int bkv_selftest_bounds(bkv_ctx* ctx) {
+  if (!ctx) return BKV_EINVAL;
+  int rc = bkv_sync(ctx);  // report earlier work first
+  if (rc != BKV_OK) return rc;
+  cudaError_t e = bkv::launch_selftest_bounds(ctx->err, ctx->stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "selftest launch");
+  return bkv_sync(ctx);
+}
+
+int bkv_checked_build(void) {
+#ifdef BKV_CHECKED
+  return 1;
+#else
+  return 0;
+#endif
+}
+
 int bkv_sync(bkv_ctx* ctx) {
   if (!ctx) return BKV_EINVAL;
   cudaError_t e = cudaStreamSynchronize(ctx->stream);
@@ -838,6 +888,8 @@ int bkv_sync(bkv_ctx* ctx) {
     cudaMemset(ctx->err, 0, sizeof(int));
     if (h == bkv::kDevBadLength)
       return fail(ctx, BKV_EINVAL, "a per-instance cache length was outside 1..capacity; that instance was left untouched");
+    if (h == bkv::kDevBounds)
+      return fail(ctx, BKV_EBOUNDS, "a device-side bounds check failed; the access was skipped and the outputs are invalid");
     return fail(ctx, BKV_ETIMEOUT, "device wait expired (code %d)", h);
   }
   return BKV_OK;

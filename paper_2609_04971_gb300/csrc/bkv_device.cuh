@@ -20,6 +20,7 @@ enum DevErr : int {
   kDevTimeoutCluster = 5,
   kDevTimeoutSelftest = 6,
   kDevBadLength = 7,  // a per-instance cache length outside 1..capacity (bkv_compress_ragged)
+  kDevBounds = 8,     // a device-side bounds check failed (builds with BKV_CHECKED only)
 };
 
 // Every spin-wait gives up after this long and reports a timeout.
@@ -33,6 +34,23 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
 
 __device__ __forceinline__ void record_error(int* err, int code) {
   if (err) atomicCAS(err, 0, code);
+}
+
+// Bounds check of an index that comes from device data (a work list, a stored size, a selection's
+// output): true when 0 <= i < n.  In a build with BKV_CHECKED defined a failing check records
+// kDevBounds in the error word and the caller skips or redirects the access; nothing traps.  In
+// the default build it is the constant true and costs nothing.
+__device__ __forceinline__ bool in_bounds(long long i, long long n, int* err) {
+#ifdef BKV_CHECKED
+  if (i >= 0 && i < n) return true;
+  record_error(err, kDevBounds);
+  return false;
+#else
+  (void)i;
+  (void)n;
+  (void)err;
+  return true;
+#endif
 }
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {

@@ -47,6 +47,7 @@ struct CfpsArgs {
   // <= cap were evicted from and merge; the others keep their buffers
   const int* Ls = nullptr;
   int budget = 0, cap = 0, group = 1;
+  int* err = nullptr;  // device error word (bounds checks of BKV_CHECKED builds)
 };
 cudaError_t launch_cfps(int d, const CfpsArgs& a, cudaStream_t st);
 // Buffers seeded with b_min fp32 rows per head (FPS picks of the prompt), size b_min.
@@ -82,12 +83,13 @@ cudaError_t launch_update_seq(const Shape& s, const __nv_bfloat16* q_steps, int 
 // device-mapped pinned host buffer, by a kernel on `st`.
 cudaError_t launch_rope_stage(const void* src, void* dst, size_t bytes, cudaStream_t st);
 cudaError_t launch_qobs(const Shape& s, const __nv_bfloat16* q_recent, const float* cent, const long long* counts,
-                        const double2* rope, int rotate, __nv_bfloat16* qobs, uint32_t* valid, cudaStream_t st);
+                        const double2* rope, int rotate, __nv_bfloat16* qobs, uint32_t* valid, int* err,
+                        cudaStream_t st);
 // Per-instance cache lengths (bkv_compress_ragged): the same build for the instances work[0 .. *n_work)
 // only, batch row b taking its own rotary table at rope + b * rope_row (double2 units).
 cudaError_t launch_qobs_ragged(const Shape& s, const __nv_bfloat16* q_recent, const float* cent,
                                const long long* counts, const double2* rope, size_t rope_row, int rotate,
-                               const int* work, const int* n_work, __nv_bfloat16* qobs, uint32_t* valid,
+                               const int* work, const int* n_work, __nv_bfloat16* qobs, uint32_t* valid, int* err,
                                cudaStream_t st);
 
 // ---- per-instance cache lengths (k_ragged.cu)
@@ -154,15 +156,18 @@ cudaError_t launch_score_causal_mean(const Shape& s, const CUtensorMap& kmap, co
                                      const CUtensorMap& qmap, const ScoreArgs& a, cudaStream_t st);
 
 cudaError_t launch_select_gather(const Shape& s, const float* r, int L, int budget, __nv_bfloat16* K,
-                                 __nv_bfloat16* V, int* kept, cudaStream_t st);
+                                 __nv_bfloat16* V, int* kept, int* err, cudaStream_t st);
 // Per-instance lengths: the instances work[0 .. *n_work), instance e with Ls[e] rows (at most cap).
 cudaError_t launch_select_gather_ragged(const Shape& s, const float* r, const int* Ls, const int* work,
                                         const int* n_work, int budget, __nv_bfloat16* K, __nv_bfloat16* V, int* kept,
-                                        cudaStream_t st);
+                                        int* err, cudaStream_t st);
 
 cudaError_t launch_keep_all(const Shape& s, int L, int budget, int* kept, cudaStream_t st);
 
 // ---- diagnostics (k_selftest.cu): a bounded wait that expires after limit_ns
 cudaError_t launch_selftest_wait(int* err, unsigned long long limit_ns, cudaStream_t st);
+// One checked access at an index one past the logical end of a buffer that is twice that long, so
+// that the access stays in memory this kernel owns whether or not bounds checks are compiled in.
+cudaError_t launch_selftest_bounds(int* err, cudaStream_t st);
 
 }  // namespace bkv

@@ -235,7 +235,8 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
     }
   }
   e = bkv::launch_qobs(s, static_cast<const __nv_bfloat16*>(q_recent), centroids,
-                       reinterpret_cast<const long long*>(counts), rope, rotate, qobs, valid, st);
+                       reinterpret_cast<const long long*>(counts), rope, rotate, qobs, valid,
+                       reinterpret_cast<int*>(dev_status), st);
   CUtensorMap kmap, kmap32;
   if (e == cudaSuccess && (!encode(&kmap, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 128) ||
                            !encode(&kmap32, K, static_cast<uint64_t>(s.n_inst) * s.cap, s.d, 32))) {
@@ -267,7 +268,7 @@ extern "C" int bkv_compress_static(const bkv_config* cfg, const float* centroids
   }
   if (e == cudaSuccess)
     e = bkv::launch_select_gather(s, rscore, L, budget, static_cast<__nv_bfloat16*>(K),
-                                  static_cast<__nv_bfloat16*>(V), kept_idx_out, st);
+                                  static_cast<__nv_bfloat16*>(V), kept_idx_out, reinterpret_cast<int*>(dev_status), st);
   if (e != cudaSuccess) {
     message(err_msg, err_len, cudaGetErrorString(e));
     return BKV_ECUDA;

@@ -294,6 +294,7 @@ __global__ void __launch_bounds__(32 * kHeadsPerCta, R == 16 ? 2 : 1) cfps_kerne
   // the rows to add, in order: update: the buffer's own rows (their cosines are rebuilt), then
   // the new queries; beacons: the buffer's rows; merge: this compress's beacons, then the window
   const int n_old = min(max(a.size[h], 0), a.b_max);
+  in_bounds(a.size[h], a.b_max, a.err);  // a stored size is 0 .. b_max - 1; the clamp above keeps accesses in range
   if (MODE == kCfpsUpdate && n_old + a.n_q < a.b_max) {
     // the buffer does not fill: the new queries are appended in order and nothing is compressed
     const int words = a.n_q * D / 2;  // 32-bit words of the new rows

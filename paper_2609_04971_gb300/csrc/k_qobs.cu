@@ -60,11 +60,12 @@ __global__ void __launch_bounds__(kQobsThreads) qobs_kernel(Shape s, const __nv_
                                                              int rotate, const int* __restrict__ work,
                                                              const int* __restrict__ n_work,
                                                              __nv_bfloat16* __restrict__ qobs,
-                                                             uint32_t* __restrict__ valid) {
+                                                             uint32_t* __restrict__ valid, int* err) {
   int e = blockIdx.x;
   if (work) {
     if (e >= *n_work) return;  // whole block
     e = work[e];
+    if (!in_bounds(e, s.n_inst, err)) return;  // whole block: every thread read the same entry
   }
   const int d = s.d, h = d / 2, h4 = h / 4;
   const int GW = s.G * s.W;
@@ -141,18 +142,19 @@ cudaError_t launch_rope_stage(const void* src, void* dst, size_t bytes, cudaStre
 }
 
 cudaError_t launch_qobs(const Shape& s, const __nv_bfloat16* q_recent, const float* cent, const long long* counts,
-                        const double2* rope, int rotate, __nv_bfloat16* qobs, uint32_t* valid, cudaStream_t st) {
+                        const double2* rope, int rotate, __nv_bfloat16* qobs, uint32_t* valid, int* err,
+                        cudaStream_t st) {
   qobs_kernel<<<s.n_inst, kQobsThreads, 0, st>>>(s, q_recent, cent, counts, rope, 0, rotate, nullptr, nullptr, qobs,
-                                                 valid);
+                                                 valid, err);
   return cudaGetLastError();
 }
 
 cudaError_t launch_qobs_ragged(const Shape& s, const __nv_bfloat16* q_recent, const float* cent,
                                const long long* counts, const double2* rope, size_t rope_row, int rotate,
-                               const int* work, const int* n_work, __nv_bfloat16* qobs, uint32_t* valid,
+                               const int* work, const int* n_work, __nv_bfloat16* qobs, uint32_t* valid, int* err,
                                cudaStream_t st) {
   qobs_kernel<<<s.n_inst, kQobsThreads, 0, st>>>(s, q_recent, cent, counts, rope, rope_row, rotate, work, n_work,
-                                                 qobs, valid);
+                                                 qobs, valid, err);
   return cudaGetLastError();
 }
 

@@ -133,8 +133,19 @@ __device__ __forceinline__ Geom inst_geom(int L, int crank, int csize, int slots
 
 // Instance of work item w and its number of keys: the compact list of a per-instance-length
 // compress, or every instance with the launch's L.
-__device__ __forceinline__ int item_inst(const ScoreArgs& a, int w) { return a.work ? a.work[w] : w; }
-__device__ __forceinline__ int inst_len(const ScoreArgs& a, int e) { return a.Ls ? a.Ls[e] : a.L; }
+// In a BKV_CHECKED build an entry outside 0 .. n_inst - 1 is recorded and replaced by instance 0, and a
+// length outside 1 .. L (the launch's longest) by L, identically in every role, so that the roles still agree on
+// each instance's job list (the outputs are then flagged invalid by the error word).
+__device__ __forceinline__ int item_inst(const ScoreArgs& a, int w, int n_inst) {
+  if (!a.work) return w;
+  const int e = a.work[w];
+  return in_bounds(e, n_inst, a.err) ? e : 0;
+}
+__device__ __forceinline__ int inst_len(const ScoreArgs& a, int e) {
+  if (!a.Ls) return a.L;
+  const int L = a.Ls[e];
+  return in_bounds(L - 1, a.L, a.err) ? L : a.L;
+}
 
 // Wait used while draining after an abort: ignores the abort flag.
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* err) {
@@ -385,7 +396,8 @@ __global__ void __launch_bounds__(kScThreads, 1)
   const int crank = csize > 1 ? static_cast<int>(cluster_ctarank()) : 0;
   const int cluster_id = blockIdx.x / csize;
   const int n_clusters = gridDim.x / csize;
-  const int n_items = a.work ? *a.n_work : s.n_inst;  // instances to compress
+  int n_items = a.work ? *a.n_work : s.n_inst;  // instances to compress
+  if (!in_bounds(n_items, s.n_inst + 1, a.err)) n_items = 0;
   const int n_my = cluster_id < n_items ? (n_items - cluster_id + n_clusters - 1) / n_clusters : 0;
   const int ring = plan.slots;                       // resident slots, used in cyclic order
   const int str_slot = ring;                         // pass-1 streaming slots; +2, +3: pass-2 slots
@@ -448,7 +460,7 @@ __global__ void __launch_bounds__(kScThreads, 1)
       bool ok = true;
       int q_issued = 0;
       for (int i = 0; ok && i < n_my; ++i) {
-        const int e = item_inst(a, cluster_id + i * n_clusters);
+        const int e = item_inst(a, cluster_id + i * n_clusters, s.n_inst);
         const Geom gm = inst_geom(inst_len(a, e), crank, csize, ring);
         const int k0 = gm.k0, k1 = gm.k1, T = gm.T, R = gm.R, n_str = gm.n_str;
         const int qb = i & 1;
@@ -502,7 +514,7 @@ __global__ void __launch_bounds__(kScThreads, 1)
       int rs = 0, ru = 0;                        // next ring slot and its use count
       bool ok = true;
       for (int i = 0; ok && i < n_my; ++i) {
-        const int e = item_inst(a, cluster_id + i * n_clusters);
+        const int e = item_inst(a, cluster_id + i * n_clusters, s.n_inst);
         const Geom gm = inst_geom(inst_len(a, e), crank, csize, ring);
         const int T = gm.T, R = gm.R, n_str = gm.n_str;
         if (!mbar_wait(&qfull_bar[i & 1], (i >> 1) & 1, abort_flag, a.err, kDevTimeoutMma)) break;
@@ -572,13 +584,13 @@ __global__ void __launch_bounds__(kScThreads, 1)
     // and 96 read are all of the instance's words in some order (their total
     // is the valid count of the mean form).
     const int vw = COMBINE ? ((col0 >> 5) + (te >> 5)) & 3 : te >> 5;  // this thread's valid word
-    int e_next = n_my > 0 ? item_inst(a, cluster_id) : 0;
+    int e_next = n_my > 0 ? item_inst(a, cluster_id, s.n_inst) : 0;
     uint32_t vnext = (te < 128 && n_my > 0) ? ld_nc_u32(&a.valid[e_next * 4 + vw]) : 0u;
     for (int i = 0; i < n_my; ++i) {
       const int e = e_next;
       const uint32_t vword = vnext;
       if (i + 1 < n_my) {
-        e_next = item_inst(a, cluster_id + (i + 1) * n_clusters);
+        e_next = item_inst(a, cluster_id + (i + 1) * n_clusters, s.n_inst);
         if (te < 128) vnext = ld_nc_u32(&a.valid[e_next * 4 + vw]);
       }
       const int L_e = inst_len(a, e);

@@ -52,7 +52,7 @@ __global__ void __launch_bounds__(kSgThreads) select_gather_kernel(Shape s, cons
                                                                     int budget, __nv_bfloat16* K, __nv_bfloat16* V,
                                                                     int* kept, const int* __restrict__ Ls,
                                                                     const int* __restrict__ work,
-                                                                    const int* __restrict__ n_work) {
+                                                                    const int* __restrict__ n_work, int* err) {
   extern __shared__ __align__(16) uint32_t keys[];  // [L]
   __shared__ uint32_t hist[kSgWarps][256];
   __shared__ uint32_t tot[256];
@@ -64,7 +64,9 @@ __global__ void __launch_bounds__(kSgThreads) select_gather_kernel(Shape s, cons
   if (work) {
     if (e >= *n_work) return;  // whole block
     e = work[e];
+    if (!in_bounds(e, s.n_inst, err)) return;  // whole block: every thread read the same entries
     L = Ls[e];
+    if (!in_bounds(L - 1, s.cap, err)) return;
   }
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int c_lo = s.n_prefix, c_hi = L - s.W;
@@ -150,16 +152,18 @@ __global__ void __launch_bounds__(kSgThreads) select_gather_kernel(Shape s, cons
     const bool keep = in && (!cand || key > T || (tie && run_tie + tie_excl < k_ties));
     int keep_excl, keep_total;
     block_count_scan(keep, wsum, keep_excl, keep_total);
-    if (keep) {
+    if (keep && in_bounds(run_keep + keep_excl, budget, err)) {
       kept_e[run_keep + keep_excl] = j;
       kept_s[run_keep + keep_excl] = j;  // position <= j: that key has been read already
-    } else if (in) {
+    } else if (in && !keep) {
       atomicMin(&sh_first_evicted, j);
     }
     run_tie += tie_total;
     run_keep += keep_total;
   }
   __syncthreads();
+  // the selection keeps exactly `budget` rows; a checked build verifies it (block-uniform)
+  if (!in_bounds(run_keep - budget, 1, err) || !in_bounds(budget - run_keep, 1, err)) return;
 
   // ---------------------------------------------------------------- in-place gather
   constexpr int kVpr = D * 2 / 16;                 // 16-byte vectors per row of one tensor
@@ -178,7 +182,11 @@ __global__ void __launch_bounds__(kSgThreads) select_gather_kernel(Shape s, cons
 #pragma unroll
     for (int u = 0; u < kPer; ++u) {
       const int row = i0 + row0 + kRowsPerPass * u;
-      if (row < budget) R[u] = __ldcg(base_t + static_cast<size_t>(kept_s[row]) * kVpr);
+      if (row < budget) {
+        int src = kept_s[row];
+        if (!in_bounds(src - row, L - row, err)) src = row;  // kept rows satisfy row <= kept[row] < L
+        R[u] = __ldcg(base_t + static_cast<size_t>(src) * kVpr);
+      }
     }
   };
   auto store_chunk = [&](int i0, const uint4 (&R)[kPer]) {
@@ -210,40 +218,42 @@ __global__ void keep_all_kernel(int n_inst, int L, int budget, int* kept) {
 
 template <int D>
 cudaError_t launch_sg_d(const Shape& s, const float* r, int L, int budget, __nv_bfloat16* K, __nv_bfloat16* V,
-                        int* kept, cudaStream_t st) {
+                        int* kept, int* err, cudaStream_t st) {
   const size_t smem = sizeof(uint32_t) * static_cast<size_t>(L);
-  cudaError_t err = cudaFuncSetAttribute(select_gather_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-  if (err != cudaSuccess) return err;
-  select_gather_kernel<D><<<s.n_inst, kSgThreads, smem, st>>>(s, r, L, budget, K, V, kept, nullptr, nullptr, nullptr);
+  const cudaError_t ce = cudaFuncSetAttribute(select_gather_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              static_cast<int>(smem));
+  if (ce != cudaSuccess) return ce;
+  select_gather_kernel<D><<<s.n_inst, kSgThreads, smem, st>>>(s, r, L, budget, K, V, kept, nullptr, nullptr, nullptr,
+                                                              err);
   return cudaGetLastError();
 }
 
 // L_max sizes the shared-memory key array (every instance has at most that many rows).
 template <int D>
 cudaError_t launch_sg_ragged_d(const Shape& s, const float* r, const int* Ls, const int* work, const int* n_work,
-                               int L_max, int budget, __nv_bfloat16* K, __nv_bfloat16* V, int* kept, cudaStream_t st) {
+                               int L_max, int budget, __nv_bfloat16* K, __nv_bfloat16* V, int* kept, int* err,
+                               cudaStream_t st) {
   const size_t smem = sizeof(uint32_t) * static_cast<size_t>(L_max);
-  cudaError_t err = cudaFuncSetAttribute(select_gather_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-  if (err != cudaSuccess) return err;
-  select_gather_kernel<D><<<s.n_inst, kSgThreads, smem, st>>>(s, r, L_max, budget, K, V, kept, Ls, work, n_work);
+  const cudaError_t ce = cudaFuncSetAttribute(select_gather_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              static_cast<int>(smem));
+  if (ce != cudaSuccess) return ce;
+  select_gather_kernel<D><<<s.n_inst, kSgThreads, smem, st>>>(s, r, L_max, budget, K, V, kept, Ls, work, n_work, err);
   return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_select_gather(const Shape& s, const float* r, int L, int budget, __nv_bfloat16* K,
-                                 __nv_bfloat16* V, int* kept, cudaStream_t st) {
-  return s.d == 128 ? launch_sg_d<128>(s, r, L, budget, K, V, kept, st)
-                    : launch_sg_d<64>(s, r, L, budget, K, V, kept, st);
+                                 __nv_bfloat16* V, int* kept, int* err, cudaStream_t st) {
+  return s.d == 128 ? launch_sg_d<128>(s, r, L, budget, K, V, kept, err, st)
+                    : launch_sg_d<64>(s, r, L, budget, K, V, kept, err, st);
 }
 
 cudaError_t launch_select_gather_ragged(const Shape& s, const float* r, const int* Ls, const int* work,
                                         const int* n_work, int budget, __nv_bfloat16* K, __nv_bfloat16* V, int* kept,
-                                        cudaStream_t st) {
-  return s.d == 128 ? launch_sg_ragged_d<128>(s, r, Ls, work, n_work, s.cap, budget, K, V, kept, st)
-                    : launch_sg_ragged_d<64>(s, r, Ls, work, n_work, s.cap, budget, K, V, kept, st);
+                                        int* err, cudaStream_t st) {
+  return s.d == 128 ? launch_sg_ragged_d<128>(s, r, Ls, work, n_work, s.cap, budget, K, V, kept, err, st)
+                    : launch_sg_ragged_d<64>(s, r, Ls, work, n_work, s.cap, budget, K, V, kept, err, st);
 }
 
 cudaError_t launch_keep_all(const Shape& s, int L, int budget, int* kept, cudaStream_t st) {

@@ -224,3 +224,35 @@ def test_static_binding_rejects_tensors_of_the_wrong_size():
             call(**over)
     with pytest.raises(TypeError, match="CUDA tensor"):
         call()
+
+
+def test_allocation_failure_hook_reports_enomem(lib):
+    """bkv_debug_fail_alloc(1) makes bkv_create's first allocation fail before anything is allocated:
+    the call returns BKV_ENOMEM with *out NULL, and the hook then disarms itself (the next create fails
+    otherwise on a machine without a GPU, or succeeds on one).  Negative arguments are rejected."""
+    cfg = bkv.BkvConfig(1, 1, 4, 2, 64, 4, 8, 0, 1088, 1e4, 0)
+    out = ctypes.c_void_p()
+    assert lib.bkv_debug_fail_alloc(-1) == bkv.BKV_EINVAL
+    try:
+        assert lib.bkv_debug_fail_alloc(1) == bkv.BKV_OK
+        assert lib.bkv_create(ctypes.byref(cfg), None, ctypes.byref(out)) == bkv.BKV_ENOMEM
+        assert not out.value
+        rc = lib.bkv_create(ctypes.byref(cfg), None, ctypes.byref(out))
+        assert rc != bkv.BKV_ENOMEM
+        if rc == bkv.BKV_OK:
+            lib.bkv_destroy(out)
+    finally:
+        lib.bkv_debug_fail_alloc(0)
+
+
+def test_checked_flavour_builds_and_exports_the_same_symbols(lib):
+    """The BKV_CHECKED flavour (device-side bounds checks compiled in) builds from the same sources,
+    exports every declared symbol and says which flavour it is."""
+    path = _build.build(checked=True)
+    assert path == _build.LIB_PATH_CHECKED != _build.LIB_PATH
+    raw = ctypes.CDLL(path)
+    missing = [n for n in _declared() if not hasattr(raw, n)]
+    assert not missing, f"declared but not exported by the checked flavour: {missing}"
+    assert raw.bkv_checked_build() == 1
+    assert lib.bkv_checked_build() == 0
+    assert "bounds" in bkv.bkv_strerror(bkv.BKV_EBOUNDS)
