@@ -731,7 +731,7 @@ def trace_bench(args, wl, job, cfps: bool, steps: int) -> dict:
     total_ms = max_over_ranks(upd_ms + sum(cmp_ms), world, dev)
 
     tokens = len(sched) * wl.n_inst * cap * world
-    # Two accountings of the updates' bytes.  The survey's (the contract): every decode step's update
+    # Two accountings of the updates' bytes.  Per step (step_roofline): every decode step's update
     # reads its queries and all centroids and writes the touched centroids.  The strict one: what the
     # update calls made need at least (a seq call reads the centroids once and writes the touched ones
     # once); the kernel table uses it.
