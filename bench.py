@@ -6,9 +6,9 @@ one compression of every (layer, batch row, KV head) cache from L = 4224 to a
 budget of 4096 rows, on the Qwen3-4B shape (36 layers, batch 16, 32 query / 8
 KV heads, head_dim 128, 8 beacons, 8-query recent window): 4608 instances.
 
-Between timed steps (outside the timed events) the 128 rows evicted by the
-previous compress are refilled with "new tokens", as a decode loop would, and
-L2 is flushed by writing 256 MB; the K/V working set (10 GB) exceeds L2 anyway.
+Between timed steps (outside the timed events) K and V are restored to the
+step's starting cache, so that every step compresses the same cache, and L2 is
+flushed by writing 256 MB; the K/V working set (10 GB) exceeds L2 anyway.
 Every step is bracketed by CUDA events on the stream the library launches on.
 
     python bench.py [--gpus N --steps K --warmup W] [--impl reference]
@@ -419,8 +419,10 @@ def step_bench(args, wl, job, cfps: bool, steps: int, warmup: int, with_e2e: boo
     inp = synth.step_inputs(wl, rank_seed(args.seed, job.rank), dev)
     K, V = inp["K"], inp["V"]
     L, budget = wl.L, wl.budget
-    new_k = K[:, :, :, budget:L].clone()      # "new tokens" written back after every compress
-    new_v = V[:, :, :, budget:L].clone()
+    # every step compresses the same cache: K and V are restored before each step (outside the timed
+    # region).  Refilling only the evicted rows lets the cache drift: the rows before the first evicted
+    # one, which the gather leaves in place, grew from 1 % to 11 % of the kept rows over 200 steps
+    K0, V0 = K.clone(), V.clone()
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     kept = torch.empty(wl.n_layers, wl.batch, wl.n_kv_heads, budget, dtype=torch.int32, device=dev)
     bk = bkv.BeaconKV.for_workload(wl, continual_fps=cfps)
@@ -429,8 +431,8 @@ def step_bench(args, wl, job, cfps: bool, steps: int, warmup: int, with_e2e: boo
 
     def prepare(i):
         if i > 0:
-            K[:, :, :, budget:L].copy_(new_k)
-            V[:, :, :, budget:L].copy_(new_v)
+            K.copy_(K0)
+            V.copy_(V0)
         flush.fill_(i & 0xFF)
 
     def step(i):
@@ -525,7 +527,7 @@ def step_bench(args, wl, job, cfps: bool, steps: int, warmup: int, with_e2e: boo
     # end to end through the public API with host buffers
     if with_e2e:
         out["e2e"] = e2e(bk, wl, inp, args, dev, world, job.barrier)
-    del new_k, new_v, flush
+    del K0, V0, flush
     if with_cpu:
         out["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds, args.seed)
     bk.close()
